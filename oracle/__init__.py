@@ -1,0 +1,24 @@
+"""CPU oracle for the paged 4-bit KV path (test infrastructure).
+
+Plain, slow, obviously correct NumPy code: fp32 IEEE emulation for the
+quantizer (the bit-exact contract) and fp64 for attention.  It shares no code
+with the CUDA library and imports nothing from the product package.
+
+Only the test suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import or run anything in this package.  The product path
+never calls it; there is no CPU fallback.
+
+Modules
+-------
+affine4     page-record layout, bf16 rounding, affine 4-bit group-64 quantizer,
+            nibble packing, dequantization, quantize-on-append.
+attention   paged decode attention (plain softmax definition), split partials
+            and their merge, causal prefill-chunk attention.
+checkpoint  page-gather checkpoint and its inverse (restore scatter).
+
+Parity status: every function here is pinned by the ``-m "not gpu"`` tests in
+``tests/test_oracle_*.py`` (closed forms, invariants, brute force on tiny
+inputs, library routines on special cases, hand-derived fixtures in
+``tests/golden/``).
+"""
+from . import affine4, attention, checkpoint  # noqa: F401
