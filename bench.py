@@ -1,0 +1,388 @@
+"""Benchmark: 4-bit paged decode attention at 256K context on GB300.
+
+Workload (default): the full-window single request -- 24 query / 4 KV heads,
+head_dim 256, 262,144 positions in 1,024 pages of 256 positions with a random
+physical page order, K/V drawn N(0,1) bf16 with 4 K channels per KV head
+scaled x20, quantized to affine 4-bit group 64 -- over a 64-layer stack of
+independent caches (19.3 GB of packed KV, far larger than L2, so no flush is
+needed between steps).
+
+One step = one decode token through the stack: per layer, quantize-append the
+token's K/V row at the last position (append, then attend), then paged decode
+attention with the split-K workspace (split kernel + merge kernel).
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+METRIC = "4-bit paged decode attention KV positions/s and HBM GB/s vs GB300 peak at 256K"
+UNIT = "positions/s"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except FileNotFoundError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[4:]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in loaded:
+            for n, flag in zip(names, r[3][1:]):
+                if flag.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in loaded),
+                "power_w_max": max(r[2] for r in loaded),
+                "samples": len(loaded), "reasons": sorted(reasons)}
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def build_stack(jf, synth, layers, seed, dev):
+    w = synth.WORKLOADS["full_window_256k"]
+    geo = w["geometry"]
+    ctx = w["context_lens"][0]
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    gcpu = synth.generator(seed)
+    pools, tables = [], []
+    req = torch.zeros(ctx, dtype=torch.int32, device=dev)
+    pos = torch.arange(ctx, dtype=torch.int32, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    chunk = 65536
+    for layer in range(layers):
+        pt, npages = synth.page_tables(gcpu, [ctx], geo.page_size)
+        pt = pt.to(dev)
+        chans = synth.outlier_channels(gcpu, geo.num_kv_heads, geo.head_dim).to(dev)
+        pool = jf.KVPool.allocate(npages, geo.page_size, geo.num_kv_heads, geo.head_dim,
+                                  device=dev, fill=None)
+        for s in range(0, ctx, chunk):
+            n = min(chunk, ctx - s)
+            k = torch.randn(n, geo.num_kv_heads, geo.head_dim, generator=g, device=dev)
+            v = torch.randn(n, geo.num_kv_heads, geo.head_dim, generator=g, device=dev)
+            for h in range(geo.num_kv_heads):
+                k[:, h, chans[h]] *= 20.0
+            jf.jf_kv_quantize_append(pool, pt, req[s:s + n], pos[s:s + n],
+                                     k.to(torch.bfloat16), v.to(torch.bfloat16), err)
+        pools.append(pool)
+        tables.append(pt)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, "append reported a device error"
+    return geo, ctx, pools, tables
+
+
+def run_ours(args, world, rank, local):
+    import paper_2609_17475_gb300 as jf
+    from paper_2609_17475_gb300 import synth
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    layers = args.layers
+    geo, ctx, pools, tables = build_stack(jf, synth, layers, 1000 + rank, dev)
+    Hq, Hkv, D = geo.num_q_heads, geo.num_kv_heads, geo.head_dim
+    splits = args.splits or jf.default_num_splits(1, Hkv)
+    scale = 1.0 / math.sqrt(D)
+    g = torch.Generator(device=dev)
+    g.manual_seed(77 + rank)
+    # per-step inputs: one query and one new K/V row per layer
+    q = torch.randn(layers, 1, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    knew = torch.randn(layers, 1, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    vnew = torch.randn(layers, 1, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    out = torch.empty(layers, 1, Hq, D, dtype=torch.bfloat16, device=dev)
+    ctx_t = torch.tensor([ctx], dtype=torch.int32, device=dev)
+    req1 = torch.zeros(1, dtype=torch.int32, device=dev)
+    pos1 = torch.tensor([ctx - 1], dtype=torch.int32, device=dev)
+    ws = jf.decode_workspace(1, Hq, Hkv, D, splits, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(qs=q, ks=knew, vs=vnew, outs=out):
+        for l in range(layers):
+            jf.jf_kv_quantize_append(pools[l], tables[l], req1, pos1, ks[l], vs[l], err,
+                                     stream=stream)
+            jf.jf_paged_decode_attn(pools[l], tables[l], ctx_t, qs[l], scale, outs[l], ws, splits,
+                                    stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            step()
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graph, stream=stream):
+            step()
+    stream.synchronize()
+
+    # ---- device-timed steps (inputs resident in HBM) ----
+    for _ in range(args.warmup):
+        graph.replay()
+    stream.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+        stream.synchronize()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+        torch.distributed.barrier()
+    clocks = clk.summary()
+
+    # ---- dominant call alone: decode (split + merge) per layer, CUDA events ----
+    reps = max(3, min(20, args.steps))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(reps * layers)]
+    with torch.cuda.stream(stream):
+        for r in range(reps):
+            for l in range(layers):
+                a, b = evs[r * layers + l]
+                a.record(stream)
+                jf.jf_paged_decode_attn(pools[l], tables[l], ctx_t, q[l], scale, out[l], ws,
+                                        splits, stream=stream)
+                b.record(stream)
+    stream.synchronize()
+    dts = [a.elapsed_time(b) for a, b in evs]
+    decode_ms = statistics.mean(dts)
+    app_ms = None
+
+    # ---- end-to-end through the public API with host buffers ----
+    qh = q.cpu().pin_memory()
+    kh = knew.cpu().pin_memory()
+    vh = vnew.cpu().pin_memory()
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    qd, kd, vd = torch.empty_like(q), torch.empty_like(knew), torch.empty_like(vnew)
+    e2e_steps = max(3, min(args.steps, 50))
+
+    def e2e_step():
+        qd.copy_(qh, non_blocking=True)
+        kd.copy_(kh, non_blocking=True)
+        vd.copy_(vh, non_blocking=True)
+        step(qd, kd, vd, out)
+        oh.copy_(out, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            e2e_step()
+        stream.synchronize()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(e2e_steps):
+            e2e_step()
+        f1.record(stream)
+    stream.synchronize()
+    e2e_ms = f0.elapsed_time(f1) / e2e_steps
+    h2d = qh.numel() * 2 + kh.numel() * 2 + vh.numel() * 2
+    d2h = oh.numel() * 2
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws) == 0, "device error flag set"
+
+    positions_per_step = ctx * layers
+    ms_per_step = ms / args.steps
+    value = positions_per_step * world / (ms_per_step / 1e3)
+    bytes_per_pos = 2 * Hkv * (D // 2 + 4 * (D // 64))
+    alg_bytes = ctx * bytes_per_pos + 2 * Hq * D * 2 + tables[0].numel() * 4 + 4
+    hbm, src = peaks()
+    achieved = alg_bytes / (decode_ms / 1e3) / 1e9
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u4/bf16 (fp16 MMA, fp32 softmax)",
+        "data": "synthetic: seeded N(0,1) bf16 K/V with x20 K outlier channels, affine 4-bit g64",
+        "config": {"workload": "full_window_256k", "num_q_heads": Hq, "num_kv_heads": Hkv,
+                   "head_dim": D, "page_size": geo.page_size, "context": ctx,
+                   "layers": layers, "num_splits": splits, "batch": 1,
+                   "l2": "inputs larger than L2 (64 independent 302 MB caches per step)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "step": "per layer: quantize-append 1 row + split-K decode + merge (CUDA graph)"},
+        "hbm_gbs_step": positions_per_step * bytes_per_pos / (ms_per_step / 1e3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "jf_paged_decode_attn (split + merge launches)",
+                     "achieved": achieved, "peak": hbm, "peak_source": src, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None,
+                     "alg_bytes_per_launch": alg_bytes, "avg_call_us": decode_ms * 1e3,
+                     "frac_of_8tbs": achieved / 8000.0},
+        "e2e": {"value": positions_per_step * world / (e2e_ms / 1e3), "unit": UNIT,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms},
+        "gpu_launches": args.steps * layers * 3,
+        "clocks": clocks,
+    }
+    if rank == 0 and args.cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(args)
+    return result
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (reference arm and cpu_baseline)
+# ---------------------------------------------------------------------------
+def cpu_baseline(args, sample_heads=1):
+    """Oracle decode of one layer's full 262,144-position window for
+    ``sample_heads`` KV head(s); scaled to positions/s of the full 4-head layer."""
+    import numpy as np
+
+    from oracle import affine4 as OA
+    from oracle import attention as OT
+    from paper_2609_17475_gb300 import synth
+
+    w = synth.WORKLOADS["full_window_256k"]
+    geo = w["geometry"]
+    ctx = w["context_lens"][0]
+    gen = synth.generator(w["seed"])
+    chans = synth.outlier_channels(gen, geo.num_kv_heads, geo.head_dim)
+    k, v = synth.kv_rows(gen, ctx, sample_heads, geo.head_dim, chans[:sample_heads])
+    pt, npages = synth.page_tables(gen, [ctx], geo.page_size)
+    q = synth.normal_bf16(gen, (1, geo.group * sample_heads, geo.head_dim))
+    req, pos = synth.append_rows_for([ctx])
+    bits = lambda t: t.contiguous().view(torch.int16).numpy().view(np.uint16)
+    L = OA.PoolLayout(sample_heads, geo.page_size, geo.head_dim)
+    pool = OA.new_pool(L, npages)
+    OA.append(pool, L, pt.numpy(), req.numpy(), pos.numpy(), bits(k), bits(v))
+    t0 = time.perf_counter()
+    OT.paged_decode(pool, L, pt.numpy(), [ctx], bits(q), 1 / math.sqrt(geo.head_dim))
+    dt = time.perf_counter() - t0
+    frac = sample_heads / geo.num_kv_heads
+    return {"value": ctx * frac / dt, "unit": UNIT, "cores": torch.get_num_threads(),
+            "kind": "oracle", "seconds": dt,
+            "sample": f"one layer, {ctx} positions, {sample_heads} of {geo.num_kv_heads} KV heads "
+                      f"({geo.group * sample_heads} query heads), NumPy fp64 paged_decode; "
+                      f"positions/s scaled to the full {geo.num_kv_heads}-head layer"}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return None
+    import numpy as np  # noqa: F401
+    samples = []
+    base = None
+    for _ in range(args.warmup):
+        pass
+    t0 = time.perf_counter()
+    for _ in range(max(1, min(args.steps, 3))):
+        base = cpu_baseline(args)
+        samples.append(base["seconds"])
+    sec = statistics.median(samples)
+    value = base["value"] if base else None
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": len(samples), "warmup": 0, "ms_per_step": sec * 1e3 * 4,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic: seeded N(0,1) bf16 K/V, affine 4-bit g64 (oracle's own quantizer)",
+            "config": {"workload": "full_window_256k", "num_q_heads": 24, "num_kv_heads": 4,
+                       "head_dim": 256, "page_size": 256, "context": 262144},
+            "impl": "reference", "cpu_baseline": base,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "wall_s": time.perf_counter() - t0}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--layers", type=int, default=64)
+    ap.add_argument("--splits", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    world, rank, local = dist_env()
+    if world > 1 and args.impl == "ours":
+        torch.distributed.init_process_group("nccl")
+    if args.impl == "reference":
+        res = run_reference(args, world, rank)
+    else:
+        res = run_ours(args, world, rank, local)
+    if rank == 0 and res is not None:
+        print(json.dumps(res))
+    if world > 1 and args.impl == "ours":
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,191 @@
+/*
+ * jfkv.h -- C ABI of the GB300 paged 4-bit KV library (libjfkv.so).
+ *
+ * The library implements the data-parallel hot path of KVExec (Sec. 3.1 and
+ * Sec. 3.4 of "JustFit: Just-in-Time State Management for Local LLM Serving"):
+ * attention that reads a paged, 4-bit quantized KV cache directly, with a
+ * temporary workspace whose size never depends on the history length, plus
+ * the quantize-on-append and page-gather checkpoint operations that produce
+ * and persist those pages.
+ *
+ * Conventions for every entry point
+ *   - All array pointers are DEVICE pointers owned by the caller.  The library
+ *     never allocates, frees or synchronizes; it only enqueues kernels on
+ *     `stream` (a cudaStream_t passed as void*, NULL = legacy default stream).
+ *   - Return value: JF_OK (0) or a negative JF_ERR_* code.  Arguments are
+ *     validated on the host before anything is launched; on an error nothing
+ *     is enqueued.  JF_ERR_CUDA means a launch was refused by the runtime.
+ *   - Inconsistencies only visible on the device (a page id outside the pool,
+ *     a position beyond the page table) never trap: the kernel skips the
+ *     affected work and ORs a JF_DEV_* bit into a device status word
+ *     (`err_flag`, or the first int32 of `workspace`), which the caller reads
+ *     after the stream completes.
+ *   - bf16 means IEEE bfloat16 bit patterns (uint16), row-major, contiguous.
+ *
+ * KV pool format (JF_FMT_AFFINE4_G64; the paper defines TQ4 for KV and only
+ * mentions affine Q4 groups for weights, so the affine group layout below is
+ * this library's reading):
+ *   page record = [K codes: Hkv x P x D/2 bytes][V codes: same]
+ *                 [K scale/bias: Hkv x P x D/64 x (bf16 scale, bf16 bias)]
+ *                 [V scale/bias: same]
+ *   Within a code row, element 2i is the low nibble of byte i (eight 4-bit
+ *   indices per little-endian 32-bit word, App. A.1 Table 3).  A 64-element
+ *   group reconstructs as x = code * scale + bias.
+ *   page_bytes = 2*Hkv*P*(D/2 + 4*D/64); for Hkv 4, P 256, D 256 that is
+ *   294,912 bytes, i.e. 1,152 bytes per position per layer (the affine-g64
+ *   analogue of Eq. 2's 16,640 bytes per position over 16 layers for TQ4).
+ */
+#ifndef JFKV_H
+#define JFKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes --------------------------------------------------- */
+#define JF_OK                       0
+#define JF_ERR_INVALID_ARG         (-1)
+#define JF_ERR_UNSUPPORTED         (-2)
+#define JF_ERR_WORKSPACE_TOO_SMALL (-3)
+#define JF_ERR_CUDA                (-4)
+
+/* ---- device status bits (ORed into err_flag / workspace word 0) ------- */
+#define JF_DEV_ERR_PAGE_ID    1   /* page id < 0 or >= num_pages          */
+#define JF_DEV_ERR_POSITION   2   /* position beyond the page-table row, or
+                                     a request index out of range          */
+#define JF_DEV_ERR_TIMEOUT    4   /* a bounded wait on a copy gave up      */
+
+/* ---- formats -------------------------------------------------------- */
+#define JF_FMT_AFFINE4_G64 0      /* implemented                            */
+#define JF_FMT_TQ4         1      /* reserved (Eq. 4 codec); unsupported    */
+
+typedef struct jf_kv_pool {
+  void*   base;          /* device pointer to num_pages page records,
+                            16-byte aligned                                */
+  int64_t num_pages;     /* >= 1                                           */
+  int32_t page_size;     /* P: 64, 128 or 256 positions                    */
+  int32_t num_kv_heads;  /* Hkv >= 1                                       */
+  int32_t head_dim;      /* D: 128 or 256                                  */
+  int32_t group_size;    /* must be 64                                     */
+  int32_t format;        /* JF_FMT_AFFINE4_G64                             */
+} jf_kv_pool;
+
+/* Bytes of one page record (0 if the geometry is unsupported). */
+size_t jf_kv_page_bytes(int32_t num_kv_heads, int32_t page_size, int32_t head_dim);
+
+/*
+ * Workspace bytes jf_paged_decode_attn needs for at most `num_splits`
+ * splits per (request, KV head): 256 + B*Hq*S*(4*D + 8) bytes.  The size
+ * depends on batch, heads, splits and head_dim only, never on the context
+ * length (Sec. 2, Eq. 3 is the paper's argument for bounding temporaries).
+ * Returns 0 for invalid arguments.
+ */
+size_t jf_attn_workspace_bytes(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,
+                               int32_t head_dim, int32_t num_splits);
+
+/* Workspace bytes jf_prefill_chunk_attn needs (a status word). */
+size_t jf_prefill_workspace_bytes(void);
+
+/*
+ * Quantize-on-append (Sec. 3.3 "pending cache writes"; Sec. 2 paged pool).
+ *
+ * For each row i < n_rows, the bf16 vectors k[i, h, :] and v[i, h, :]
+ * (layout [n_rows, Hkv, D]) are quantized per 64-element group --
+ *   bias  = group minimum (-0 stored as +0),
+ *   scale = bf16_rne(fp32(max - min) / 15)            (IEEE, no FMA),
+ *   code  = #{k in 0..14 : fp32(x - bias) / scale > k + 1/2}, 0 if scale == 0
+ *   (midpoint thresholds with strict >, App. A.1 Table 3) --
+ * and written to slot row_pos[i] % P of physical page
+ * page_table[row_req[i] * pt_stride + row_pos[i] / P].
+ *   page_table  int32 [num_requests, pt_stride]
+ *   row_req     int32 [n_rows], 0 <= row_req[i] < num_requests
+ *   row_pos     int32 [n_rows], 0 <= row_pos[i] < pt_stride * P
+ *   k, v        bf16 [n_rows, Hkv, D], 16-byte aligned
+ *   err_flag    device int32 or NULL; JF_DEV_* bits are ORed into it for
+ *               rows that were skipped.
+ * Rows must not target the same slot twice in one call (the result of such
+ * a call is one of the rows, unspecified which).  n_rows == 0 is a no-op.
+ */
+int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                          int32_t num_requests, const int32_t* row_req, const int32_t* row_pos,
+                          const void* k, const void* v, int32_t n_rows, int32_t* err_flag,
+                          void* stream);
+
+/*
+ * Paged decode attention, one query token per request (Sec. 3.1: the decode
+ * kernel reads compressed pages where they are used; Eq. 5 head grouping).
+ *
+ *   out[b, h, :] = sum_t softmax_t(softmax_scale * <q[b, h], K_t>) V_t
+ * over logical positions t < context_lens[b] of request b, with KV head
+ * floor(h / (Hq / Hkv)) and K_t, V_t reconstructed from the page named by
+ * page_table[b * pt_stride + t / P].  context_lens counts positions already
+ * appended, the current token included.  A zero context gives a zero output.
+ *
+ *   page_table    int32 [batch, pt_stride]
+ *   context_lens  int32 [batch], 0 <= ctx <= pt_stride * P
+ *   q             bf16 [batch, Hq, D];   out: bf16 [batch, Hq, D]
+ *   Hq % Hkv == 0 and Hq / Hkv <= 8.
+ *   workspace     device buffer of >= jf_attn_workspace_bytes(batch, Hq,
+ *                 Hkv, D, num_splits) bytes, 256-byte aligned.  Its first
+ *                 int32 is the device status word (JF_DEV_* bits, ORed);
+ *                 the caller zeroes it when it wants a fresh status.
+ *   num_splits    >= 1: maximum number of split-K partitions per (request,
+ *                 KV head).  Each partition keeps (max, sum, partial output)
+ *                 in the workspace; a second kernel merges them.
+ * Numerics: K codes and q enter fp16 tensor-core products with fp32
+ * accumulation (q must satisfy |q| < 65504); the softmax runs in fp32 with the
+ * maximum subtracted; probabilities scaled by the V group scale enter fp16
+ * products, so V group scales must stay below 65504.  Output rounded RNE.
+ */
+int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                         const int32_t* context_lens, int32_t batch, const void* q,
+                         int32_t num_q_heads, float softmax_scale, void* out, void* workspace,
+                         size_t workspace_bytes, int32_t num_splits, void* stream);
+
+/*
+ * Prefill-chunk attention for one request (Sec. 3.1 "decode and prefill need
+ * different kernels"; Eq. 5).  chunk_len queries q[i] at absolute positions
+ * q_start + i attend positions [0, q_start + i] (causal != 0) or
+ * [0, q_start + chunk_len) (causal == 0) of the request's cache, which must
+ * already hold the chunk's own rows (append, then attend).
+ *   page_table_row  int32 [>= ceil((q_start + chunk_len) / P)]
+ *   q, out          bf16 [chunk_len, Hq, D]
+ *   workspace       >= jf_prefill_workspace_bytes(); int32 status word.
+ */
+int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
+                          const void* q, int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
+                          float softmax_scale, int32_t causal, void* out, void* workspace,
+                          size_t workspace_bytes, void* stream);
+
+/*
+ * Page-gather checkpoint (Sec. 3.4: read the request's page runs in place and
+ * emit one packed stream).  dst[k * page_bytes .. (k+1) * page_bytes) =
+ * page record page_table_row[k] for k < num_pages, tail bytes included.
+ *   dst        device buffer, >= num_pages * page_bytes bytes, 16-byte aligned
+ *   err_flag   device int32 or NULL (JF_DEV_ERR_PAGE_ID for bad ids; the
+ *              record is left untouched in dst).
+ */
+int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
+                     void* dst, size_t dst_bytes, int32_t* err_flag, void* stream);
+
+/*
+ * Restore (Sec. 3.4: restoration writes packed runs into the existing pool):
+ * the inverse of jf_kv_checkpoint.  Page record page_table_row[k] of the pool
+ * = src[k * page_bytes ..).  Page ids must be distinct.
+ */
+int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
+                  const void* src, size_t src_bytes, int32_t* err_flag, void* stream);
+
+/* Human-readable name of a JF_* status code. */
+const char* jf_status_string(int status);
+
+/* Library version string. */
+const char* jf_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* JFKV_H */

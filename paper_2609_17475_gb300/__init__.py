@@ -1,0 +1,11 @@
+"""GB300-native paged 4-bit KV attention (the KVExec hot path of JustFit).
+
+The compute lives in libjfkv.so (hand-written sm_103a CUDA behind a C ABI,
+include/jfkv.h); ``binding`` marshals torch tensors into those calls.
+"""
+from .binding import (  # noqa: F401
+    KVPool, JfError, decode_workspace, default_num_splits, jf_attn_workspace_bytes,
+    jf_kv_checkpoint, jf_kv_page_bytes, jf_kv_quantize_append, jf_kv_restore,
+    jf_paged_decode_attn, jf_prefill_chunk_attn, jf_prefill_workspace_bytes, lib,
+    status_string, version, workspace_status,
+)

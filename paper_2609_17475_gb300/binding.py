@@ -1,0 +1,258 @@
+"""Thin Python binding over libjfkv.so (include/jfkv.h).
+
+Argument marshalling only: every step of the path runs in the library's CUDA
+kernels.  PyTorch supplies device memory and the current stream.  There is no
+CPU fallback: if the library is missing or a call fails, this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libjfkv.so")
+
+JF_OK = 0
+JF_ERR_INVALID_ARG = -1
+JF_ERR_UNSUPPORTED = -2
+JF_ERR_WORKSPACE_TOO_SMALL = -3
+JF_ERR_CUDA = -4
+JF_DEV_ERR_PAGE_ID = 1
+JF_DEV_ERR_POSITION = 2
+JF_DEV_ERR_TIMEOUT = 4
+JF_FMT_AFFINE4_G64 = 0
+JF_FMT_TQ4 = 1
+
+EXPORTS = [
+    "jf_kv_page_bytes", "jf_attn_workspace_bytes", "jf_prefill_workspace_bytes",
+    "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
+    "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
+]
+
+
+class JfError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {status} ({status_string(status)})")
+
+
+class _Pool(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_void_p), ("num_pages", ctypes.c_int64),
+                ("page_size", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("group_size", ctypes.c_int32),
+                ("format", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libjfkv.so (built in-tree by __graft_entry__.build())."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        P, I32, I64, SZ, F32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64,
+                                ctypes.c_size_t, ctypes.c_float)
+        PP = ctypes.POINTER(_Pool)
+        sig = {
+            "jf_kv_page_bytes": (SZ, [I32, I32, I32]),
+            "jf_attn_workspace_bytes": (SZ, [I32, I32, I32, I32, I32]),
+            "jf_prefill_workspace_bytes": (SZ, []),
+            "jf_kv_quantize_append": (ctypes.c_int, [PP, P, I32, I32, P, P, P, P, I32, P, P]),
+            "jf_paged_decode_attn": (ctypes.c_int, [PP, P, I32, P, I32, P, I32, F32, P, P, SZ,
+                                                    I32, P]),
+            "jf_prefill_chunk_attn": (ctypes.c_int, [PP, P, P, I32, I32, I32, F32, I32, P, P,
+                                                     SZ, P]),
+            "jf_kv_checkpoint": (ctypes.c_int, [PP, P, I32, P, SZ, P, P]),
+            "jf_kv_restore": (ctypes.c_int, [PP, P, I32, P, SZ, P, P]),
+            "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+            "jf_version": (ctypes.c_char_p, []),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().jf_status_string(int(status)).decode()
+
+
+def version() -> str:
+    return lib().jf_version().decode()
+
+
+def _check(fn: str, status: int) -> None:
+    if status != JF_OK:
+        raise JfError(fn, status)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _need(t: torch.Tensor, dtype, name: str) -> None:
+    if not isinstance(t, torch.Tensor) or t.dtype != dtype or not t.is_cuda or not t.is_contiguous():
+        raise TypeError(f"{name} must be a contiguous CUDA tensor of dtype {dtype}")
+
+
+@dataclasses.dataclass
+class KVPool:
+    """A paged 4-bit KV pool: ``data`` is a CUDA uint8 tensor [num_pages, page_bytes]."""
+    data: torch.Tensor
+    page_size: int
+    num_kv_heads: int
+    head_dim: int
+    group_size: int = 64
+    format: int = JF_FMT_AFFINE4_G64
+
+    @staticmethod
+    def allocate(num_pages: int, page_size: int, num_kv_heads: int, head_dim: int,
+                 device="cuda", fill: Optional[int] = 0) -> "KVPool":
+        pb = jf_kv_page_bytes(num_kv_heads, page_size, head_dim)
+        if pb == 0:
+            raise ValueError("unsupported pool geometry")
+        if fill is None:
+            data = torch.empty(num_pages, pb, dtype=torch.uint8, device=device)
+        else:
+            data = torch.full((num_pages, pb), fill, dtype=torch.uint8, device=device)
+        return KVPool(data, page_size, num_kv_heads, head_dim)
+
+    @property
+    def num_pages(self) -> int:
+        return self.data.shape[0]
+
+    @property
+    def page_bytes(self) -> int:
+        return self.data.shape[1]
+
+    def c_struct(self) -> _Pool:
+        return _Pool(self.data.data_ptr(), self.num_pages, self.page_size, self.num_kv_heads,
+                     self.head_dim, self.group_size, self.format)
+
+
+def jf_kv_page_bytes(num_kv_heads: int, page_size: int, head_dim: int) -> int:
+    return int(lib().jf_kv_page_bytes(num_kv_heads, page_size, head_dim))
+
+
+def jf_attn_workspace_bytes(batch: int, num_q_heads: int, num_kv_heads: int, head_dim: int,
+                            num_splits: int) -> int:
+    return int(lib().jf_attn_workspace_bytes(batch, num_q_heads, num_kv_heads, head_dim,
+                                             num_splits))
+
+
+def jf_prefill_workspace_bytes() -> int:
+    return int(lib().jf_prefill_workspace_bytes())
+
+
+def decode_workspace(batch, num_q_heads, num_kv_heads, head_dim, num_splits, device="cuda"):
+    n = jf_attn_workspace_bytes(batch, num_q_heads, num_kv_heads, head_dim, num_splits)
+    if n == 0:
+        raise ValueError("invalid workspace geometry")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def workspace_status(workspace: torch.Tensor) -> int:
+    """Device status word (JF_DEV_* bits) stored in the first 4 bytes."""
+    return int(workspace[:4].view(torch.int32).item())
+
+
+def jf_kv_quantize_append(pool: KVPool, page_table: torch.Tensor, row_req: torch.Tensor,
+                          row_pos: torch.Tensor, k: torch.Tensor, v: torch.Tensor,
+                          err_flag: Optional[torch.Tensor] = None, stream=None) -> None:
+    _need(page_table, torch.int32, "page_table")
+    _need(row_req, torch.int32, "row_req")
+    _need(row_pos, torch.int32, "row_pos")
+    _need(k, torch.bfloat16, "k")
+    _need(v, torch.bfloat16, "v")
+    n = row_req.numel()
+    if row_pos.numel() != n or k.shape != (n, pool.num_kv_heads, pool.head_dim) or v.shape != k.shape:
+        raise ValueError("shape mismatch")
+    if err_flag is not None:
+        _need(err_flag, torch.int32, "err_flag")
+    pt = page_table if page_table.dim() == 2 else page_table.view(1, -1)
+    st = lib().jf_kv_quantize_append(ctypes.byref(pool.c_struct()), _ptr(pt), pt.shape[1],
+                                      pt.shape[0], _ptr(row_req), _ptr(row_pos), _ptr(k), _ptr(v),
+                                      n, _ptr(err_flag), _stream(stream))
+    _check("jf_kv_quantize_append", st)
+
+
+def jf_paged_decode_attn(pool: KVPool, page_table: torch.Tensor, context_lens: torch.Tensor,
+                         q: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                         workspace: torch.Tensor, num_splits: int, stream=None) -> None:
+    _need(page_table, torch.int32, "page_table")
+    _need(context_lens, torch.int32, "context_lens")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    _need(workspace, torch.uint8, "workspace")
+    B, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim or page_table.shape[0] != B or context_lens.numel() != B:
+        raise ValueError("shape mismatch")
+    st = lib().jf_paged_decode_attn(ctypes.byref(pool.c_struct()), _ptr(page_table),
+                                     page_table.shape[1], _ptr(context_lens), B, _ptr(q), Hq,
+                                     float(softmax_scale), _ptr(out), _ptr(workspace),
+                                     workspace.numel(), int(num_splits), _stream(stream))
+    _check("jf_paged_decode_attn", st)
+
+
+def jf_prefill_chunk_attn(pool: KVPool, page_table_row: torch.Tensor, q: torch.Tensor,
+                          q_start: int, softmax_scale: float, causal: bool, out: torch.Tensor,
+                          workspace: torch.Tensor, stream=None) -> None:
+    _need(page_table_row, torch.int32, "page_table_row")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    _need(workspace, torch.uint8, "workspace")
+    C, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim:
+        raise ValueError("shape mismatch")
+    st = lib().jf_prefill_chunk_attn(ctypes.byref(pool.c_struct()), _ptr(page_table_row), _ptr(q),
+                                      int(q_start), C, Hq, float(softmax_scale), int(bool(causal)),
+                                      _ptr(out), _ptr(workspace), workspace.numel(),
+                                      _stream(stream))
+    _check("jf_prefill_chunk_attn", st)
+
+
+def jf_kv_checkpoint(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
+                     dst: torch.Tensor, err_flag: Optional[torch.Tensor] = None,
+                     stream=None) -> None:
+    _need(page_table_row, torch.int32, "page_table_row")
+    _need(dst, torch.uint8, "dst")
+    if err_flag is not None:
+        _need(err_flag, torch.int32, "err_flag")
+    st = lib().jf_kv_checkpoint(ctypes.byref(pool.c_struct()), _ptr(page_table_row),
+                                 int(num_pages), _ptr(dst), dst.numel(), _ptr(err_flag),
+                                 _stream(stream))
+    _check("jf_kv_checkpoint", st)
+
+
+def jf_kv_restore(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
+                  src: torch.Tensor, err_flag: Optional[torch.Tensor] = None,
+                  stream=None) -> None:
+    _need(page_table_row, torch.int32, "page_table_row")
+    _need(src, torch.uint8, "src")
+    if err_flag is not None:
+        _need(err_flag, torch.int32, "err_flag")
+    st = lib().jf_kv_restore(ctypes.byref(pool.c_struct()), _ptr(page_table_row), int(num_pages),
+                              _ptr(src), src.numel(), _ptr(err_flag), _stream(stream))
+    _check("jf_kv_restore", st)
+
+
+def default_num_splits(batch: int, num_kv_heads: int, device=None) -> int:
+    """Splits per (request, KV head) so the split grid fills the GPU twice over."""
+    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
+    target = 2 * props.multi_processor_count
+    return max(1, -(-target // (batch * num_kv_heads)))

@@ -1,0 +1,205 @@
+// extern "C" entry points of libjfkv.so: host-side validation, TMA tensor-map
+// construction and kernel dispatch.  See include/jfkv.h for the contract.
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace jfkv {
+int launch_append(const Geom&, const jf_kv_pool&, const int32_t*, int32_t, int32_t,
+                  const int32_t*, const int32_t*, const void*, const void*, int32_t, int32_t*,
+                  cudaStream_t);
+int launch_page_copy(const Geom&, const jf_kv_pool&, const int32_t*, int32_t, void*, int32_t*,
+                     bool, cudaStream_t);
+int launch_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*, int32_t,
+                  const int32_t*, int32_t, const void*, int32_t, float, void*, void*, int32_t,
+                  cudaStream_t);
+size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S);
+int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
+                   const void*, int32_t, int32_t, int32_t, float, int32_t, void*, void*,
+                   cudaStream_t);
+}  // namespace jfkv
+
+using namespace jfkv;
+
+namespace {
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int check_pool(const jf_kv_pool* pool) {
+  if (!pool || !pool->base) return JF_ERR_INVALID_ARG;
+  if (!aligned(pool->base, 16)) return JF_ERR_INVALID_ARG;
+  if (pool->num_pages < 1 || pool->num_kv_heads < 1) return JF_ERR_INVALID_ARG;
+  if (pool->format != JF_FMT_AFFINE4_G64) return JF_ERR_UNSUPPORTED;
+  if (pool->group_size != 64) return JF_ERR_UNSUPPORTED;
+  if (pool->head_dim != 128 && pool->head_dim != 256) return JF_ERR_UNSUPPORTED;
+  if (pool->page_size != 64 && pool->page_size != 128 && pool->page_size != 256)
+    return JF_ERR_UNSUPPORTED;
+  if (pool->num_kv_heads > 65535) return JF_ERR_UNSUPPORTED;
+  if (pool->num_pages > 0x7FFFFFFFLL) return JF_ERR_UNSUPPORTED;
+  return JF_OK;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+
+// 5-D map over the code rows of a pool: (byte in row, slot, KV head, K|V, page),
+// box = (row bytes, rows_per_box, 1, 1, 1), 128B (or 64B) swizzle.
+int make_codes_map(const Geom& g, void* base, int rows_per_box, CUtensorMap* map) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return JF_ERR_CUDA;
+  cuuint64_t dims[5] = {(cuuint64_t)g.CB, (cuuint64_t)g.P, (cuuint64_t)g.Hkv, 2,
+                        (cuuint64_t)g.num_pages};
+  cuuint64_t strides[4] = {(cuuint64_t)g.CB, (cuuint64_t)g.P * g.CB,
+                           (cuuint64_t)g.codes_region, (cuuint64_t)g.page_bytes};
+  cuuint32_t box[5] = {(cuuint32_t)g.CB, (cuuint32_t)rows_per_box, 1, 1, 1};
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  CUtensorMapSwizzle sw = g.CB == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 5, base, dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? JF_OK : JF_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t jf_kv_page_bytes(int32_t num_kv_heads, int32_t page_size, int32_t head_dim) {
+  if (num_kv_heads < 1 || page_size < 1 || (head_dim != 128 && head_dim != 256)) return 0;
+  jf_kv_pool p{};
+  p.num_pages = 1;
+  p.page_size = page_size;
+  p.num_kv_heads = num_kv_heads;
+  p.head_dim = head_dim;
+  return (size_t)make_geom(p).page_bytes;
+}
+
+size_t jf_attn_workspace_bytes(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,
+                               int32_t head_dim, int32_t num_splits) {
+  if (batch < 1 || num_q_heads < 1 || num_kv_heads < 1 || num_splits < 1) return 0;
+  if (num_q_heads % num_kv_heads) return 0;
+  if (head_dim != 128 && head_dim != 256) return 0;
+  return decode_workspace_bytes(batch, num_q_heads, head_dim, num_splits);
+}
+
+size_t jf_prefill_workspace_bytes(void) { return 256; }
+
+int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                          int32_t num_requests, const int32_t* row_req, const int32_t* row_pos,
+                          const void* k, const void* v, int32_t n_rows, int32_t* err_flag,
+                          void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (n_rows < 0 || pt_stride < 1 || num_requests < 1) return JF_ERR_INVALID_ARG;
+  if (n_rows == 0) return JF_OK;
+  if (!page_table || !row_req || !row_pos || !k || !v) return JF_ERR_INVALID_ARG;
+  if (!aligned(k, 16) || !aligned(v, 16)) return JF_ERR_INVALID_ARG;
+  const Geom g = make_geom(*pool);
+  return launch_append(g, *pool, page_table, pt_stride, num_requests, row_req, row_pos, k, v,
+                       n_rows, err_flag, static_cast<cudaStream_t>(stream));
+}
+
+int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                         const int32_t* context_lens, int32_t batch, const void* q,
+                         int32_t num_q_heads, float softmax_scale, void* out, void* workspace,
+                         size_t workspace_bytes, int32_t num_splits, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (!page_table || !context_lens || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
+  if (batch < 1 || batch > 65535 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
+  if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
+  if (num_q_heads / pool->num_kv_heads > 8) return JF_ERR_UNSUPPORTED;
+  if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
+  if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return JF_ERR_INVALID_ARG;
+  const size_t need = jf_attn_workspace_bytes(batch, num_q_heads, pool->num_kv_heads,
+                                              pool->head_dim, num_splits);
+  if (workspace_bytes < need) return JF_ERR_WORKSPACE_TOO_SMALL;
+  const Geom g = make_geom(*pool);
+  CUtensorMap tmap;
+  st = make_codes_map(g, pool->base, 32, &tmap);
+  if (st) return st;
+  return launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q,
+                       num_q_heads, softmax_scale, out, workspace, num_splits,
+                       static_cast<cudaStream_t>(stream));
+}
+
+int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row, const void* q,
+                          int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
+                          float softmax_scale, int32_t causal, void* out, void* workspace,
+                          size_t workspace_bytes, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (!page_table_row || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
+  if (q_start < 0 || chunk_len < 0 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
+  if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
+  if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
+  if (workspace_bytes < jf_prefill_workspace_bytes()) return JF_ERR_WORKSPACE_TOO_SMALL;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 16)) return JF_ERR_INVALID_ARG;
+  if ((int64_t)q_start + chunk_len > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
+  if (chunk_len == 0) return JF_OK;
+  const Geom g = make_geom(*pool);
+  CUtensorMap tmap;
+  st = make_codes_map(g, pool->base, 64, &tmap);
+  if (st) return st;
+  return launch_prefill(g, *pool, tmap, page_table_row, q, q_start, chunk_len, num_q_heads,
+                        softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
+}
+
+int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
+                     void* dst, size_t dst_bytes, int32_t* err_flag, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (num_pages < 0) return JF_ERR_INVALID_ARG;
+  if (num_pages == 0) return JF_OK;
+  if (!page_table_row || !dst || !aligned(dst, 16)) return JF_ERR_INVALID_ARG;
+  const Geom g = make_geom(*pool);
+  if (dst_bytes < (size_t)num_pages * (size_t)g.page_bytes) return JF_ERR_INVALID_ARG;
+  return launch_page_copy(g, *pool, page_table_row, num_pages, dst, err_flag, true,
+                          static_cast<cudaStream_t>(stream));
+}
+
+int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
+                  const void* src, size_t src_bytes, int32_t* err_flag, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (num_pages < 0) return JF_ERR_INVALID_ARG;
+  if (num_pages == 0) return JF_OK;
+  if (!page_table_row || !src || !aligned(src, 16)) return JF_ERR_INVALID_ARG;
+  const Geom g = make_geom(*pool);
+  if (src_bytes < (size_t)num_pages * (size_t)g.page_bytes) return JF_ERR_INVALID_ARG;
+  return launch_page_copy(g, *pool, page_table_row, num_pages, const_cast<void*>(src), err_flag,
+                          false, static_cast<cudaStream_t>(stream));
+}
+
+const char* jf_status_string(int status) {
+  switch (status) {
+    case JF_OK: return "JF_OK";
+    case JF_ERR_INVALID_ARG: return "JF_ERR_INVALID_ARG";
+    case JF_ERR_UNSUPPORTED: return "JF_ERR_UNSUPPORTED";
+    case JF_ERR_WORKSPACE_TOO_SMALL: return "JF_ERR_WORKSPACE_TOO_SMALL";
+    case JF_ERR_CUDA: return "JF_ERR_CUDA";
+    default: return "JF_ERR_UNKNOWN";
+  }
+}
+
+const char* jf_version(void) { return "jfkv 0.1 (sm_103a)"; }
+
+}  // extern "C"

@@ -1,0 +1,150 @@
+// Quantize-on-append: bf16 K/V rows -> affine 4-bit group-64 codes in their
+// page slots (Sec. 3.3 "pending cache writes"; Sec. 2 paged pool; App. A.1
+// Table 3 midpoint thresholds with strict >).
+//
+// One vector (row, KV head, K|V) of D bf16 elements is handled by D/8 lanes,
+// each loading 16 bytes (8 elements), so a warp reads 512 contiguous bytes at
+// D = 256 and writes one 128-byte code row plus four 4-byte scale/bias words.
+// A 64-element group spans 8 consecutive lanes; its min/max is reduced with
+// three xor-shuffles.  All arithmetic is IEEE fp32 with explicit rounding
+// intrinsics (no contraction) so the codes match the CPU oracle bit for bit.
+#include "common.cuh"
+
+namespace jfkv {
+
+struct AppendArgs {
+  uint8_t* pool;
+  int64_t num_pages;
+  int64_t page_bytes;
+  int64_t codes_region;
+  int64_t sb_region;
+  int32_t P;
+  int32_t Hkv;
+  const int32_t* page_table;
+  int32_t pt_stride;
+  int32_t num_requests;
+  const int32_t* row_req;
+  const int32_t* row_pos;
+  const uint16_t* k;
+  const uint16_t* v;
+  int32_t n_rows;
+  int32_t* err;
+};
+
+template <int D>
+__global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
+  constexpr int LPV = D / 8;        // lanes per vector
+  constexpr int VPW = 32 / LPV;     // vectors per warp
+  constexpr int CB = D / 2;
+  constexpr int SBB = D / 16;       // 4 bytes per 64-group
+  const int lane = threadIdx.x & 31;
+  const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int li = lane % LPV;
+  const int64_t vec = warp_id * VPW + lane / LPV;
+  const int64_t total = (int64_t)a.n_rows * a.Hkv * 2;
+  const bool active = vec < total;
+
+  int64_t row = 0;
+  int kind = 0, head = 0;
+  float x[8];
+  if (active) {
+    row = vec / (2 * a.Hkv);
+    const int rem = (int)(vec % (2 * a.Hkv));
+    kind = rem / a.Hkv;
+    head = rem % a.Hkv;
+    const uint16_t* src = (kind ? a.v : a.k) + (row * a.Hkv + head) * D + li * 8;
+    const uint4 w = *reinterpret_cast<const uint4*>(src);
+    x[0] = bf16lo_to_f32(w.x); x[1] = bf16hi_to_f32(w.x);
+    x[2] = bf16lo_to_f32(w.y); x[3] = bf16hi_to_f32(w.y);
+    x[4] = bf16lo_to_f32(w.z); x[5] = bf16hi_to_f32(w.z);
+    x[6] = bf16lo_to_f32(w.w); x[7] = bf16hi_to_f32(w.w);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) x[i] = 0.f;
+  }
+
+  // group min / max over 8 lanes x 8 elements (exact)
+  float mn = x[0], mx = x[0];
+#pragma unroll
+  for (int i = 1; i < 8; ++i) { mn = fminf(mn, x[i]); mx = fmaxf(mx, x[i]); }
+#pragma unroll
+  for (int o = 1; o < 8; o <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  if (!active) return;
+
+  const float bias = __fadd_rn(mn, 0.0f);                 // -0 -> +0
+  const float range = __fsub_rn(mx, mn);
+  const __nv_bfloat16 scale_h = __float2bfloat16_rn(__fdiv_rn(range, 15.0f));
+  const float scale = __bfloat162float(scale_h);
+  uint32_t word = 0;
+  if (scale != 0.0f) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float r = __fdiv_rn(__fsub_rn(x[i], bias), scale);
+      // code = number of thresholds k + 1/2 (k = 0..14) that r strictly exceeds
+      int c = (int)ceilf(__fsub_rn(r, 0.5f));
+      c = min(max(c, 0), 15);
+      word |= (uint32_t)c << (4 * i);
+    }
+  }
+
+  // destination slot
+  const int32_t req = a.row_req[row];
+  const int32_t pos = a.row_pos[row];
+  if (req < 0 || req >= a.num_requests || pos < 0 || pos / a.P >= a.pt_stride) {
+    if (li == 0) flag_error(a.err, JF_DEV_ERR_POSITION);
+    return;
+  }
+  const int32_t page = a.page_table[(int64_t)req * a.pt_stride + pos / a.P];
+  if (page < 0 || page >= a.num_pages) {
+    if (li == 0) flag_error(a.err, JF_DEV_ERR_PAGE_ID);
+    return;
+  }
+  const int slot = pos % a.P;
+  uint8_t* base = a.pool + (int64_t)page * a.page_bytes;
+  const int64_t vrow = (int64_t)head * a.P + slot;
+  *reinterpret_cast<uint32_t*>(base + kind * a.codes_region + vrow * CB + li * 4) = word;
+  if ((li & 7) == 0) {
+    const uint32_t sb = (uint32_t)__bfloat16_as_ushort(scale_h) |
+                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(bias)) << 16);
+    *reinterpret_cast<uint32_t*>(base + 2 * a.codes_region + kind * a.sb_region + vrow * SBB +
+                                 (li >> 3) * 4) = sb;
+  }
+}
+
+int launch_append(const Geom& g, const jf_kv_pool& pool, const int32_t* page_table,
+                  int32_t pt_stride, int32_t num_requests, const int32_t* row_req,
+                  const int32_t* row_pos, const void* k, const void* v, int32_t n_rows,
+                  int32_t* err, cudaStream_t stream) {
+  AppendArgs a;
+  a.pool = static_cast<uint8_t*>(pool.base);
+  a.num_pages = g.num_pages;
+  a.page_bytes = g.page_bytes;
+  a.codes_region = g.codes_region;
+  a.sb_region = g.sb_region;
+  a.P = g.P;
+  a.Hkv = g.Hkv;
+  a.page_table = page_table;
+  a.pt_stride = pt_stride;
+  a.num_requests = num_requests;
+  a.row_req = row_req;
+  a.row_pos = row_pos;
+  a.k = static_cast<const uint16_t*>(k);
+  a.v = static_cast<const uint16_t*>(v);
+  a.n_rows = n_rows;
+  a.err = err;
+  const int64_t vectors = (int64_t)n_rows * g.Hkv * 2;
+  const int vpw = 32 / (g.D / 8);
+  const int64_t warps = (vectors + vpw - 1) / vpw;
+  const int64_t blocks = (warps + 7) / 8;
+  if (blocks > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
+  if (g.D == 256)
+    append_kernel<256><<<(unsigned)blocks, 256, 0, stream>>>(a);
+  else
+    append_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(a);
+  return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
+}
+
+}  // namespace jfkv

@@ -1,0 +1,618 @@
+// Paged 4-bit decode attention with a fixed split-K workspace (Sec. 3.1:
+// decode reads the compressed pages where they are used; Sec. 2, Eq. 3: never
+// size temporaries by the history length; Eq. 5: contiguous GQA head groups).
+//
+// Kernel 1 (split phase).  CTA = (split s, KV head, request b), 4 warps.  The
+// split's 32-position chunks are dealt round-robin to the warps; each warp owns
+// a private ring of DSTAGES shared-memory stages that it refills itself with
+// TMA: a 5-D tiled copy (128-byte swizzle) for the K and V code rows of the
+// chunk and two 1-D bulk copies for their scale/bias words.
+//
+// Dequantization never leaves registers and never builds bf16 K/V:
+//  * A 4-bit code n placed in the low bits of an fp16 is the subnormal
+//    n * 2^-24 exactly (the hi nibble of a byte gives 16 n * 2^-24), so
+//    `w & 0x000F000F` turns two packed codes into an f16x2 MMA operand.
+//  * QK^T: A = K codes [16 positions x 16 d] (ldmatrix), B = q [16 d x 8 heads]
+//    (the G <= 8 heads of the KV head share every K fragment).  Each k-step
+//    stays inside one 64-element group, so a group's partial dot product
+//    acc_g = 2^-24 sum_d q_d n_d is kept apart and the affine fix-up is exact:
+//        s_t = sum_g scale_{t,g} 2^24 acc_g + bias_{t,g} sum_{d in g} q_d.
+//  * PV: A = V codes transposed [16 d x 16 positions] (ldmatrix.trans gives the
+//    position pairs), B = p_t * scale_{t,g} as f16 [16 positions x 8 heads]
+//    (the QK accumulator transposed with movmatrix); bias terms accumulate as
+//    sum_t bias_{t,g} p_t in fp32.
+//  * Online softmax in the log2 domain with warp-shuffle maxima; accumulators
+//    are rescaled only when a head's running maximum grows.
+// The four warps' states are combined in shared memory and written as one
+// split partial (m, l, O) to the workspace, or straight to the output when
+// num_splits == 1.
+//
+// Kernel 2 (merge).  One CTA per (request, query head) combines the partials:
+//   o = sum_s 2^{m_s - m*} O_s / sum_s 2^{m_s - m*} l_s.
+#include <cmath>
+#include <cfloat>
+
+#include "common.cuh"
+
+namespace jfkv {
+
+constexpr int DTOK = 32;      // positions per pipeline stage (one chunk)
+constexpr int DWARPS = 4;     // warps per split CTA
+constexpr int DSTAGES = 3;    // stages per warp
+constexpr int MIN_CPS = 16;   // minimum chunks per split (512 positions)
+
+struct DecodeArgs {
+  const uint8_t* pool;
+  int64_t num_pages;
+  int64_t page_bytes;
+  int64_t sb_base;     // offset of the K scale/bias region in a page record
+  int64_t sb_region;   // bytes of one scale/bias region (K or V)
+  int32_t P, Hkv, Hq, G;
+  const int32_t* page_table;
+  int32_t pt_stride;
+  const int32_t* ctx;
+  const uint16_t* q;
+  uint16_t* out;
+  float* part_ml;      // [B, Hq, S, 2]
+  float* part_o;       // [B, Hq, S, D]
+  int32_t* status;
+  int32_t num_splits;
+  float scale_log2;    // softmax_scale * log2(e)
+};
+
+__host__ __device__ inline void split_plan(int ctx, int num_splits, int& nch, int& cps,
+                                           int& nsplit) {
+  nch = (ctx + DTOK - 1) / DTOK;
+  if (nch <= 0) { nch = 0; cps = MIN_CPS; nsplit = 0; return; }
+  cps = (nch + num_splits - 1) / num_splits;
+  if (cps < MIN_CPS) cps = MIN_CPS;
+  nsplit = (nch + cps - 1) / cps;
+}
+
+__device__ __forceinline__ int checked_ctx(const DecodeArgs& a, int b) {
+  int ctx = a.ctx[b];
+  const int64_t cap = (int64_t)a.pt_stride * a.P;
+  if (ctx < 0 || ctx > cap) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) flag_error(a.status, JF_DEV_ERR_POSITION);
+    ctx = ctx < 0 ? 0 : (int)cap;
+  }
+  return ctx;
+}
+
+// Byte offset of 16-byte chunk `ch` of code row `t` inside a TMA-swizzled
+// stage buffer (128B swizzle for 128-byte rows, 64B swizzle for 64-byte rows).
+template <int CB>
+__device__ __forceinline__ uint32_t swz(int t, int ch) {
+  if constexpr (CB == 128)
+    return t * 128 + ((ch ^ (t & 7)) << 4);
+  else
+    return t * 64 + ((ch ^ ((t >> 1) & 3)) << 4);
+}
+
+__device__ __forceinline__ uint32_t nib0(uint32_t w) { return w & 0x000F000Fu; }
+__device__ __forceinline__ uint32_t nib1(uint32_t w) { return w & 0x00F000F0u; }
+__device__ __forceinline__ uint32_t nib2(uint32_t w) { return (w >> 8) & 0x000F000Fu; }
+__device__ __forceinline__ uint32_t nib3(uint32_t w) { return (w >> 8) & 0x00F000F0u; }
+
+template <int D>
+struct DecodeSmem {
+  static constexpr int CB = D / 2;
+  static constexpr int NG = D / 64;
+  static constexpr int SBB = 4 * NG;
+  static constexpr int CODE_BUF = DTOK * CB;
+  static constexpr int SB_BUF = DTOK * SBB;
+  static constexpr int NBUF = DWARPS * DSTAGES;
+  static constexpr int CODES_BYTES = NBUF * 2 * CODE_BUF;
+  static constexpr int SB_BYTES = NBUF * 2 * SB_BUF;
+  static constexpr int BAR_BYTES = NBUF * 8;
+  static constexpr int TOTAL = 1024 + CODES_BYTES + SB_BYTES + BAR_BYTES;
+  static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
+  static_assert(DWARPS * 8 * D * 4 <= CODES_BYTES, "combine buffer must fit");
+  static_assert(DWARPS * 8 * 2 * 4 <= SB_BYTES, "combine ml buffer must fit");
+};
+
+template <int D>
+__global__ void __launch_bounds__(DWARPS * 32, 2)
+decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
+  using L = DecodeSmem<D>;
+  constexpr int NG = L::NG;
+  constexpr int CB = L::CB;
+  constexpr int SBB = L::SBB;
+  constexpr float NEG_INF = -INFINITY;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* codes = smem;
+  uint8_t* sbuf = codes + L::CODES_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES);
+
+  const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = lane >> 2, c = lane & 3;
+  const bool direct = (a.num_splits == 1);
+
+  const int ctx = checked_ctx(a, b);
+  int nch, cps, nsplit;
+  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  if (split >= nsplit) {
+    if (direct && split == 0) {   // empty context: zero output
+      for (int i = threadIdx.x; i < a.G * D; i += blockDim.x)
+        a.out[((int64_t)b * a.Hq + kvh * a.G + i / D) * D + i % D] = 0;
+    }
+    return;
+  }
+  const int c_begin = split * cps;
+  const int c_end = min(c_begin + cps, nch);
+  const int my_n = (c_end - c_begin > warp) ? (c_end - c_begin - warp + DWARPS - 1) / DWARPS : 0;
+
+  if (threadIdx.x == 0) prefetch_tensormap(&tmap);
+  if (lane == 0) {
+    for (int s = 0; s < DSTAGES; ++s) mbar_init(&bars[warp * DSTAGES + s], 1);
+    fence_barrier_init();
+  }
+  __syncwarp();
+
+  // ---- query fragments (B operand of QK^T) ---------------------------------
+  const int hq0 = kvh * a.G;
+  const bool head_ok = r < a.G;
+  const uint16_t* qrow = a.q + ((int64_t)b * a.Hq + hq0 + (head_ok ? r : 0)) * D;
+  uint4 qlo[NG], qhi[NG];
+  float qmax = 0.f;
+#pragma unroll
+  for (int g = 0; g < NG; ++g) {
+    if (head_ok) {
+      qlo[g] = *reinterpret_cast<const uint4*>(qrow + 64 * g + 8 * c);
+      qhi[g] = *reinterpret_cast<const uint4*>(qrow + 64 * g + 32 + 8 * c);
+    } else {
+      qlo[g] = make_uint4(0, 0, 0, 0);
+      qhi[g] = make_uint4(0, 0, 0, 0);
+    }
+    const uint32_t ws[8] = {qlo[g].x, qlo[g].y, qlo[g].z, qlo[g].w,
+                            qhi[g].x, qhi[g].y, qhi[g].z, qhi[g].w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      qmax = fmaxf(qmax, fmaxf(fabsf(bf16lo_to_f32(ws[i])), fabsf(bf16hi_to_f32(ws[i]))));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) qmax = fmaxf(qmax, __shfl_xor_sync(0xffffffffu, qmax, o));
+  // keep |q| * 2^-qe < 2^14 so the fp16 operand cannot overflow
+  const int qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
+  const float qs = ldexpf(1.f, -qe);
+  const float qs16 = qs * 0.0625f;
+
+  uint32_t qf[NG][4][2];
+  float Qg[NG];
+#pragma unroll
+  for (int g = 0; g < NG; ++g) {
+    float e[16];
+    const uint32_t ws[8] = {qlo[g].x, qlo[g].y, qlo[g].z, qlo[g].w,
+                            qhi[g].x, qhi[g].y, qhi[g].z, qhi[g].w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) { e[2 * i] = bf16lo_to_f32(ws[i]); e[2 * i + 1] = bf16hi_to_f32(ws[i]); }
+    // word W covers d = base..base+7; nib0 -> (base, base+4), nib1 -> (base+1, base+5) x16,
+    // nib2 -> (base+2, base+6), nib3 -> (base+3, base+7) x16
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float* x = e + 8 * h;
+      qf[g][2 * h + 0][0] = pack_f16x2(x[0] * qs, x[4] * qs);
+      qf[g][2 * h + 0][1] = pack_f16x2(x[1] * qs16, x[5] * qs16);
+      qf[g][2 * h + 1][0] = pack_f16x2(x[2] * qs, x[6] * qs);
+      qf[g][2 * h + 1][1] = pack_f16x2(x[3] * qs16, x[7] * qs16);
+    }
+    float sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) sum += e[i];
+    sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+    sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+    Qg[g] = sum;
+  }
+  float Qh[NG][2];
+#pragma unroll
+  for (int g = 0; g < NG; ++g) {
+    Qh[g][0] = __shfl_sync(0xffffffffu, Qg[g], (2 * c) * 4);
+    Qh[g][1] = __shfl_sync(0xffffffffu, Qg[g], (2 * c + 1) * 4);
+  }
+  const float cA = a.scale_log2 * 16777216.f * ldexpf(1.f, qe);
+  const float cB = a.scale_log2;
+
+  // ---- TMA producer (lane 0 of each warp feeds its own ring) -------------
+  uint32_t valid = 0;
+  auto issue = [&](int it) {
+    const int s = it % DSTAGES;
+    int ok = 1;
+    if (lane == 0) {
+      const int ch = c_begin + warp + it * DWARPS;
+      const int tok0 = ch * DTOK;
+      const int pidx = tok0 / a.P, inp = tok0 % a.P;
+      uint64_t* bar = &bars[warp * DSTAGES + s];
+      int page = -1;
+      if (pidx < a.pt_stride) page = a.page_table[(int64_t)b * a.pt_stride + pidx];
+      if (page < 0 || page >= a.num_pages) {
+        flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+        ok = 0;
+        mbar_arrive(bar);
+      } else {
+        uint8_t* kc = codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF;
+        uint8_t* ks = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
+        const uint8_t* gsb = a.pool + (int64_t)page * a.page_bytes + a.sb_base +
+                             ((int64_t)kvh * a.P + inp) * SBB;
+        mbar_arrive_expect_tx(bar, L::STAGE_TX);
+        tma_load_5d(kc, &tmap, 0, inp, kvh, 0, page, bar);
+        tma_load_5d(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar);
+        bulk_g2s(ks, gsb, L::SB_BUF, bar);
+        bulk_g2s(ks + L::SB_BUF, gsb + a.sb_region, L::SB_BUF, bar);
+      }
+    }
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    valid = (valid & ~(1u << s)) | ((uint32_t)ok << s);
+  };
+
+  const int npro = my_n < DSTAGES ? my_n : DSTAGES;
+  for (int it = 0; it < npro; ++it) issue(it);
+
+  // ---- running state ---------------------------------------------------
+  float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
+  float O[NG][4][4];
+  float Bs[NG][2];
+#pragma unroll
+  for (int g = 0; g < NG; ++g) {
+    Bs[g][0] = Bs[g][1] = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) O[g][e][i] = 0.f;
+  }
+
+  // ldmatrix row address pieces: matrix m = lane>>3 -> (position half, chunk)
+  const int ld_t = (lane & 7) + 8 * ((lane >> 3) & 1);
+  const int ld_ch = lane >> 4;
+
+  int done = 0;
+  for (int it = 0; it < my_n; ++it) {
+    const int s = it % DSTAGES;
+    const uint32_t par = (it / DSTAGES) & 1;
+    if (!mbar_wait_bounded(&bars[warp * DSTAGES + s], par)) {
+      if (lane == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
+      break;
+    }
+    done = it + 1;
+    const bool ok = (valid >> s) & 1u;
+    const int tokbase = (c_begin + warp + it * DWARPS) * DTOK;
+    const uint32_t kc = smem_u32(codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF);
+    const uint32_t vc = kc + L::CODE_BUF;
+    const uint8_t* ksb = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
+    const uint8_t* vsb = ksb + L::SB_BUF;
+
+    float sc[2][4];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int ta = 16 * j + r, tb = ta + 8;
+      const bool va = ok && (tokbase + ta < ctx);
+      const bool vb = ok && (tokbase + tb < ctx);
+      float acc[NG][4];
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        uint32_t w0, w1, w2, w3;
+        ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + ld_t, 2 * g + ld_ch));
+        acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
+        mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), qf[g][0][0], qf[g][0][1]);
+        mma_f16(acc[g], nib2(w0), nib2(w1), nib3(w0), nib3(w1), qf[g][1][0], qf[g][1][1]);
+        mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), qf[g][2][0], qf[g][2][1]);
+        mma_f16(acc[g], nib2(w2), nib2(w3), nib3(w2), nib3(w3), qf[g][3][0], qf[g][3][1]);
+      }
+      uint32_t wa[NG], wb[NG];
+      if constexpr (NG == 4) {
+        const uint4 xa = *reinterpret_cast<const uint4*>(ksb + ta * SBB);
+        const uint4 xb = *reinterpret_cast<const uint4*>(ksb + tb * SBB);
+        wa[0] = xa.x; wa[1] = xa.y; wa[2] = xa.z; wa[3] = xa.w;
+        wb[0] = xb.x; wb[1] = xb.y; wb[2] = xb.z; wb[3] = xb.w;
+      } else {
+        const uint2 xa = *reinterpret_cast<const uint2*>(ksb + ta * SBB);
+        const uint2 xb = *reinterpret_cast<const uint2*>(ksb + tb * SBB);
+        wa[0] = xa.x; wa[1] = xa.y;
+        wb[0] = xb.x; wb[1] = xb.y;
+      }
+      float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        const float sa = bf16lo_to_f32(wa[g]), ba = bf16hi_to_f32(wa[g]);
+        const float sbv = bf16lo_to_f32(wb[g]), bbv = bf16hi_to_f32(wb[g]);
+        t1[0] = fmaf(sa, acc[g][0], t1[0]);
+        t1[1] = fmaf(sa, acc[g][1], t1[1]);
+        t1[2] = fmaf(sbv, acc[g][2], t1[2]);
+        t1[3] = fmaf(sbv, acc[g][3], t1[3]);
+        t2[0] = fmaf(ba, Qh[g][0], t2[0]);
+        t2[1] = fmaf(ba, Qh[g][1], t2[1]);
+        t2[2] = fmaf(bbv, Qh[g][0], t2[2]);
+        t2[3] = fmaf(bbv, Qh[g][1], t2[3]);
+      }
+      sc[j][0] = va ? fmaf(t1[0], cA, t2[0] * cB) : NEG_INF;
+      sc[j][1] = va ? fmaf(t1[1], cA, t2[1] * cB) : NEG_INF;
+      sc[j][2] = vb ? fmaf(t1[2], cA, t2[2] * cB) : NEG_INF;
+      sc[j][3] = vb ? fmaf(t1[3], cA, t2[3] * cB) : NEG_INF;
+    }
+
+    // ---- online softmax over the 32 positions of this chunk -------------
+    float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][2]), fmaxf(sc[1][0], sc[1][2]));
+    float mx1 = fmaxf(fmaxf(sc[0][1], sc[0][3]), fmaxf(sc[1][1], sc[1][3]));
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+    }
+    const float nm0 = fmaxf(m0, mx0), nm1 = fmaxf(m1, mx1);
+    if (__any_sync(0xffffffffu, (nm0 > m0) || (nm1 > m1))) {
+      const float f0 = (nm0 > m0) ? fast_exp2(m0 - nm0) : 1.f;
+      const float f1 = (nm1 > m1) ? fast_exp2(m1 - nm1) : 1.f;
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          O[g][e][0] *= f0; O[g][e][2] *= f0;
+          O[g][e][1] *= f1; O[g][e][3] *= f1;
+        }
+        Bs[g][0] *= f0;
+        Bs[g][1] *= f1;
+      }
+      l0 *= f0;
+      l1 *= f1;
+      m0 = nm0;
+      m1 = nm1;
+    }
+    float p[2][4];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - m0);
+      p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - m1);
+      p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - m0);
+      p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - m1);
+      l0 += p[j][0] + p[j][2];
+      l1 += p[j][1] + p[j][3];
+    }
+
+    // ---- PV ---------------------------------------------------------------
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const int ta = 16 * j + r, tb = ta + 8;
+      const bool va = ok && (tokbase + ta < ctx);
+      const bool vb = ok && (tokbase + tb < ctx);
+      uint32_t wa[NG], wb[NG];
+      if constexpr (NG == 4) {
+        const uint4 xa = *reinterpret_cast<const uint4*>(vsb + ta * SBB);
+        const uint4 xb = *reinterpret_cast<const uint4*>(vsb + tb * SBB);
+        wa[0] = xa.x; wa[1] = xa.y; wa[2] = xa.z; wa[3] = xa.w;
+        wb[0] = xb.x; wb[1] = xb.y; wb[2] = xb.z; wb[3] = xb.w;
+      } else {
+        const uint2 xa = *reinterpret_cast<const uint2*>(vsb + ta * SBB);
+        const uint2 xb = *reinterpret_cast<const uint2*>(vsb + tb * SBB);
+        wa[0] = xa.x; wa[1] = xa.y;
+        wb[0] = xb.x; wb[1] = xb.y;
+      }
+#pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        const float sva = va ? bf16lo_to_f32(wa[g]) : 0.f;
+        const float bva = va ? bf16hi_to_f32(wa[g]) : 0.f;
+        const float svb = vb ? bf16lo_to_f32(wb[g]) : 0.f;
+        const float bvb = vb ? bf16hi_to_f32(wb[g]) : 0.f;
+        Bs[g][0] = fmaf(bva, p[j][0], fmaf(bvb, p[j][2], Bs[g][0]));
+        Bs[g][1] = fmaf(bva, p[j][1], fmaf(bvb, p[j][3], Bs[g][1]));
+        const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
+        const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
+        uint32_t v0, v1, v2, v3;
+        ldsm_x4_t(v0, v1, v2, v3, vc + swz<CB>(16 * j + ld_t, 2 * g + ld_ch));
+        mma_f16(O[g][0], nib0(v0), nib0(v2), nib0(v1), nib0(v3), b0, b1);
+        mma_f16(O[g][1], nib1(v0), nib1(v2), nib1(v1), nib1(v3), b0, b1);
+        mma_f16(O[g][2], nib2(v0), nib2(v2), nib2(v1), nib2(v3), b0, b1);
+        mma_f16(O[g][3], nib3(v0), nib3(v2), nib3(v1), nib3(v3), b0, b1);
+      }
+    }
+
+    __syncwarp();
+    if (it + DSTAGES < my_n) {
+      fence_proxy_async_smem();
+      issue(it + DSTAGES);
+    }
+  }
+  if (done < my_n) {
+    // a wait gave up: give copies still in flight a bounded chance to land
+    for (int it = done; it < my_n && it < done + DSTAGES; ++it)
+      mbar_wait_bounded(&bars[warp * DSTAGES + it % DSTAGES], (it / DSTAGES) & 1, 1u << 16);
+  }
+
+  // ---- per-warp finalize ---------------------------------------------------
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      Bs[g][0] += __shfl_xor_sync(0xffffffffu, Bs[g][0], o);
+      Bs[g][1] += __shfl_xor_sync(0xffffffffu, Bs[g][1], o);
+    }
+  }
+  __syncthreads();   // every warp is past its last stage: reuse the rings
+  float* so = reinterpret_cast<float*>(codes);    // [DWARPS][8][D]
+  float* sml = reinterpret_cast<float*>(sbuf);    // [DWARPS][8][2]
+  {
+    float* w0 = so + (warp * 8 + 2 * c) * D;
+    float* w1 = w0 + D;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float fe = (e & 1) ? 1048576.f : 16777216.f;   // 2^24, or 2^24/16 for hi nibbles
+        const int d0 = 64 * g + 4 * r + e, d1 = d0 + 32;
+        w0[d0] = fmaf(O[g][e][0], fe, Bs[g][0]);
+        w1[d0] = fmaf(O[g][e][1], fe, Bs[g][1]);
+        w0[d1] = fmaf(O[g][e][2], fe, Bs[g][0]);
+        w1[d1] = fmaf(O[g][e][3], fe, Bs[g][1]);
+      }
+    }
+    if (r == 0) {
+      sml[(warp * 8 + 2 * c) * 2 + 0] = m0;
+      sml[(warp * 8 + 2 * c) * 2 + 1] = l0;
+      sml[(warp * 8 + 2 * c + 1) * 2 + 0] = m1;
+      sml[(warp * 8 + 2 * c + 1) * 2 + 1] = l1;
+    }
+  }
+  __syncthreads();
+
+  // ---- combine the warps of this CTA --------------------------------------
+  for (int idx = threadIdx.x; idx < a.G * D; idx += blockDim.x) {
+    const int h = idx / D, d = idx % D;
+    float M = NEG_INF;
+#pragma unroll
+    for (int w = 0; w < DWARPS; ++w) M = fmaxf(M, sml[(w * 8 + h) * 2]);
+    float Lsum = 0.f, Osum = 0.f;
+    if (M != NEG_INF) {
+#pragma unroll
+      for (int w = 0; w < DWARPS; ++w) {
+        const float mw = sml[(w * 8 + h) * 2];
+        if (mw != NEG_INF) {
+          const float f = fast_exp2(mw - M);
+          Lsum = fmaf(f, sml[(w * 8 + h) * 2 + 1], Lsum);
+          Osum = fmaf(f, so[(w * 8 + h) * D + d], Osum);
+        }
+      }
+    }
+    const int hq = hq0 + h;
+    if (direct) {
+      a.out[((int64_t)b * a.Hq + hq) * D + d] =
+          __bfloat16_as_ushort(__float2bfloat16_rn(Lsum > 0.f ? Osum / Lsum : 0.f));
+    } else {
+      const int64_t row = ((int64_t)b * a.Hq + hq) * a.num_splits + split;
+      a.part_o[row * D + d] = Osum;
+      if (d == 0) {
+        a.part_ml[row * 2 + 0] = M;
+        a.part_ml[row * 2 + 1] = Lsum;
+      }
+    }
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(1024) decode_merge_kernel(const DecodeArgs a) {
+  constexpr int X = D / 4;
+  constexpr int Y = 1024 / X;
+  extern __shared__ float msm[];   // [2*S padded to 4] ml, then [Y][X] float4
+  const int hq = blockIdx.x, b = blockIdx.y;
+  const int tid = threadIdx.x;
+  const int ctx = checked_ctx(a, b);
+  int nch, cps, nsplit;
+  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D;
+  if (nsplit == 0) {
+    if (tid < D) orow[tid] = 0;
+    return;
+  }
+  const int64_t row0 = ((int64_t)b * a.Hq + hq) * a.num_splits;
+  for (int i = tid; i < 2 * nsplit; i += blockDim.x) msm[i] = a.part_ml[row0 * 2 + i];
+  __syncthreads();
+  float M = -INFINITY;
+  for (int s = 0; s < nsplit; ++s) M = fmaxf(M, msm[2 * s]);
+  const int x = tid % X, y = tid / X;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float Lsum = 0.f;
+  if (M != -INFINITY) {
+    for (int s = 0; s < nsplit; ++s) {
+      const float ms = msm[2 * s];
+      if (ms != -INFINITY) Lsum = fmaf(fast_exp2(ms - M), msm[2 * s + 1], Lsum);
+    }
+#pragma unroll 4
+    for (int s = y; s < nsplit; s += Y) {
+      const float ms = msm[2 * s];
+      if (ms == -INFINITY) continue;
+      const float f = fast_exp2(ms - M);
+      const float4 o = *reinterpret_cast<const float4*>(a.part_o + (row0 + s) * D + 4 * x);
+      acc.x = fmaf(f, o.x, acc.x);
+      acc.y = fmaf(f, o.y, acc.y);
+      acc.z = fmaf(f, o.z, acc.z);
+      acc.w = fmaf(f, o.w, acc.w);
+    }
+  }
+  float4* red = reinterpret_cast<float4*>(msm + ((2 * a.num_splits + 3) & ~3));
+  red[y * X + x] = acc;
+  __syncthreads();
+  if (y == 0) {
+    float4 t = red[x];
+    for (int yy = 1; yy < Y; ++yy) {
+      const float4 u = red[yy * X + x];
+      t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
+    }
+    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+    const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.x * inv)) |
+                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.y * inv)) << 16);
+    const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.z * inv)) |
+                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.w * inv)) << 16);
+    *reinterpret_cast<uint2*>(orow + 4 * x) = make_uint2(lo, hi);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S) {
+  const int64_t rows = B * Hq * S;
+  const int64_t ml = (rows * 8 + 255) / 256 * 256;
+  return (size_t)(256 + ml + rows * D * 4);
+}
+
+template <int D>
+static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
+                           cudaStream_t stream) {
+  using L = DecodeSmem<D>;
+  static bool attr_done = false;
+  if (!attr_done) {
+    if (cudaFuncSetAttribute(decode_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             L::TOTAL) != cudaSuccess)
+      return JF_ERR_CUDA;
+    attr_done = true;
+  }
+  dim3 grid((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
+  decode_split_kernel<D><<<grid, DWARPS * 32, L::TOTAL, stream>>>(tmap, a);
+  if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  if (a.num_splits > 1) {
+    const size_t smem = (size_t)((2 * a.num_splits + 3) & ~3) * 4 + 1024 * 16;
+    if (smem > 48 * 1024) {
+      if (cudaFuncSetAttribute(decode_merge_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)smem) != cudaSuccess)
+        return JF_ERR_CUDA;
+    }
+    decode_merge_kernel<D><<<dim3((unsigned)a.Hq, (unsigned)B), 1024, smem, stream>>>(a);
+    if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  }
+  return JF_OK;
+}
+
+int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
+                  const int32_t* page_table, int32_t pt_stride, const int32_t* context_lens,
+                  int32_t batch, const void* q, int32_t Hq, float softmax_scale, void* out,
+                  void* workspace, int32_t num_splits, cudaStream_t stream) {
+  DecodeArgs a;
+  a.pool = static_cast<const uint8_t*>(pool.base);
+  a.num_pages = g.num_pages;
+  a.page_bytes = g.page_bytes;
+  a.sb_base = 2 * g.codes_region;
+  a.sb_region = g.sb_region;
+  a.P = g.P;
+  a.Hkv = g.Hkv;
+  a.Hq = Hq;
+  a.G = Hq / g.Hkv;
+  a.page_table = page_table;
+  a.pt_stride = pt_stride;
+  a.ctx = context_lens;
+  a.q = static_cast<const uint16_t*>(q);
+  a.out = static_cast<uint16_t*>(out);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const int64_t rows = (int64_t)batch * Hq * num_splits;
+  a.status = reinterpret_cast<int32_t*>(ws);
+  a.part_ml = reinterpret_cast<float*>(ws + 256);
+  a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
+  a.num_splits = num_splits;
+  a.scale_log2 = softmax_scale * 1.4426950408889634f;
+  if (g.D == 256) return launch_decode_t<256>(tmap, a, batch, stream);
+  return launch_decode_t<128>(tmap, a, batch, stream);
+}
+
+}  // namespace jfkv

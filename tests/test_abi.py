@@ -1,0 +1,112 @@
+"""Host-only checks of the C ABI: the library loads, exports every symbol the
+header declares, and rejects bad arguments before launching anything (these
+calls never touch the GPU, so they run on CPU-only machines)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_17475_gb300 import binding as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "jfkv.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(jf_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_library_exports_every_declared_symbol():
+    L = B.lib()
+    names = _declared()
+    assert "jf_paged_decode_attn" in names and len(names) >= 10
+    for n in names:
+        assert hasattr(L, n), n
+    assert sorted(B.EXPORTS) == names
+
+
+def test_sizes():
+    assert B.jf_kv_page_bytes(4, 256, 256) == 294912
+    assert B.jf_kv_page_bytes(2, 256, 128) == 73728
+    assert B.jf_kv_page_bytes(2, 64, 128) == 18432
+    assert B.jf_kv_page_bytes(4, 256, 64) == 0
+    # fixed workspace: independent of context length, linear in splits
+    w1 = B.jf_attn_workspace_bytes(1, 24, 4, 256, 32)
+    w2 = B.jf_attn_workspace_bytes(1, 24, 4, 256, 64)
+    assert w1 >= 24 * 32 * (4 * 256 + 8)
+    assert w2 - w1 == 24 * 32 * 4 * 256 + (24 * 64 * 8 - 24 * 32 * 8)
+    assert B.jf_attn_workspace_bytes(2, 24, 5, 256, 4) == 0     # Hq % Hkv != 0
+    assert B.jf_attn_workspace_bytes(1, 8, 2, 96, 4) == 0        # unsupported head_dim
+    assert B.jf_prefill_workspace_bytes() >= 4
+    assert B.status_string(-3) == "JF_ERR_WORKSPACE_TOO_SMALL"
+    assert "sm_103a" in B.version()
+
+
+def _pool(**kw):
+    d = dict(base=0x10000, num_pages=8, page_size=256, num_kv_heads=2, head_dim=128,
+             group_size=64, format=0)
+    d.update(kw)
+    return B._Pool(**d)
+
+
+FAKE = ctypes.c_void_p(0x20000)   # aligned, never dereferenced: validation fails first
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(base=None), B.JF_ERR_INVALID_ARG),
+    (dict(base=0x10004), B.JF_ERR_INVALID_ARG),
+    (dict(head_dim=96), B.JF_ERR_UNSUPPORTED),
+    (dict(page_size=100), B.JF_ERR_UNSUPPORTED),
+    (dict(group_size=32), B.JF_ERR_UNSUPPORTED),
+    (dict(format=1), B.JF_ERR_UNSUPPORTED),
+    (dict(num_pages=0), B.JF_ERR_INVALID_ARG),
+])
+def test_decode_rejects_bad_pool(kw, expect):
+    p = _pool(**kw)
+    st = B.lib().jf_paged_decode_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 8, 0.1, FAKE,
+                                       FAKE, 1 << 20, 4, None)
+    assert st == expect
+
+
+def test_decode_rejects_bad_arguments():
+    p = _pool()
+    L = B.lib()
+    call = lambda **kw: L.jf_paged_decode_attn(
+        ctypes.byref(p), kw.get("pt", FAKE), 4, FAKE, kw.get("batch", 1), FAKE,
+        kw.get("hq", 8), kw.get("scale", 0.1), FAKE, kw.get("ws", FAKE),
+        kw.get("wsb", 1 << 20), kw.get("splits", 4), None)
+    assert call(pt=None) == B.JF_ERR_INVALID_ARG
+    assert call(hq=7) == B.JF_ERR_INVALID_ARG            # Hq % Hkv
+    assert call(hq=18) == B.JF_ERR_UNSUPPORTED           # G = 9 > 8
+    assert call(splits=0) == B.JF_ERR_INVALID_ARG
+    assert call(batch=0) == B.JF_ERR_INVALID_ARG
+    assert call(scale=float("nan")) == B.JF_ERR_INVALID_ARG
+    assert call(wsb=100) == B.JF_ERR_WORKSPACE_TOO_SMALL
+    assert call(ws=ctypes.c_void_p(0x20010)) == B.JF_ERR_INVALID_ARG   # not 256-aligned
+
+
+def test_append_checkpoint_prefill_reject_bad_arguments():
+    p = _pool()
+    L = B.lib()
+    assert L.jf_kv_quantize_append(ctypes.byref(p), FAKE, 4, 1, FAKE, FAKE, FAKE, FAKE, -1,
+                                   None, None) == B.JF_ERR_INVALID_ARG
+    assert L.jf_kv_quantize_append(ctypes.byref(p), FAKE, 4, 1, FAKE, FAKE, FAKE, FAKE, 0,
+                                   None, None) == B.JF_OK          # empty append: no-op
+    assert L.jf_kv_quantize_append(ctypes.byref(p), FAKE, 4, 1, FAKE, FAKE,
+                                   ctypes.c_void_p(0x20002), FAKE, 5, None,
+                                   None) == B.JF_ERR_INVALID_ARG  # misaligned k
+    pb = B.jf_kv_page_bytes(2, 256, 128)
+    assert L.jf_kv_checkpoint(ctypes.byref(p), FAKE, 3, FAKE, 3 * pb - 1, None,
+                              None) == B.JF_ERR_INVALID_ARG       # dst too small
+    assert L.jf_kv_checkpoint(ctypes.byref(p), FAKE, 0, FAKE, 0, None, None) == B.JF_OK
+    assert L.jf_kv_restore(ctypes.byref(p), FAKE, -1, FAKE, 0, None,
+                           None) == B.JF_ERR_INVALID_ARG
+    assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 16, 8, 0.1, 1, FAKE, FAKE, 0,
+                                   None) == B.JF_ERR_WORKSPACE_TOO_SMALL
+    assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, -1, 16, 8, 0.1, 1, FAKE, FAKE,
+                                   256, None) == B.JF_ERR_INVALID_ARG
+    assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 0, 8, 0.1, 1, FAKE, FAKE,
+                                   256, None) == B.JF_OK           # empty chunk: no-op

@@ -1,0 +1,290 @@
+"""GPU parity tests: quantize-append and checkpoint bit-exact, paged decode
+attention within tolerance of the fp64 oracle, plus invariants and edge cases.
+All calls go through the C ABI (libjfkv.so) via the thin binding."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_17475_gb300 as jf
+from oracle import affine4 as OA
+from oracle import attention as OT
+from oracle import checkpoint as OC
+from tests.cases import assert_attention_close, bits, make_case
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def gpu_append(case, fill=0):
+    pool = jf.KVPool.allocate(case.num_pages, case.P, case.Hkv, case.D, device=DEV, fill=fill)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, case.page_table.to(DEV), case.req.to(DEV), case.pos.to(DEV),
+                             case.k.to(DEV), case.v.to(DEV), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    return pool
+
+
+def pool_from_numpy(case, arr):
+    pool = jf.KVPool.allocate(case.num_pages, case.P, case.Hkv, case.D, device=DEV, fill=None)
+    pool.data.copy_(torch.from_numpy(arr))
+    return pool
+
+
+def gpu_decode(case, pool, splits, ctx=None, q=None, scale=None, page_table=None):
+    ctx = case.ctx if ctx is None else ctx
+    q = case.q if q is None else q
+    pt = case.page_table if page_table is None else page_table
+    B = len(ctx)
+    out = torch.full((B, case.Hq, case.D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(B, case.Hq, case.Hkv, case.D, splits, device=DEV)
+    scale = 1 / math.sqrt(case.D) if scale is None else scale
+    jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor(ctx, dtype=torch.int32, device=DEV),
+                            q.to(DEV), scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    return out
+
+
+# --------------------------------------------------------------------------
+# quantize-append: bit-exact against the oracle
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hkv,D,P,ctx,outliers", [
+    (2, 128, 256, [256], False),                   # the tiny workload's 256-row append
+    (2, 128, 64, [1, 63, 130], False),
+    (4, 256, 256, [1000, 517], True),
+    (3, 256, 128, [300], True),
+    (1, 128, 128, [4096], False),
+])
+def test_append_bit_exact(Hkv, D, P, ctx, outliers):
+    case = make_case(100 + sum(ctx), 2 * Hkv, Hkv, D, P, ctx, outliers=outliers,
+                     num_pages=sum(-(-c // P) for c in ctx) + 2)
+    ref = case.oracle_pool(fill=0x5A)
+    pool = gpu_append(case, fill=0x5A)
+    got = pool.data.cpu().numpy()
+    assert np.array_equal(got, ref)
+
+
+def test_append_special_groups_bit_exact():
+    """Constant groups, signed zeros, exact midpoints, subnormals, huge ranges."""
+    D, Hkv, P = 256, 2, 64
+    rng = np.random.default_rng(4)
+    n = 64
+    x = rng.standard_normal((2, n, Hkv, D)).astype(np.float32)
+    x[:, 0] = 3.0                                        # constant
+    x[:, 1] = 0.0
+    x[:, 1, :, ::3] = -0.0                               # signed zeros
+    x[:, 2] = np.tile(np.arange(64) % 16 + 0.5, D // 64)  # midpoints
+    x[:, 2, :, ::64] = 0.0
+    x[:, 2, :, 1::64] = 15.0
+    x[:, 3] *= 1e-39                                     # subnormal range
+    x[:, 4] *= 1e30                                      # huge range
+    x[:, 5, :, :32] = 1e20
+    kv = torch.from_numpy(x).to(torch.bfloat16)
+    case = make_case(7, 2 * Hkv, Hkv, D, P, [n])
+    case.k, case.v = kv[0].contiguous(), kv[1].contiguous()
+    ref = case.oracle_pool(fill=0)
+    pool = gpu_append(case, fill=0)
+    assert np.array_equal(pool.data.cpu().numpy(), ref)
+
+
+def test_append_flags_bad_rows_and_skips_them():
+    case = make_case(9, 4, 2, 128, 64, [100], num_pages=3)
+    pool = jf.KVPool.allocate(case.num_pages, 64, 2, 128, device=DEV, fill=0x11)
+    pt = case.page_table.clone()
+    pt[0, 1] = 999                                       # page id outside the pool
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, pt.to(DEV), case.req.to(DEV), case.pos.to(DEV),
+                             case.k.to(DEV), case.v.to(DEV), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) & jf.binding.JF_DEV_ERR_PAGE_ID
+    got = pool.data.cpu().numpy()
+    L = case.layout
+    ref = OA.new_pool(L, case.num_pages, fill=0x11)
+    OA.append(ref, L, case.page_table.numpy(), case.req.numpy()[:64], case.pos.numpy()[:64],
+              bits(case.k[:64]), bits(case.v[:64]))
+    assert np.array_equal(got, ref)                      # rows 64..99 skipped
+    pos = case.pos.clone()
+    pos[5] = 10_000                                      # beyond the page-table row
+    err.zero_()
+    jf.jf_kv_quantize_append(pool, case.page_table.to(DEV), case.req.to(DEV), pos.to(DEV),
+                             case.k.to(DEV), case.v.to(DEV), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) & jf.binding.JF_DEV_ERR_POSITION
+
+
+# --------------------------------------------------------------------------
+# checkpoint / restore: bit-exact
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hkv,D,P,ctx", [(2, 128, 256, [3000]), (4, 256, 64, [700]),
+                                         (4, 256, 256, [38912])])
+def test_checkpoint_and_restore_bit_exact(Hkv, D, P, ctx):
+    case = make_case(11, 2 * Hkv, Hkv, D, P, ctx, num_pages=-(-ctx[0] // P) + 3)
+    ref = case.oracle_pool(fill=0x33)
+    pool = pool_from_numpy(case, ref)
+    n = -(-ctx[0] // P)
+    blob = torch.empty(n * pool.page_bytes, dtype=torch.uint8, device=DEV)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_checkpoint(pool, case.page_table[0].to(DEV), n, blob, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    assert np.array_equal(blob.cpu().numpy(), OC.checkpoint(ref, case.page_table[0].numpy(), n))
+    fresh = jf.KVPool.allocate(case.num_pages, P, Hkv, D, device=DEV, fill=0)
+    jf.jf_kv_restore(fresh, case.page_table[0].to(DEV), n, blob, err)
+    torch.cuda.synchronize()
+    exp = OA.new_pool(case.layout, case.num_pages, fill=0)
+    OC.restore(exp, case.page_table[0].numpy(), n, OC.checkpoint(ref, case.page_table[0].numpy(), n))
+    assert np.array_equal(fresh.data.cpu().numpy(), exp)
+
+
+# --------------------------------------------------------------------------
+# paged decode attention
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,splits,outliers", [
+    (8, 2, 128, 256, [4096], 1, False),            # tiny workload, one split
+    (8, 2, 128, 256, [4096], 8, False),            # tiny workload, split-K + merge
+    (8, 2, 128, 64, [1, 33, 517, 2000], 4, False),  # ragged batch, partial pages
+    (24, 4, 256, 256, [5000], 3, True),            # paper geometry, outliers
+    (24, 4, 256, 128, [777, 1], 16, True),
+    (4, 4, 256, 64, [1500], 2, False),             # G = 1
+    (16, 2, 256, 256, [2500], 5, False),           # G = 8
+    (12, 2, 128, 128, [999], 64, False),           # more splits than needed
+])
+def test_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
+    case = make_case(200 + Hq + sum(ctx), Hq, Hkv, D, P, ctx, outliers=outliers)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    out = gpu_decode(case, pool, splits)
+    ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), ctx, bits(case.q),
+                          1 / math.sqrt(D))
+    assert_attention_close(out, ref)
+
+
+def test_decode_edge_contexts():
+    case = make_case(5, 8, 2, 128, 64, [0, 1, 64, 65])
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    for splits in (1, 4):
+        out = gpu_decode(case, pool, splits)
+        assert (out[0].float() == 0).all()                        # empty context -> zeros
+        ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), case.ctx,
+                              bits(case.q), 1 / math.sqrt(128))
+        assert_attention_close(out, ref)
+        # ctx = 1: the output is the single reconstructed V row (up to bf16 rounding)
+        v0 = OA.gather_head(ref_pool, case.layout, case.page_table.numpy()[1], 1, 0, OA.KIND_V)[0]
+        assert np.abs(out[1, 0].float().cpu().numpy() - v0).max() <= 2 ** -8 * np.abs(v0).max()
+
+
+def test_decode_page_permutation_is_bitwise_invariant():
+    case = make_case(31, 24, 4, 256, 256, [3000], num_pages=20)
+    ref_pool = case.oracle_pool()
+    out_a = gpu_decode(case, pool_from_numpy(case, ref_pool), 4)
+    perm = np.random.default_rng(2).permutation(20)
+    moved = np.empty_like(ref_pool)
+    moved[perm] = ref_pool
+    pt = case.page_table.clone()
+    n = -(-3000 // 256)
+    pt[0, :n] = torch.from_numpy(perm[case.page_table[0, :n].numpy()].astype(np.int32))
+    out_b = gpu_decode(case, pool_from_numpy(case, moved), 4, page_table=pt)
+    assert torch.equal(out_a, out_b)
+
+
+def test_decode_split_count_changes_only_rounding():
+    case = make_case(41, 24, 4, 256, 256, [20000], outliers=True)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), case.ctx, bits(case.q),
+                          1 / 16)
+    outs = [gpu_decode(case, pool, s) for s in (1, 2, 7, 39)]
+    for o in outs:
+        assert_attention_close(o, ref)
+    for o in outs[1:]:
+        assert (o.float() - outs[0].float()).abs().max().item() <= 1e-2
+
+
+def test_decode_head_subset_is_bitwise_identical():
+    """A pool holding only KV heads {1, 2} gives bitwise the same outputs for
+    their query heads as the full 4-head pool (Eq. 5: heads are independent)."""
+    full = make_case(51, 24, 4, 256, 256, [3333])
+    sub = make_case(51, 12, 2, 256, 256, [3333])
+    sub.k, sub.v = full.k[:, 1:3].contiguous(), full.v[:, 1:3].contiguous()
+    sub.page_table, sub.num_pages = full.page_table, full.num_pages
+    sub.q = full.q[:, 6:18].contiguous()
+    out_full = gpu_decode(full, gpu_append(full), 5)
+    out_sub = gpu_decode(sub, gpu_append(sub), 5)
+    assert torch.equal(out_full[:, 6:18], out_sub)
+
+
+def test_decode_poison_pages_and_tail_never_leak():
+    """NaN scales in pages outside the page table and in tail slots beyond the
+    context must not reach the output (App. E.4 poison-page protocol)."""
+    case = make_case(61, 8, 2, 128, 64, [200], num_pages=10)
+    ref_pool = case.oracle_pool(fill=0xFF)        # 0xFFFF scale/bias = NaN everywhere unwritten
+    used = set(case.page_table[0, :4].tolist())
+    assert any(p not in used for p in range(10))
+    pool = pool_from_numpy(case, ref_pool)
+    out = gpu_decode(case, pool, 2)
+    ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), case.ctx, bits(case.q),
+                          1 / math.sqrt(128))
+    assert_attention_close(out, ref)
+
+
+def test_decode_reports_bad_page_id():
+    case = make_case(71, 8, 2, 128, 64, [300])
+    pool = pool_from_numpy(case, case.oracle_pool())
+    pt = case.page_table.clone()
+    pt[0, 2] = 12345
+    out = torch.empty(1, 8, 128, dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(1, 8, 2, 128, 2, device=DEV)
+    jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor([300], dtype=torch.int32, device=DEV),
+                            case.q.to(DEV), 0.1, out, ws, 2)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) & jf.binding.JF_DEV_ERR_PAGE_ID
+
+
+def test_decode_full_window_256k_sampled_heads():
+    """The 256K full-window workload (24/4/256, 1,024 pages in a random physical
+    order, 4 K channels per KV head x20) at full size, in the launch shape the
+    benchmark uses; KV heads 0 and 3 checked against the oracle."""
+    from paper_2609_17475_gb300 import synth
+    w = synth.WORKLOADS["full_window_256k"]
+    geo = w["geometry"]
+    ctx = w["context_lens"][0]
+    gen = synth.generator(w["seed"])
+    channels = synth.outlier_channels(gen, geo.num_kv_heads, geo.head_dim)
+    k, v = synth.kv_rows(gen, ctx, geo.num_kv_heads, geo.head_dim, channels)
+    pt, npages = synth.page_tables(gen, [ctx], geo.page_size)
+    q = synth.normal_bf16(gen, (1, geo.num_q_heads, geo.head_dim))
+    req, pos = synth.append_rows_for([ctx])
+    pool = jf.KVPool.allocate(npages, geo.page_size, geo.num_kv_heads, geo.head_dim, device=DEV)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, pt.to(DEV), req.to(DEV), pos.to(DEV), k.to(DEV), v.to(DEV), err)
+    splits = jf.default_num_splits(1, geo.num_kv_heads)
+    out = torch.empty(1, geo.num_q_heads, geo.head_dim, dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(1, geo.num_q_heads, geo.num_kv_heads, geo.head_dim, splits, device=DEV)
+    scale = 1 / math.sqrt(geo.head_dim)
+    jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor([ctx], dtype=torch.int32, device=DEV),
+                            q.to(DEV), scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws) == 0
+    G = geo.group
+    for kvh in (0, 3):
+        # oracle pool holding only this KV head, built from the same bf16 rows
+        L1 = OA.PoolLayout(1, geo.page_size, geo.head_dim)
+        opool = OA.new_pool(L1, npages)
+        OA.append(opool, L1, pt.numpy(), req.numpy(), pos.numpy(),
+                  bits(k[:, kvh:kvh + 1]), bits(v[:, kvh:kvh + 1]))
+        ref = OT.paged_decode(opool, L1, pt.numpy(), [ctx], bits(q[:, kvh * G:(kvh + 1) * G]),
+                              scale)
+        assert_attention_close(out[:, kvh * G:(kvh + 1) * G], ref)
+        # sampled pages: the GPU's bytes for this head decode to the oracle's vectors
+        gp = pool.data.cpu().numpy()
+        for page in pt[0, [0, 511, 1023]].tolist():
+            for kind in (OA.KIND_K, OA.KIND_V):
+                L4 = OA.PoolLayout(geo.num_kv_heads, geo.page_size, geo.head_dim)
+                o4 = L4.codes_offset(kind, kvh, 0)
+                o1 = L1.codes_offset(kind, 0, 0)
+                n = geo.page_size * L4.code_bytes
+                assert np.array_equal(gp[page, o4:o4 + n], opool[page, o1:o1 + n])
