@@ -111,12 +111,187 @@ struct DecodeSmem {
   static_assert(DWARPS * 8 * 2 * 4 <= SB_BYTES, "combine ml buffer must fit");
 };
 
+// Per-warp online-softmax state.  Thread (r, c) of the warp owns query heads
+// 2c and 2c+1 (columns of the m16n8 accumulators) and, for PV, the d-rows
+// {64g + 4r + e, 64g + 32 + 4r + e}.
+template <int NG>
+struct DecodeState {
+  float m0, m1, l0, l1;
+  float O[NG][4][4];
+  float Bs[NG][2];
+  __device__ __forceinline__ void init() {
+    m0 = m1 = -INFINITY;
+    l0 = l1 = 0.f;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      Bs[g][0] = Bs[g][1] = 0.f;
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) O[g][e][i] = 0.f;
+    }
+  }
+};
+
+template <int NG>
+struct ChunkCtx {
+  const uint32_t (&qf)[NG][4][2];
+  const float (&Qh)[NG][2];
+  float cA, cB;
+  int r, c, ld_t, ld_ch;
+};
+
+template <int NG>
+__device__ __forceinline__ void load_sb_words(const uint8_t* p, uint32_t (&w)[NG]) {
+  if constexpr (NG == 4) {
+    const uint4 x = *reinterpret_cast<const uint4*>(p);
+    w[0] = x.x; w[1] = x.y; w[2] = x.z; w[3] = x.w;
+  } else {
+    const uint2 x = *reinterpret_cast<const uint2*>(p);
+    w[0] = x.x; w[1] = x.y;
+  }
+}
+
+// One 32-position chunk (two 16-position MMA tiles).  FULL: every position is
+// valid, so no masking work is done; otherwise positions >= nvalid are masked
+// (their logits become -inf and their scale/bias words are never used, so
+// whatever bytes sit in unused slots cannot leak into the result).
+template <int D, bool FULL>
+__device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const ChunkCtx<D / 64>& cc,
+                                              uint32_t kc, const uint8_t* ksb, int nvalid) {
+  constexpr int NG = D / 64;
+  constexpr int CB = D / 2;
+  constexpr int SBB = 4 * NG;
+  constexpr int SB_BUF = DTOK * SBB;
+  constexpr float NEG_INF = -INFINITY;
+  const uint32_t vc = kc + DTOK * CB;
+  const uint8_t* vsb = ksb + SB_BUF;
+  const int r = cc.r;
+
+  float sc[2][4];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int ta = 16 * j + r, tb = ta + 8;
+    float acc[NG][4];
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      uint32_t w0, w1, w2, w3;
+      ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
+      acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
+      mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), cc.qf[g][0][0], cc.qf[g][0][1]);
+      mma_f16(acc[g], nib2(w0), nib2(w1), nib3(w0), nib3(w1), cc.qf[g][1][0], cc.qf[g][1][1]);
+      mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), cc.qf[g][2][0], cc.qf[g][2][1]);
+      mma_f16(acc[g], nib2(w2), nib2(w3), nib3(w2), nib3(w3), cc.qf[g][3][0], cc.qf[g][3][1]);
+    }
+    uint32_t wa[NG], wb[NG];
+    load_sb_words<NG>(ksb + ta * SBB, wa);
+    load_sb_words<NG>(ksb + tb * SBB, wb);
+    float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      const float sa = bf16lo_to_f32(wa[g]), ba = bf16hi_to_f32(wa[g]);
+      const float sbv = bf16lo_to_f32(wb[g]), bbv = bf16hi_to_f32(wb[g]);
+      t1[0] = fmaf(sa, acc[g][0], t1[0]);
+      t1[1] = fmaf(sa, acc[g][1], t1[1]);
+      t1[2] = fmaf(sbv, acc[g][2], t1[2]);
+      t1[3] = fmaf(sbv, acc[g][3], t1[3]);
+      t2[0] = fmaf(ba, cc.Qh[g][0], t2[0]);
+      t2[1] = fmaf(ba, cc.Qh[g][1], t2[1]);
+      t2[2] = fmaf(bbv, cc.Qh[g][0], t2[2]);
+      t2[3] = fmaf(bbv, cc.Qh[g][1], t2[3]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) sc[j][i] = fmaf(t1[i], cc.cA, t2[i] * cc.cB);
+    if constexpr (!FULL) {
+      if (ta >= nvalid) sc[j][0] = sc[j][1] = NEG_INF;
+      if (tb >= nvalid) sc[j][2] = sc[j][3] = NEG_INF;
+    }
+  }
+
+  // ---- online softmax over the 32 positions of this chunk -------------
+  float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][2]), fmaxf(sc[1][0], sc[1][2]));
+  float mx1 = fmaxf(fmaxf(sc[0][1], sc[0][3]), fmaxf(sc[1][1], sc[1][3]));
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+  }
+  const float nm0 = fmaxf(st.m0, mx0), nm1 = fmaxf(st.m1, mx1);
+  if (__any_sync(0xffffffffu, (nm0 > st.m0) || (nm1 > st.m1))) {
+    const float f0 = (nm0 > st.m0) ? fast_exp2(st.m0 - nm0) : 1.f;
+    const float f1 = (nm1 > st.m1) ? fast_exp2(st.m1 - nm1) : 1.f;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        st.O[g][e][0] *= f0; st.O[g][e][2] *= f0;
+        st.O[g][e][1] *= f1; st.O[g][e][3] *= f1;
+      }
+      st.Bs[g][0] *= f0;
+      st.Bs[g][1] *= f1;
+    }
+    st.l0 *= f0;
+    st.l1 *= f1;
+    st.m0 = nm0;
+    st.m1 = nm1;
+  }
+  float p[2][4];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    if constexpr (FULL) {
+      p[j][0] = fast_exp2(sc[j][0] - st.m0);
+      p[j][1] = fast_exp2(sc[j][1] - st.m1);
+      p[j][2] = fast_exp2(sc[j][2] - st.m0);
+      p[j][3] = fast_exp2(sc[j][3] - st.m1);
+    } else {
+      p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
+      p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
+      p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
+      p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
+    }
+    st.l0 += p[j][0] + p[j][2];
+    st.l1 += p[j][1] + p[j][3];
+  }
+
+  // ---- PV ---------------------------------------------------------------
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int ta = 16 * j + r, tb = ta + 8;
+    uint32_t wa[NG], wb[NG];
+    load_sb_words<NG>(vsb + ta * SBB, wa);
+    load_sb_words<NG>(vsb + tb * SBB, wb);
+    bool va = true, vb = true;
+    if constexpr (!FULL) {
+      va = ta < nvalid;
+      vb = tb < nvalid;
+    }
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      float sva = bf16lo_to_f32(wa[g]), bva = bf16hi_to_f32(wa[g]);
+      float svb = bf16lo_to_f32(wb[g]), bvb = bf16hi_to_f32(wb[g]);
+      if constexpr (!FULL) {
+        if (!va) sva = bva = 0.f;
+        if (!vb) svb = bvb = 0.f;
+      }
+      st.Bs[g][0] = fmaf(bva, p[j][0], fmaf(bvb, p[j][2], st.Bs[g][0]));
+      st.Bs[g][1] = fmaf(bva, p[j][1], fmaf(bvb, p[j][3], st.Bs[g][1]));
+      const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
+      const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
+      uint32_t v0, v1, v2, v3;
+      ldsm_x4_t(v0, v1, v2, v3, vc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
+      mma_f16(st.O[g][0], nib0(v0), nib0(v2), nib0(v1), nib0(v3), b0, b1);
+      mma_f16(st.O[g][1], nib1(v0), nib1(v2), nib1(v1), nib1(v3), b0, b1);
+      mma_f16(st.O[g][2], nib2(v0), nib2(v2), nib2(v1), nib2(v3), b0, b1);
+      mma_f16(st.O[g][3], nib3(v0), nib3(v2), nib3(v1), nib3(v3), b0, b1);
+    }
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(DWARPS * 32, 2)
 decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
   using L = DecodeSmem<D>;
   constexpr int NG = L::NG;
-  constexpr int CB = L::CB;
   constexpr int SBB = L::SBB;
   constexpr float NEG_INF = -INFINITY;
 
@@ -216,21 +391,35 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const float cA = a.scale_log2 * 16777216.f * ldexpf(1.f, qe);
   const float cB = a.scale_log2;
 
+  // ---- page ids: lane i holds the page of this warp's iteration 32k + i ------
+  // (two blocks of 32 in flight so the dependent load never stalls an issue)
+  auto load_pages = [&](int blk) -> int {
+    const int it = blk * 32 + lane;
+    int page = -1;
+    if (it < my_n) {
+      const int pidx = ((c_begin + warp + it * DWARPS) * DTOK) / a.P;
+      if (pidx < a.pt_stride) page = __ldg(a.page_table + (int64_t)b * a.pt_stride + pidx);
+    }
+    return page;
+  };
+  int pg_cur = load_pages(0);
+  int pg_next = load_pages(1);
+
   // ---- TMA producer (lane 0 of each warp feeds its own ring) -------------
   uint32_t valid = 0;
   auto issue = [&](int it) {
     const int s = it % DSTAGES;
-    int ok = 1;
+    if (it >= 32 && (it & 31) == 0) {
+      pg_cur = pg_next;
+      pg_next = load_pages((it >> 5) + 1);
+    }
+    const int page = __shfl_sync(0xffffffffu, pg_cur, it & 31);
+    const bool ok = page >= 0 && page < a.num_pages;
     if (lane == 0) {
-      const int ch = c_begin + warp + it * DWARPS;
-      const int tok0 = ch * DTOK;
-      const int pidx = tok0 / a.P, inp = tok0 % a.P;
+      const int inp = ((c_begin + warp + it * DWARPS) * DTOK) % a.P;
       uint64_t* bar = &bars[warp * DSTAGES + s];
-      int page = -1;
-      if (pidx < a.pt_stride) page = a.page_table[(int64_t)b * a.pt_stride + pidx];
-      if (page < 0 || page >= a.num_pages) {
+      if (!ok) {
         flag_error(a.status, JF_DEV_ERR_PAGE_ID);
-        ok = 0;
         mbar_arrive(bar);
       } else {
         uint8_t* kc = codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF;
@@ -244,7 +433,6 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
         bulk_g2s(ks + L::SB_BUF, gsb + a.sb_region, L::SB_BUF, bar);
       }
     }
-    ok = __shfl_sync(0xffffffffu, ok, 0);
     valid = (valid & ~(1u << s)) | ((uint32_t)ok << s);
   };
 
@@ -252,21 +440,13 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   for (int it = 0; it < npro; ++it) issue(it);
 
   // ---- running state ---------------------------------------------------
-  float m0 = NEG_INF, m1 = NEG_INF, l0 = 0.f, l1 = 0.f;
-  float O[NG][4][4];
-  float Bs[NG][2];
-#pragma unroll
-  for (int g = 0; g < NG; ++g) {
-    Bs[g][0] = Bs[g][1] = 0.f;
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-#pragma unroll
-      for (int i = 0; i < 4; ++i) O[g][e][i] = 0.f;
-  }
+  DecodeState<NG> st;
+  st.init();
 
   // ldmatrix row address pieces: matrix m = lane>>3 -> (position half, chunk)
   const int ld_t = (lane & 7) + 8 * ((lane >> 3) & 1);
   const int ld_ch = lane >> 4;
+  const ChunkCtx<NG> cc{qf, Qh, cA, cB, r, c, ld_t, ld_ch};
 
   int done = 0;
   for (int it = 0; it < my_n; ++it) {
@@ -280,133 +460,11 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const bool ok = (valid >> s) & 1u;
     const int tokbase = (c_begin + warp + it * DWARPS) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF);
-    const uint32_t vc = kc + L::CODE_BUF;
     const uint8_t* ksb = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
-    const uint8_t* vsb = ksb + L::SB_BUF;
-
-    float sc[2][4];
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int ta = 16 * j + r, tb = ta + 8;
-      const bool va = ok && (tokbase + ta < ctx);
-      const bool vb = ok && (tokbase + tb < ctx);
-      float acc[NG][4];
-#pragma unroll
-      for (int g = 0; g < NG; ++g) {
-        uint32_t w0, w1, w2, w3;
-        ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + ld_t, 2 * g + ld_ch));
-        acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
-        mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), qf[g][0][0], qf[g][0][1]);
-        mma_f16(acc[g], nib2(w0), nib2(w1), nib3(w0), nib3(w1), qf[g][1][0], qf[g][1][1]);
-        mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), qf[g][2][0], qf[g][2][1]);
-        mma_f16(acc[g], nib2(w2), nib2(w3), nib3(w2), nib3(w3), qf[g][3][0], qf[g][3][1]);
-      }
-      uint32_t wa[NG], wb[NG];
-      if constexpr (NG == 4) {
-        const uint4 xa = *reinterpret_cast<const uint4*>(ksb + ta * SBB);
-        const uint4 xb = *reinterpret_cast<const uint4*>(ksb + tb * SBB);
-        wa[0] = xa.x; wa[1] = xa.y; wa[2] = xa.z; wa[3] = xa.w;
-        wb[0] = xb.x; wb[1] = xb.y; wb[2] = xb.z; wb[3] = xb.w;
-      } else {
-        const uint2 xa = *reinterpret_cast<const uint2*>(ksb + ta * SBB);
-        const uint2 xb = *reinterpret_cast<const uint2*>(ksb + tb * SBB);
-        wa[0] = xa.x; wa[1] = xa.y;
-        wb[0] = xb.x; wb[1] = xb.y;
-      }
-      float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int g = 0; g < NG; ++g) {
-        const float sa = bf16lo_to_f32(wa[g]), ba = bf16hi_to_f32(wa[g]);
-        const float sbv = bf16lo_to_f32(wb[g]), bbv = bf16hi_to_f32(wb[g]);
-        t1[0] = fmaf(sa, acc[g][0], t1[0]);
-        t1[1] = fmaf(sa, acc[g][1], t1[1]);
-        t1[2] = fmaf(sbv, acc[g][2], t1[2]);
-        t1[3] = fmaf(sbv, acc[g][3], t1[3]);
-        t2[0] = fmaf(ba, Qh[g][0], t2[0]);
-        t2[1] = fmaf(ba, Qh[g][1], t2[1]);
-        t2[2] = fmaf(bbv, Qh[g][0], t2[2]);
-        t2[3] = fmaf(bbv, Qh[g][1], t2[3]);
-      }
-      sc[j][0] = va ? fmaf(t1[0], cA, t2[0] * cB) : NEG_INF;
-      sc[j][1] = va ? fmaf(t1[1], cA, t2[1] * cB) : NEG_INF;
-      sc[j][2] = vb ? fmaf(t1[2], cA, t2[2] * cB) : NEG_INF;
-      sc[j][3] = vb ? fmaf(t1[3], cA, t2[3] * cB) : NEG_INF;
-    }
-
-    // ---- online softmax over the 32 positions of this chunk -------------
-    float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][2]), fmaxf(sc[1][0], sc[1][2]));
-    float mx1 = fmaxf(fmaxf(sc[0][1], sc[0][3]), fmaxf(sc[1][1], sc[1][3]));
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) {
-      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-    }
-    const float nm0 = fmaxf(m0, mx0), nm1 = fmaxf(m1, mx1);
-    if (__any_sync(0xffffffffu, (nm0 > m0) || (nm1 > m1))) {
-      const float f0 = (nm0 > m0) ? fast_exp2(m0 - nm0) : 1.f;
-      const float f1 = (nm1 > m1) ? fast_exp2(m1 - nm1) : 1.f;
-#pragma unroll
-      for (int g = 0; g < NG; ++g) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          O[g][e][0] *= f0; O[g][e][2] *= f0;
-          O[g][e][1] *= f1; O[g][e][3] *= f1;
-        }
-        Bs[g][0] *= f0;
-        Bs[g][1] *= f1;
-      }
-      l0 *= f0;
-      l1 *= f1;
-      m0 = nm0;
-      m1 = nm1;
-    }
-    float p[2][4];
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - m0);
-      p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - m1);
-      p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - m0);
-      p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - m1);
-      l0 += p[j][0] + p[j][2];
-      l1 += p[j][1] + p[j][3];
-    }
-
-    // ---- PV ---------------------------------------------------------------
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-      const int ta = 16 * j + r, tb = ta + 8;
-      const bool va = ok && (tokbase + ta < ctx);
-      const bool vb = ok && (tokbase + tb < ctx);
-      uint32_t wa[NG], wb[NG];
-      if constexpr (NG == 4) {
-        const uint4 xa = *reinterpret_cast<const uint4*>(vsb + ta * SBB);
-        const uint4 xb = *reinterpret_cast<const uint4*>(vsb + tb * SBB);
-        wa[0] = xa.x; wa[1] = xa.y; wa[2] = xa.z; wa[3] = xa.w;
-        wb[0] = xb.x; wb[1] = xb.y; wb[2] = xb.z; wb[3] = xb.w;
-      } else {
-        const uint2 xa = *reinterpret_cast<const uint2*>(vsb + ta * SBB);
-        const uint2 xb = *reinterpret_cast<const uint2*>(vsb + tb * SBB);
-        wa[0] = xa.x; wa[1] = xa.y;
-        wb[0] = xb.x; wb[1] = xb.y;
-      }
-#pragma unroll
-      for (int g = 0; g < NG; ++g) {
-        const float sva = va ? bf16lo_to_f32(wa[g]) : 0.f;
-        const float bva = va ? bf16hi_to_f32(wa[g]) : 0.f;
-        const float svb = vb ? bf16lo_to_f32(wb[g]) : 0.f;
-        const float bvb = vb ? bf16hi_to_f32(wb[g]) : 0.f;
-        Bs[g][0] = fmaf(bva, p[j][0], fmaf(bvb, p[j][2], Bs[g][0]));
-        Bs[g][1] = fmaf(bva, p[j][1], fmaf(bvb, p[j][3], Bs[g][1]));
-        const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
-        const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
-        uint32_t v0, v1, v2, v3;
-        ldsm_x4_t(v0, v1, v2, v3, vc + swz<CB>(16 * j + ld_t, 2 * g + ld_ch));
-        mma_f16(O[g][0], nib0(v0), nib0(v2), nib0(v1), nib0(v3), b0, b1);
-        mma_f16(O[g][1], nib1(v0), nib1(v2), nib1(v1), nib1(v3), b0, b1);
-        mma_f16(O[g][2], nib2(v0), nib2(v2), nib2(v1), nib2(v3), b0, b1);
-        mma_f16(O[g][3], nib3(v0), nib3(v2), nib3(v1), nib3(v3), b0, b1);
-      }
-    }
+    if (ok && tokbase + DTOK <= ctx)
+      process_chunk<D, true>(st, cc, kc, ksb, 0);
+    else
+      process_chunk<D, false>(st, cc, kc, ksb, ok ? ctx - tokbase : 0);
 
     __syncwarp();
     if (it + DSTAGES < my_n) {
@@ -419,6 +477,12 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     for (int it = done; it < my_n && it < done + DSTAGES; ++it)
       mbar_wait_bounded(&bars[warp * DSTAGES + it % DSTAGES], (it / DSTAGES) & 1, 1u << 16);
   }
+  float& m0 = st.m0;
+  float& m1 = st.m1;
+  float& l0 = st.l0;
+  float& l1 = st.l1;
+  auto& O = st.O;
+  auto& Bs = st.Bs;
 
   // ---- per-warp finalize ---------------------------------------------------
 #pragma unroll
