@@ -78,7 +78,8 @@ size_t jf_kv_page_bytes(int32_t num_kv_heads, int32_t page_size, int32_t head_di
 
 /*
  * Workspace bytes jf_paged_decode_attn needs for at most `num_splits`
- * splits per (request, KV head): 256 + B*Hq*S*(4*D + 8) bytes.  The size
+ * splits per (request, KV head): 256 + roundup(8*B*Hq*S, 256) + 4*B*Hq*S*D
+ * bytes (status word, per-split (max, sum) pairs, per-split outputs).  The size
  * depends on batch, heads, splits and head_dim only, never on the context
  * length (Sec. 2, Eq. 3 is the paper's argument for bounding temporaries).
  * Returns 0 for invalid arguments.
@@ -136,7 +137,8 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
  *                 KV head).  Each partition keeps (max, sum, partial output)
  *                 in the workspace; a second kernel merges them.
  * Numerics: K codes and q enter fp16 tensor-core products with fp32
- * accumulation (q must satisfy |q| < 65504); the softmax runs in fp32 with the
+ * accumulation (q is rescaled by a power of two per KV head when max|q| >= 2^14,
+ * so any finite bf16 q is accepted); the softmax runs in fp32 with the
  * maximum subtracted; probabilities scaled by the V group scale enter fp16
  * products, so V group scales must stay below 65504.  Output rounded RNE.
  */
@@ -178,6 +180,38 @@ int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int3
  */
 int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
                   const void* src, size_t src_bytes, int32_t* err_flag, void* stream);
+
+/*
+ * Decode attention without a caller-supplied workspace.  The paper has no
+ * counterpart; this entry point exists for callers that cannot allocate
+ * device memory themselves -- for example a plug-in running inside a host
+ * runtime that owns the whole device-memory budget and hands out no
+ * allocator, or a plain C caller with no CUDA allocator of its own.
+ *
+ * Same arguments and result as jf_paged_decode_attn minus the workspace:
+ * the split partials live in a file-scope device array of
+ * JF_STATIC_WORKSPACE_BYTES bytes inside libjfkv.so, which every GPU that
+ * loads the library holds until the process exits.  Nothing is allocated
+ * or freed by this call.
+ *   - Calls whose jf_attn_workspace_bytes(batch, Hq, Hkv, D, num_splits)
+ *     exceeds JF_STATIC_WORKSPACE_BYTES return JF_ERR_WORKSPACE_TOO_SMALL
+ *     (lower num_splits or the batch).
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first
+ *     call before any stream capture.
+ *   - All calls on a device share the one array and it keeps the last
+ *     call's contents; the call clears the status word it needs to start
+ *     at zero.  Calls that overlap on the GPU (different streams, or
+ *     several host threads) race on the array: serialize them.
+ *   - err_flag: device int32 or NULL; receives this call's device status
+ *     word (JF_DEV_* bits) once the call completes on `stream`.
+ */
+#define JF_STATIC_WORKSPACE_BYTES ((size_t)8 << 20)
+
+int jf_paged_decode_attn_noalloc(const jf_kv_pool* pool, const int32_t* page_table,
+                                 int32_t pt_stride, const int32_t* context_lens, int32_t batch,
+                                 const void* q, int32_t num_q_heads, float softmax_scale,
+                                 void* out, int32_t num_splits, int32_t* err_flag, void* stream);
 
 /* Human-readable name of a JF_* status code. */
 const char* jf_status_string(int status);

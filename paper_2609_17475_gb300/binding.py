@@ -31,7 +31,9 @@ EXPORTS = [
     "jf_kv_page_bytes", "jf_attn_workspace_bytes", "jf_prefill_workspace_bytes",
     "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
+    "jf_paged_decode_attn_noalloc",
 ]
+JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
 
 class JfError(RuntimeError):
@@ -71,6 +73,8 @@ def lib() -> ctypes.CDLL:
                                                      SZ, P]),
             "jf_kv_checkpoint": (ctypes.c_int, [PP, P, I32, P, SZ, P, P]),
             "jf_kv_restore": (ctypes.c_int, [PP, P, I32, P, SZ, P, P]),
+            "jf_paged_decode_attn_noalloc": (ctypes.c_int, [PP, P, I32, P, I32, P, I32, F32, P,
+                                                            I32, P, P]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -207,6 +211,31 @@ def jf_paged_decode_attn(pool: KVPool, page_table: torch.Tensor, context_lens: t
                                      float(softmax_scale), _ptr(out), _ptr(workspace),
                                      workspace.numel(), int(num_splits), _stream(stream))
     _check("jf_paged_decode_attn", st)
+
+
+def jf_paged_decode_attn_noalloc(pool: KVPool, page_table: torch.Tensor,
+                                 context_lens: torch.Tensor, q: torch.Tensor, softmax_scale: float,
+                                 out: torch.Tensor, num_splits: int,
+                                 err_flag: Optional[torch.Tensor] = None, stream=None) -> None:
+    """Decode attention for callers that cannot allocate device memory: the
+    split partials live in a fixed device array inside libjfkv.so
+    (JF_STATIC_WORKSPACE_BYTES), shared by every call on the device, so calls
+    that overlap on the GPU race.  The first call on a device sets the array up
+    and should come before any stream capture."""
+    _need(page_table, torch.int32, "page_table")
+    _need(context_lens, torch.int32, "context_lens")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    if err_flag is not None:
+        _need(err_flag, torch.int32, "err_flag")
+    B, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim or page_table.shape[0] != B or context_lens.numel() != B:
+        raise ValueError("shape mismatch")
+    st = lib().jf_paged_decode_attn_noalloc(ctypes.byref(pool.c_struct()), _ptr(page_table),
+                                             page_table.shape[1], _ptr(context_lens), B, _ptr(q),
+                                             Hq, float(softmax_scale), _ptr(out), int(num_splits),
+                                             _ptr(err_flag), _stream(stream))
+    _check("jf_paged_decode_attn_noalloc", st)
 
 
 def jf_prefill_chunk_attn(pool: KVPool, page_table_row: torch.Tensor, q: torch.Tensor,

@@ -189,6 +189,75 @@ int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t
                           false, static_cast<cudaStream_t>(stream));
 }
 
+// ---------------------------------------------------------------------------
+// Decode without a caller-supplied workspace: scratch in a file-scope device
+// array.  In host code `jf_static_decode_ws` only names the symbol; its device
+// address comes from cudaGetSymbolAddress, looked up once per device.
+// ---------------------------------------------------------------------------
+}  // extern "C"
+
+static __device__ __align__(256) unsigned char jf_static_decode_ws[JF_STATIC_WORKSPACE_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 256;
+std::mutex g_static_ws_mu;
+void* g_static_ws_ptr[kMaxDevices] = {};
+
+// Device address of the static workspace on the current device (set-up on the
+// first call per device, with that device current).
+int static_workspace(void** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return JF_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return JF_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_static_ws_mu);
+  if (!g_static_ws_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, jf_static_decode_ws) != cudaSuccess || !p) return JF_ERR_CUDA;
+    g_static_ws_ptr[dev] = p;
+  }
+  *out = g_static_ws_ptr[dev];
+  return JF_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int jf_paged_decode_attn_noalloc(const jf_kv_pool* pool, const int32_t* page_table,
+                                 int32_t pt_stride, const int32_t* context_lens, int32_t batch,
+                                 const void* q, int32_t num_q_heads, float softmax_scale,
+                                 void* out, int32_t num_splits, int32_t* err_flag, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (!page_table || !context_lens || !q || !out) return JF_ERR_INVALID_ARG;
+  if (batch < 1 || batch > 65535 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
+  if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
+  if (num_q_heads / pool->num_kv_heads > 8) return JF_ERR_UNSUPPORTED;
+  if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
+  if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16)) return JF_ERR_INVALID_ARG;
+  const size_t need = jf_attn_workspace_bytes(batch, num_q_heads, pool->num_kv_heads,
+                                              pool->head_dim, num_splits);
+  if (need == 0) return JF_ERR_INVALID_ARG;
+  if (need > JF_STATIC_WORKSPACE_BYTES) return JF_ERR_WORKSPACE_TOO_SMALL;
+  void* ws = nullptr;
+  st = static_workspace(&ws);
+  if (st) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the status word is the only scratch that must start at zero
+  if (cudaMemsetAsync(ws, 0, sizeof(int32_t), s) != cudaSuccess) return JF_ERR_CUDA;
+  const Geom g = make_geom(*pool);
+  CUtensorMap tmap;
+  st = make_codes_map(g, pool->base, 32, &tmap);
+  if (st) return st;
+  st = launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q, num_q_heads,
+                     softmax_scale, out, ws, num_splits, s);
+  if (st) return st;
+  if (err_flag &&
+      cudaMemcpyAsync(err_flag, ws, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return JF_ERR_CUDA;
+  return JF_OK;
+}
+
 const char* jf_status_string(int status) {
   switch (status) {
     case JF_OK: return "JF_OK";
