@@ -156,9 +156,8 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
   if ((int64_t)q_start + chunk_len > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
   if (chunk_len == 0) return JF_OK;
   const Geom g = make_geom(*pool);
-  CUtensorMap tmap;
-  st = make_codes_map(g, pool->base, 64, &tmap);
-  if (st) return st;
+  if (num_q_heads / pool->num_kv_heads > 128) return JF_ERR_UNSUPPORTED;
+  CUtensorMap tmap{};
   return launch_prefill(g, *pool, tmap, page_table_row, q, q_start, chunk_len, num_q_heads,
                         softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
 }

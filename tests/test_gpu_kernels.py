@@ -288,3 +288,72 @@ def test_decode_full_window_256k_sampled_heads():
                 o1 = L1.codes_offset(kind, 0, 0)
                 n = geo.page_size * L4.code_bytes
                 assert np.array_equal(gp[page, o4:o4 + n], opool[page, o1:o1 + n])
+
+
+# --------------------------------------------------------------------------
+# prefill chunk attention (tcgen05)
+# --------------------------------------------------------------------------
+def gpu_prefill(case, pool, q, q_start, causal, scale):
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=DEV)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), q_start, scale, causal,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    return out
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,P,q_start,C,causal", [
+    (8, 2, 128, 256, 0, 256, True),          # tiny geometry, first chunk
+    (8, 2, 128, 64, 300, 77, True),           # ragged chunk, partial pages
+    (24, 4, 256, 256, 0, 130, True),          # G = 6: 21 queries per CTA
+    (24, 4, 256, 256, 1000, 64, True),
+    (24, 4, 256, 128, 517, 200, False),       # non-causal
+    (4, 4, 256, 64, 100, 129, True),          # G = 1: 128 queries per CTA
+    (16, 2, 128, 128, 64, 40, True),          # G = 8
+])
+def test_prefill_matches_oracle(Hq, Hkv, D, P, q_start, C, causal):
+    total = q_start + C
+    case = make_case(300 + Hq + total, Hq, Hkv, D, P, [total], outliers=True)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    from paper_2609_17475_gb300 import synth
+    q = synth.normal_bf16(synth.generator(7 + C), (C, Hq, D))
+    scale = 1 / math.sqrt(D)
+    out = gpu_prefill(case, pool, q, q_start, causal, scale)
+    ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q), q_start,
+                           scale, causal=causal)
+    assert_attention_close(out, ref)
+
+
+def test_prefill_32k_prefix_sampled_rows():
+    """The last 2,048-query chunk of the 32K prompt (24/4/256, P 256): sampled
+    query rows checked against the oracle's decode at ctx = position + 1."""
+    Hq, Hkv, D, P, C = 24, 4, 256, 256, 2048
+    q_start = 32768 - C
+    case = make_case(404, Hq, Hkv, D, P, [32768])
+    pool = gpu_append(case)
+    from paper_2609_17475_gb300 import synth
+    q = synth.normal_bf16(synth.generator(405), (C, Hq, D))
+    out = gpu_prefill(case, pool, q, q_start, True, 1 / 16)
+    G = Hq // Hkv
+    for kvh in (0, 3):
+        L1 = OA.PoolLayout(1, P, D)
+        opool = OA.new_pool(L1, case.num_pages)
+        OA.append(opool, L1, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
+                  bits(case.k[:, kvh:kvh + 1]), bits(case.v[:, kvh:kvh + 1]))
+        for i in (0, 1, 20, 21, 1000, C - 1):
+            ref = OT.paged_decode(opool, L1, case.page_table.numpy(), [q_start + i + 1],
+                                  bits(q[i:i + 1, kvh * G:(kvh + 1) * G]), 1 / 16)
+            assert_attention_close(out[i:i + 1, kvh * G:(kvh + 1) * G], ref)
+
+
+def test_prefill_poison_pages_never_leak():
+    case = make_case(77, 8, 2, 128, 64, [300], num_pages=12)
+    ref_pool = case.oracle_pool(fill=0xFF)
+    pool = pool_from_numpy(case, ref_pool)
+    from paper_2609_17475_gb300 import synth
+    q = synth.normal_bf16(synth.generator(78), (100, 8, 128))
+    out = gpu_prefill(case, pool, q, 200, True, 0.1)
+    ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q), 200, 0.1)
+    assert_attention_close(out, ref)
