@@ -293,9 +293,193 @@ def run_ours(args, world, rank, local):
         "gpu_launches": args.steps * layers * 3,
         "clocks": clocks,
     }
+    if args.rows:
+        import json as _json
+        pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+        peak_tf = float(_json.load(open(pk))["bf16_tflops"]) if os.path.exists(pk) else 1900.0
+        result["rows"] = bench_rows(jf, synth, dev, stream, hbm, peak_tf)
+        result["rows"]["peak_tensor_tflops_f16"] = peak_tf
     if rank == 0 and args.cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(args)
     return result
+
+
+# ---------------------------------------------------------------------------
+# the other rows of the path, each on its own workload shape
+# ---------------------------------------------------------------------------
+def _event_time(fn, reps, stream):
+    """Mean milliseconds per call of fn() on `stream`, CUDA events, after 2 warm calls."""
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
+    """Append, prefill chunk, checkpoint, two-request and mixed-batch decode.
+    Every tensor is allocated on `stream`, the stream the kernels run on, so the
+    caching allocator never hands a buffer back out while a kernel still reads it."""
+    with torch.cuda.stream(stream):
+        return _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf)
+
+
+def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
+    out = {}
+
+    def check(section, *words):
+        stream.synchronize()
+        bad = {"err": int(err.item())}
+        for i, w in enumerate(words):
+            bad[f"ws{i}"] = jf.workspace_status(w)
+        assert not any(bad.values()), f"device status set in {section}: {bad}"
+
+    g = torch.Generator(device=dev)
+    g.manual_seed(4242)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    # ---- prefill-then-decode shapes: 24/4/256, P 256, 32K prompt + 6K decode
+    Hq, Hkv, D, P = 24, 4, 256, 256
+    prompt, chunk, steps = 32768, 2048, 6144
+    total = prompt + steps
+    npages = total // P
+    pt = torch.randperm(npages, device=dev, generator=g).to(torch.int32).view(1, -1)
+    pool = jf.KVPool.allocate(npages, P, Hkv, D, device=dev, fill=0)
+    zero_req = torch.zeros(chunk, dtype=torch.int32, device=dev)
+    kc = torch.randn(chunk, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    vc = torch.randn(chunk, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    qc = torch.randn(chunk, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    oc = torch.empty_like(qc)
+    pws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=dev)
+    scale = 1 / math.sqrt(D)
+    # a1: append of one 2,048-row chunk (positions 0..2047)
+    pos0 = torch.arange(chunk, dtype=torch.int32, device=dev)
+    t_app = _event_time(lambda: jf.jf_kv_quantize_append(pool, pt, zero_req, pos0, kc, vc, err,
+                                                         stream=stream), 50, stream)
+    app_bytes = 2 * chunk * Hkv * D * 2 + chunk * 2 * Hkv * (D // 2 + 4 * D // 64) + chunk * 8
+    check("a1 append")
+    out["a1_append_2048_rows"] = {"us": t_app * 1e3, "GBps": app_bytes / (t_app / 1e3) / 1e9,
+                                  "frac_hbm": app_bytes / (t_app / 1e3) / 1e9 / peaks_gbs,
+                                  "alg_bytes": app_bytes}
+    # fill the whole prompt: 16 appends, each followed by its prefill chunk (timed end to end)
+    def prefill_all():
+        for c in range(prompt // chunk):
+            pos = torch.arange(c * chunk, (c + 1) * chunk, dtype=torch.int32, device=dev)
+            jf.jf_kv_quantize_append(pool, pt, zero_req, pos, kc, vc, err, stream=stream)
+            jf.jf_prefill_chunk_attn(pool, pt[0], qc, c * chunk, scale, True, oc, pws,
+                                     stream=stream)
+    t_pf_all = _event_time(prefill_all, 3, stream)
+    check("a1+a4 prompt", pws)
+    flops_all = sum(4 * Hq * D * (chunk * c * chunk + chunk * (chunk + 1) // 2)
+                    for c in range(prompt // chunk))
+    # a4: the last chunk alone (2,048 causal queries over a 30,720-position prefix)
+    q_last = prompt - chunk
+    t_pf = _event_time(lambda: jf.jf_prefill_chunk_attn(pool, pt[0], qc, q_last, scale, True, oc,
+                                                        pws, stream=stream), 10, stream)
+    flops = 4 * Hq * D * (chunk * q_last + chunk * (chunk + 1) // 2)
+    out["a4_prefill_chunk_2048_at_30720"] = {
+        "ms": t_pf, "TFLOPs": flops / (t_pf / 1e3) / 1e12,
+        "frac_tensor": flops / (t_pf / 1e3) / 1e12 / peak_tf, "flops": flops}
+    out["a1a4_prompt_32k_16_chunks"] = {
+        "ms": t_pf_all, "TFLOPs_attention": flops_all / (t_pf_all / 1e3) / 1e12,
+        "prompt_positions_per_s": prompt / (t_pf_all / 1e3)}
+    # decode loop of the 32K+6K workload: 6,144 x (append 1 row, decode) in one CUDA graph
+    q1 = torch.randn(1, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o1 = torch.empty_like(q1)
+    k1 = torch.randn(1, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    v1 = torch.randn(1, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    splits = jf.default_num_splits(1, Hkv)
+    dws = jf.decode_workspace(1, Hq, Hkv, D, splits, device=dev)
+    ctx_all = torch.arange(prompt + 1, total + 1, dtype=torch.int32, device=dev)
+    pos_all = torch.arange(prompt, total, dtype=torch.int32, device=dev)
+    one_req = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def decode_loop():
+        for t in range(steps):
+            jf.jf_kv_quantize_append(pool, pt, one_req, pos_all[t:t + 1], k1, v1, err,
+                                     stream=stream)
+            jf.jf_paged_decode_attn(pool, pt, ctx_all[t:t + 1], q1, scale, o1, dws, splits,
+                                    stream=stream)
+    with torch.cuda.stream(stream):
+        decode_loop()
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graph, stream=stream):
+            decode_loop()
+    t_dec = _event_time(graph.replay, 2, stream)
+    check("decode loop", dws)
+    pos_sum = int((prompt + 1 + total) * steps // 2)
+    bpp = 2 * Hkv * (D // 2 + 4 * D // 64)
+    out["a2a3_decode_6144_steps_32k_to_38k"] = {
+        "ms": t_dec, "us_per_step": t_dec * 1e3 / steps,
+        "positions_per_s": pos_sum / (t_dec / 1e3),
+        "GBps": pos_sum * bpp / (t_dec / 1e3) / 1e9}
+    del graph
+    # a5: checkpoint of all 152 pages
+    blob = torch.empty(npages * pool.page_bytes, dtype=torch.uint8, device=dev)
+    t_ck = _event_time(lambda: jf.jf_kv_checkpoint(pool, pt[0], npages, blob, err,
+                                                   stream=stream), 20, stream)
+    check("checkpoint")
+    ck_bytes = 2 * npages * pool.page_bytes
+    out["a5_checkpoint_152_pages"] = {"us": t_ck * 1e3, "GBps": ck_bytes / (t_ck / 1e3) / 1e9,
+                                      "frac_hbm": ck_bytes / (t_ck / 1e3) / 1e9 / peaks_gbs,
+                                      "alg_bytes": ck_bytes}
+    del pool, blob
+    # ---- two requests, 196,608 + 131,072 positions, 1,280-page pool, 32 splits
+    ctxs = [196608, 131072]
+    gc = synth.generator(3)
+    pt2 = synth.interleaved_page_tables(gc, ctxs, P, 1280).to(dev)
+    pool2 = jf.KVPool.allocate(1280, P, Hkv, D, device=dev, fill=None)
+    for b, c in enumerate(ctxs):
+        for s0 in range(0, c, 65536):
+            n = min(65536, c - s0)
+            kk = torch.randn(n, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+            vv = torch.randn(n, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+            jf.jf_kv_quantize_append(pool2, pt2, torch.full((n,), b, dtype=torch.int32, device=dev),
+                                     torch.arange(s0, s0 + n, dtype=torch.int32, device=dev),
+                                     kk, vv, err, stream=stream)
+    q2 = torch.randn(2, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o2 = torch.empty_like(q2)
+    ws2 = jf.decode_workspace(2, Hq, Hkv, D, 32, device=dev)
+    c2 = torch.tensor(ctxs, dtype=torch.int32, device=dev)
+    t2 = _event_time(lambda: jf.jf_paged_decode_attn(pool2, pt2, c2, q2, scale, o2, ws2, 32,
+                                                     stream=stream), 20, stream)
+    check("two-request", ws2)
+    out["two_request_320k_32_splits"] = {"us": t2 * 1e3, "positions_per_s": sum(ctxs) / (t2 / 1e3),
+                                         "GBps": sum(ctxs) * bpp / (t2 / 1e3) / 1e9}
+    del pool2
+    # ---- 32 requests, contexts uniform in [1,024, 65,536], page size sweep
+    gm = synth.generator(5)
+    ctxm = synth.context_lengths(gm, 32, 1024, 65536)
+    qm = torch.randn(32, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    om = torch.empty_like(qm)
+    cm = torch.tensor(ctxm, dtype=torch.int32, device=dev)
+    sweep = {}
+    for PS in (64, 128, 256):
+        ptm, npm = synth.page_tables(gm, ctxm, PS)
+        ptm = ptm.to(dev)
+        poolm = jf.KVPool.allocate(npm, PS, Hkv, D, device=dev, fill=None)
+        for b, c in enumerate(ctxm):
+            kk = torch.randn(c, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+            vv = torch.randn(c, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+            jf.jf_kv_quantize_append(poolm, ptm, torch.full((c,), b, dtype=torch.int32, device=dev),
+                                     torch.arange(c, dtype=torch.int32, device=dev), kk, vv, err,
+                                     stream=stream)
+        sm_ = jf.default_num_splits(32, Hkv)
+        wsm = jf.decode_workspace(32, Hq, Hkv, D, sm_, device=dev)
+        tm = _event_time(lambda: jf.jf_paged_decode_attn(poolm, ptm, cm, qm, scale, om, wsm, sm_,
+                                                         stream=stream), 20, stream)
+        check(f"mixed batch P={PS}", wsm)
+        sweep[f"page_{PS}"] = {"us": tm * 1e3, "positions_per_s": sum(ctxm) / (tm / 1e3),
+                               "GBps": sum(ctxm) * bpp / (tm / 1e3) / 1e9}
+        del poolm
+    out["mixed_batch_32"] = {"sum_context": sum(ctxm), **sweep}
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -369,6 +553,8 @@ def main():
     ap.add_argument("--layers", type=int, default=64)
     ap.add_argument("--splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--no-rows", dest="rows", action="store_false",
+                    help="skip the append / prefill / checkpoint / multi-request measurements")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     world, rank, local = dist_env()
