@@ -16,18 +16,21 @@
 //    (the G <= 8 heads of the KV head share every K fragment).  Each k-step
 //    stays inside one 64-element group, so a group's partial dot product
 //    acc_g = 2^-24 sum_d q_d n_d is kept apart and the affine fix-up is exact:
-//        s_t = sum_g scale_{t,g} 2^24 acc_g + bias_{t,g} sum_{d in g} q_d.
+//        s_t = sum_g scale_{t,g} 2^24 acc_g + sum_g bias_{t,g} Q_g,
+//    Q_g = sum_{d in g} q_d; the bias term is a bf16 MMA of the bias words
+//    against Q_g split into bf16 high and low parts.
 //  * PV: A = V codes transposed [16 d x 16 positions] (ldmatrix.trans gives the
 //    position pairs), B = p_t * scale_{t,g} as f16 [16 positions x 8 heads]
-//    (the QK accumulator transposed with movmatrix); bias terms accumulate as
-//    sum_t bias_{t,g} p_t in fp32.
-//  * Online softmax in the log2 domain with warp-shuffle maxima; accumulators
-//    are rescaled only when a head's running maximum grows.
+//    (the QK accumulator transposed with movmatrix); the bias term
+//    sum_t bias_{t,g} p_t is one more bf16 MMA.
+//  * Online softmax in the log2 domain.  The reference maximum moves only when
+//    a logit exceeds it by more than 2^DTAU, so the common chunk needs no
+//    cross-lane reduction; the accumulators are rescaled only then.
 // The four warps' states are combined in shared memory and written as one
 // split partial (m, l, O) to the workspace, or straight to the output when
 // num_splits == 1.
 //
-// Kernel 2 (merge).  One CTA per (request, query head) combines the partials:
+// Kernel 2 (merge).  CTAs over (32-wide d slice, query head, request) combine:
 //   o = sum_s 2^{m_s - m*} O_s / sum_s 2^{m_s - m*} l_s.
 #include <cmath>
 #include <cfloat>
@@ -40,6 +43,7 @@ constexpr int DTOK = 32;      // positions per pipeline stage (one chunk)
 constexpr int DWARPS = 4;     // warps per split CTA
 constexpr int DSTAGES = 3;    // stages per warp
 constexpr int MIN_CPS = 16;   // minimum chunks per split (512 positions)
+constexpr float DTAU = 4.f;   // log2 headroom before the reference maximum moves
 
 struct DecodeArgs {
   const uint8_t* pool;
@@ -89,10 +93,32 @@ __device__ __forceinline__ uint32_t swz(int t, int ch) {
     return t * 64 + ((ch ^ ((t >> 1) & 3)) << 4);
 }
 
+// (w >> 8) as an integer multiply-high, which runs on the FMA pipe and spares
+// the ALU pipe that the nibble masks already load.
+__device__ __forceinline__ uint32_t shr8(uint32_t w) { return __umulhi(w, 0x01000000u); }
 __device__ __forceinline__ uint32_t nib0(uint32_t w) { return w & 0x000F000Fu; }
 __device__ __forceinline__ uint32_t nib1(uint32_t w) { return w & 0x00F000F0u; }
-__device__ __forceinline__ uint32_t nib2(uint32_t w) { return (w >> 8) & 0x000F000Fu; }
-__device__ __forceinline__ uint32_t nib3(uint32_t w) { return (w >> 8) & 0x00F000F0u; }
+
+// bf16 MMA (m16n8k16, fp32 accumulate) for the bias terms
+__device__ __forceinline__ void mma_bf16(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                         uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// high halves (the bias bf16 values) of two scale/bias words
+__device__ __forceinline__ uint32_t hi_halves(uint32_t a, uint32_t b) {
+  return __byte_perm(a, b, 0x7632);
+}
 
 template <int D>
 struct DecodeSmem {
@@ -108,7 +134,7 @@ struct DecodeSmem {
   static constexpr int TOTAL = 1024 + CODES_BYTES + SB_BYTES + BAR_BYTES;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
   static_assert(DWARPS * 8 * D * 4 <= CODES_BYTES, "combine buffer must fit");
-  static_assert(DWARPS * 8 * 2 * 4 <= SB_BYTES, "combine ml buffer must fit");
+  static_assert(DWARPS * 8 * (2 + NG) * 4 <= SB_BYTES, "combine ml/bias buffer must fit");
 };
 
 // Per-warp online-softmax state.  Thread (r, c) of the warp owns query heads
@@ -118,13 +144,13 @@ template <int NG>
 struct DecodeState {
   float m0, m1, l0, l1;
   float O[NG][4][4];
-  float Bs[NG][2];
+  float Bs[4];   // bias term sum_t bias_{t,g} p_t (MMA layout: row = group, col = head)
   __device__ __forceinline__ void init() {
     m0 = m1 = -INFINITY;
     l0 = l1 = 0.f;
+    Bs[0] = Bs[1] = Bs[2] = Bs[3] = 0.f;
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
-      Bs[g][0] = Bs[g][1] = 0.f;
 #pragma unroll
       for (int e = 0; e < 4; ++e)
 #pragma unroll
@@ -136,7 +162,7 @@ struct DecodeState {
 template <int NG>
 struct ChunkCtx {
   const uint32_t (&qf)[NG][4][2];
-  const float (&Qh)[NG][2];
+  uint32_t bq;   // B fragment of the QK bias MMA: (Q_g high | low parts) for head r
   float cA, cB;
   int r, c, ld_t, ld_ch;
 };
@@ -178,27 +204,36 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
       uint32_t w0, w1, w2, w3;
       ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
       acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
+      const uint32_t h0 = shr8(w0), h1 = shr8(w1), h2 = shr8(w2), h3 = shr8(w3);
       mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), cc.qf[g][0][0], cc.qf[g][0][1]);
-      mma_f16(acc[g], nib2(w0), nib2(w1), nib3(w0), nib3(w1), cc.qf[g][1][0], cc.qf[g][1][1]);
+      mma_f16(acc[g], nib0(h0), nib0(h1), nib1(h0), nib1(h1), cc.qf[g][1][0], cc.qf[g][1][1]);
       mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), cc.qf[g][2][0], cc.qf[g][2][1]);
-      mma_f16(acc[g], nib2(w2), nib2(w3), nib3(w2), nib3(w3), cc.qf[g][3][0], cc.qf[g][3][1]);
+      mma_f16(acc[g], nib0(h2), nib0(h3), nib1(h2), nib1(h3), cc.qf[g][3][0], cc.qf[g][3][1]);
     }
     uint32_t wa[NG], wb[NG];
     load_sb_words<NG>(ksb + ta * SBB, wa);
     load_sb_words<NG>(ksb + tb * SBB, wb);
-    float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f};
+    // bias term sum_g bias_{t,g} Q_g: A rows = positions, k-slots = groups x (Q high, Q low)
+    float t2[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      uint32_t aa, ab;
+      if constexpr (NG == 4) {
+        aa = (cc.c & 1) ? hi_halves(wa[2], wa[3]) : hi_halves(wa[0], wa[1]);
+        ab = (cc.c & 1) ? hi_halves(wb[2], wb[3]) : hi_halves(wb[0], wb[1]);
+      } else {
+        aa = (cc.c < 2) ? hi_halves(wa[0], wa[1]) : 0u;
+        ab = (cc.c < 2) ? hi_halves(wb[0], wb[1]) : 0u;
+      }
+      mma_bf16(t2, aa, ab, 0u, 0u, cc.bq, 0u);
+    }
+    float t1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
-      const float sa = bf16lo_to_f32(wa[g]), ba = bf16hi_to_f32(wa[g]);
-      const float sbv = bf16lo_to_f32(wb[g]), bbv = bf16hi_to_f32(wb[g]);
+      const float sa = bf16lo_to_f32(wa[g]), sbv = bf16lo_to_f32(wb[g]);
       t1[0] = fmaf(sa, acc[g][0], t1[0]);
       t1[1] = fmaf(sa, acc[g][1], t1[1]);
       t1[2] = fmaf(sbv, acc[g][2], t1[2]);
       t1[3] = fmaf(sbv, acc[g][3], t1[3]);
-      t2[0] = fmaf(ba, cc.Qh[g][0], t2[0]);
-      t2[1] = fmaf(ba, cc.Qh[g][1], t2[1]);
-      t2[2] = fmaf(bbv, cc.Qh[g][0], t2[2]);
-      t2[3] = fmaf(bbv, cc.Qh[g][1], t2[3]);
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) sc[j][i] = fmaf(t1[i], cc.cA, t2[i] * cc.cB);
@@ -208,16 +243,16 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
     }
   }
 
-  // ---- online softmax over the 32 positions of this chunk -------------
+  // ---- online softmax with a lazily moved reference maximum -------------
   float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][2]), fmaxf(sc[1][0], sc[1][2]));
   float mx1 = fmaxf(fmaxf(sc[0][1], sc[0][3]), fmaxf(sc[1][1], sc[1][3]));
+  if (__any_sync(0xffffffffu, (mx0 > st.m0 + DTAU) || (mx1 > st.m1 + DTAU))) {
 #pragma unroll
-  for (int o = 4; o < 32; o <<= 1) {
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-  }
-  const float nm0 = fmaxf(st.m0, mx0), nm1 = fmaxf(st.m1, mx1);
-  if (__any_sync(0xffffffffu, (nm0 > st.m0) || (nm1 > st.m1))) {
+    for (int o = 4; o < 32; o <<= 1) {
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+    }
+    const float nm0 = fmaxf(st.m0, mx0), nm1 = fmaxf(st.m1, mx1);
     const float f0 = (nm0 > st.m0) ? fast_exp2(st.m0 - nm0) : 1.f;
     const float f1 = (nm1 > st.m1) ? fast_exp2(st.m1 - nm1) : 1.f;
 #pragma unroll
@@ -227,9 +262,9 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
         st.O[g][e][0] *= f0; st.O[g][e][2] *= f0;
         st.O[g][e][1] *= f1; st.O[g][e][3] *= f1;
       }
-      st.Bs[g][0] *= f0;
-      st.Bs[g][1] *= f1;
     }
+    st.Bs[0] *= f0; st.Bs[2] *= f0;
+    st.Bs[1] *= f1; st.Bs[3] *= f1;
     st.l0 *= f0;
     st.l1 *= f1;
     st.m0 = nm0;
@@ -265,24 +300,46 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
       va = ta < nvalid;
       vb = tb < nvalid;
     }
+    // bias term: A rows = groups (r < NG), k-slots = positions 2c, 2c+1, 2c+8, 2c+9
+    {
+      uint32_t a0 = 0, a2 = 0;
+      if (r < NG) {
+        const uint8_t* base = vsb + (16 * j + 2 * cc.c) * SBB + r * 4;
+        uint32_t x0 = *reinterpret_cast<const uint32_t*>(base);
+        uint32_t x1 = *reinterpret_cast<const uint32_t*>(base + SBB);
+        uint32_t x2 = *reinterpret_cast<const uint32_t*>(base + 8 * SBB);
+        uint32_t x3 = *reinterpret_cast<const uint32_t*>(base + 9 * SBB);
+        if constexpr (!FULL) {
+          const int t0 = 16 * j + 2 * cc.c;
+          if (t0 >= nvalid) x0 = 0;
+          if (t0 + 1 >= nvalid) x1 = 0;
+          if (t0 + 8 >= nvalid) x2 = 0;
+          if (t0 + 9 >= nvalid) x3 = 0;
+        }
+        a0 = hi_halves(x0, x1);
+        a2 = hi_halves(x2, x3);
+      }
+      const uint32_t pb0 = movm_t(pack_bf16x2(p[j][0], p[j][1]));
+      const uint32_t pb1 = movm_t(pack_bf16x2(p[j][2], p[j][3]));
+      mma_bf16(st.Bs, a0, 0u, a2, 0u, pb0, pb1);
+    }
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
-      float sva = bf16lo_to_f32(wa[g]), bva = bf16hi_to_f32(wa[g]);
-      float svb = bf16lo_to_f32(wb[g]), bvb = bf16hi_to_f32(wb[g]);
+      float sva = bf16lo_to_f32(wa[g]);
+      float svb = bf16lo_to_f32(wb[g]);
       if constexpr (!FULL) {
-        if (!va) sva = bva = 0.f;
-        if (!vb) svb = bvb = 0.f;
+        if (!va) sva = 0.f;
+        if (!vb) svb = 0.f;
       }
-      st.Bs[g][0] = fmaf(bva, p[j][0], fmaf(bvb, p[j][2], st.Bs[g][0]));
-      st.Bs[g][1] = fmaf(bva, p[j][1], fmaf(bvb, p[j][3], st.Bs[g][1]));
       const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
       const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
       uint32_t v0, v1, v2, v3;
       ldsm_x4_t(v0, v1, v2, v3, vc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
+      const uint32_t h0 = shr8(v0), h1 = shr8(v1), h2 = shr8(v2), h3 = shr8(v3);
       mma_f16(st.O[g][0], nib0(v0), nib0(v2), nib0(v1), nib0(v3), b0, b1);
       mma_f16(st.O[g][1], nib1(v0), nib1(v2), nib1(v1), nib1(v3), b0, b1);
-      mma_f16(st.O[g][2], nib2(v0), nib2(v2), nib2(v1), nib2(v3), b0, b1);
-      mma_f16(st.O[g][3], nib3(v0), nib3(v2), nib3(v1), nib3(v3), b0, b1);
+      mma_f16(st.O[g][2], nib0(h0), nib0(h2), nib0(h1), nib0(h3), b0, b1);
+      mma_f16(st.O[g][3], nib1(h0), nib1(h2), nib1(h1), nib1(h3), b0, b1);
     }
   }
 }
@@ -306,6 +363,9 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
   const bool direct = (a.num_splits == 1);
+  // launched with programmatic dependent launch: wait for the previous
+  // kernel (e.g. the append that wrote the newest position) before any read
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
   const int ctx = checked_ctx(a, b);
   int nch, cps, nsplit;
@@ -366,7 +426,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
 #pragma unroll
     for (int i = 0; i < 8; ++i) { e[2 * i] = bf16lo_to_f32(ws[i]); e[2 * i + 1] = bf16hi_to_f32(ws[i]); }
     // word W covers d = base..base+7; nib0 -> (base, base+4), nib1 -> (base+1, base+5) x16,
-    // nib2 -> (base+2, base+6), nib3 -> (base+3, base+7) x16
+    // nib0 of W>>8 -> (base+2, base+6), nib1 of W>>8 -> (base+3, base+7) x16
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const float* x = e + 8 * h;
@@ -382,11 +442,25 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     sum += __shfl_xor_sync(0xffffffffu, sum, 2);
     Qg[g] = sum;
   }
-  float Qh[NG][2];
+  // QK bias B fragment for head r: k-slot k < NG is Q_k high, NG <= k < 2 NG
+  // is Q_{k-NG} low (the bf16 residual); thread c holds slots 2c, 2c+1.
+  uint32_t bq = 0;
+  {
+    float hi[NG], lo[NG];
 #pragma unroll
-  for (int g = 0; g < NG; ++g) {
-    Qh[g][0] = __shfl_sync(0xffffffffu, Qg[g], (2 * c) * 4);
-    Qh[g][1] = __shfl_sync(0xffffffffu, Qg[g], (2 * c + 1) * 4);
+    for (int g = 0; g < NG; ++g) {
+      hi[g] = __bfloat162float(__float2bfloat16_rn(Qg[g]));
+      lo[g] = Qg[g] - hi[g];
+    }
+    if constexpr (NG == 4) {
+      if (c == 0) bq = pack_bf16x2(hi[0], hi[1]);
+      else if (c == 1) bq = pack_bf16x2(hi[2], hi[3]);
+      else if (c == 2) bq = pack_bf16x2(lo[0], lo[1]);
+      else bq = pack_bf16x2(lo[2], lo[3]);
+    } else {
+      if (c == 0) bq = pack_bf16x2(hi[0], hi[1]);
+      else if (c == 1) bq = pack_bf16x2(lo[0], lo[1]);
+    }
   }
   const float cA = a.scale_log2 * 16777216.f * ldexpf(1.f, qe);
   const float cB = a.scale_log2;
@@ -446,7 +520,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   // ldmatrix row address pieces: matrix m = lane>>3 -> (position half, chunk)
   const int ld_t = (lane & 7) + 8 * ((lane >> 3) & 1);
   const int ld_ch = lane >> 4;
-  const ChunkCtx<NG> cc{qf, Qh, cA, cB, r, c, ld_t, ld_ch};
+  const ChunkCtx<NG> cc{qf, bq, cA, cB, r, c, ld_t, ld_ch};
 
   int done = 0;
   for (int it = 0; it < my_n; ++it) {
@@ -482,18 +556,22 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   float& l0 = st.l0;
   float& l1 = st.l1;
   auto& O = st.O;
-  auto& Bs = st.Bs;
+
+  // the merge kernel may start launching; it waits for this grid to finish
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
   // ---- per-warp finalize ---------------------------------------------------
 #pragma unroll
   for (int o = 4; o < 32; o <<= 1) {
     l0 += __shfl_xor_sync(0xffffffffu, l0, o);
     l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+  }
+  // bias sums: lane (r = g, c) of the MMA accumulator holds group g, heads 2c, 2c+1
+  float Bs[NG][2];
 #pragma unroll
-    for (int g = 0; g < NG; ++g) {
-      Bs[g][0] += __shfl_xor_sync(0xffffffffu, Bs[g][0], o);
-      Bs[g][1] += __shfl_xor_sync(0xffffffffu, Bs[g][1], o);
-    }
+  for (int g = 0; g < NG; ++g) {
+    Bs[g][0] = __shfl_sync(0xffffffffu, st.Bs[0], g * 4 + c);
+    Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
   }
   __syncthreads();   // every warp is past its last stage: reuse the rings
   float* so = reinterpret_cast<float*>(codes);    // [DWARPS][8][D]
@@ -555,61 +633,65 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   }
 }
 
+// One CTA per (32-wide slice of head_dim, query head, request); its 8 warps
+// take interleaved splits and reduce through shared memory, so the merge is
+// spread over the whole GPU and each thread issues only a few loads.
+constexpr int MERGE_THREADS = 256;
+constexpr int MERGE_DSLICE = 32;
+
 template <int D>
-__global__ void __launch_bounds__(1024) decode_merge_kernel(const DecodeArgs a) {
-  constexpr int X = D / 4;
-  constexpr int Y = 1024 / X;
-  extern __shared__ float msm[];   // [2*S padded to 4] ml, then [Y][X] float4
-  const int hq = blockIdx.x, b = blockIdx.y;
-  const int tid = threadIdx.x;
+__global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const DecodeArgs a) {
+  constexpr int NSG = MERGE_THREADS / MERGE_DSLICE;   // split groups
+  __shared__ float red[NSG][MERGE_DSLICE];
+  __shared__ float sM, sL;
+  // the split kernel's partials must be complete and visible
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  const int d0 = blockIdx.x * MERGE_DSLICE, hq = blockIdx.y, b = blockIdx.z;
+  const int t = threadIdx.x, dd = t % MERGE_DSLICE, sg = t / MERGE_DSLICE;
   const int ctx = checked_ctx(a, b);
   int nch, cps, nsplit;
   split_plan(ctx, a.num_splits, nch, cps, nsplit);
-  uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D;
+  uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D + d0;
   if (nsplit == 0) {
-    if (tid < D) orow[tid] = 0;
+    if (t < MERGE_DSLICE) orow[t] = 0;
     return;
   }
   const int64_t row0 = ((int64_t)b * a.Hq + hq) * a.num_splits;
-  for (int i = tid; i < 2 * nsplit; i += blockDim.x) msm[i] = a.part_ml[row0 * 2 + i];
+  const float2* ml = reinterpret_cast<const float2*>(a.part_ml) + row0;
+  if (t < 32) {   // warp 0: global max and normalizer
+    float M = -INFINITY;
+    for (int s = t; s < nsplit; s += 32) M = fmaxf(M, ml[s].x);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float L = 0.f;
+    if (M != -INFINITY)
+      for (int s = t; s < nsplit; s += 32) {
+        const float2 v = ml[s];
+        if (v.x != -INFINITY) L = fmaf(fast_exp2(v.x - M), v.y, L);
+      }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (t == 0) { sM = M; sL = L; }
+  }
   __syncthreads();
-  float M = -INFINITY;
-  for (int s = 0; s < nsplit; ++s) M = fmaxf(M, msm[2 * s]);
-  const int x = tid % X, y = tid / X;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  float Lsum = 0.f;
+  const float M = sM;
+  float acc = 0.f;
   if (M != -INFINITY) {
-    for (int s = 0; s < nsplit; ++s) {
-      const float ms = msm[2 * s];
-      if (ms != -INFINITY) Lsum = fmaf(fast_exp2(ms - M), msm[2 * s + 1], Lsum);
-    }
 #pragma unroll 4
-    for (int s = y; s < nsplit; s += Y) {
-      const float ms = msm[2 * s];
+    for (int s = sg; s < nsplit; s += NSG) {
+      const float ms = ml[s].x;
       if (ms == -INFINITY) continue;
-      const float f = fast_exp2(ms - M);
-      const float4 o = *reinterpret_cast<const float4*>(a.part_o + (row0 + s) * D + 4 * x);
-      acc.x = fmaf(f, o.x, acc.x);
-      acc.y = fmaf(f, o.y, acc.y);
-      acc.z = fmaf(f, o.z, acc.z);
-      acc.w = fmaf(f, o.w, acc.w);
+      acc = fmaf(fast_exp2(ms - M), a.part_o[(row0 + s) * D + d0 + dd], acc);
     }
   }
-  float4* red = reinterpret_cast<float4*>(msm + ((2 * a.num_splits + 3) & ~3));
-  red[y * X + x] = acc;
+  red[sg][dd] = acc;
   __syncthreads();
-  if (y == 0) {
-    float4 t = red[x];
-    for (int yy = 1; yy < Y; ++yy) {
-      const float4 u = red[yy * X + x];
-      t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
-    }
-    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-    const uint32_t lo = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.x * inv)) |
-                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.y * inv)) << 16);
-    const uint32_t hi = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.z * inv)) |
-                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(t.w * inv)) << 16);
-    *reinterpret_cast<uint2*>(orow + 4 * x) = make_uint2(lo, hi);
+  if (t < MERGE_DSLICE) {
+    float o = 0.f;
+#pragma unroll
+    for (int k = 0; k < NSG; ++k) o += red[k][t];
+    const float L = sL;
+    orow[t] = __bfloat16_as_ushort(__float2bfloat16_rn(L > 0.f ? o / L : 0.f));
   }
 }
 
@@ -633,18 +715,29 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
       return JF_ERR_CUDA;
     attr_done = true;
   }
-  dim3 grid((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
-  decode_split_kernel<D><<<grid, DWARPS * 32, L::TOTAL, stream>>>(tmap, a);
-  if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  // Both kernels use programmatic dependent launch: each may be scheduled
+  // while the previous kernel in the stream drains, and waits (griddepcontrol)
+  // before it reads anything that kernel wrote.
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
+  cfg.blockDim = dim3(DWARPS * 32);
+  cfg.dynamicSmemBytes = L::TOTAL;
+  cfg.stream = stream;
+  cfg.attrs = pdl;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, decode_split_kernel<D>, tmap, a) != cudaSuccess) return JF_ERR_CUDA;
   if (a.num_splits > 1) {
-    const size_t smem = (size_t)((2 * a.num_splits + 3) & ~3) * 4 + 1024 * 16;
-    if (smem > 48 * 1024) {
-      if (cudaFuncSetAttribute(decode_merge_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)smem) != cudaSuccess)
-        return JF_ERR_CUDA;
-    }
-    decode_merge_kernel<D><<<dim3((unsigned)a.Hq, (unsigned)B), 1024, smem, stream>>>(a);
-    if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+    cudaLaunchConfig_t mc = {};
+    mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.Hq, (unsigned)B);
+    mc.blockDim = dim3(MERGE_THREADS);
+    mc.dynamicSmemBytes = 0;
+    mc.stream = stream;
+    mc.attrs = pdl;
+    mc.numAttrs = 1;
+    if (cudaLaunchKernelEx(&mc, decode_merge_kernel<D>, a) != cudaSuccess) return JF_ERR_CUDA;
   }
   return JF_OK;
 }
