@@ -2,7 +2,7 @@
 // decode reads the compressed pages where they are used; Sec. 2, Eq. 3: never
 // size temporaries by the history length; Eq. 5: contiguous GQA head groups).
 //
-// Kernel 1 (split phase).  CTA = (split s, KV head, request b), 4 warps.  The
+// Kernel 1 (split phase).  CTA = (split s, KV head, request b), 6 warps.  The
 // split's 32-position chunks are dealt round-robin to the warps; each warp owns
 // a private ring of DSTAGES shared-memory stages that it refills itself with
 // TMA: a 5-D tiled copy (128-byte swizzle) for the K and V code rows of the
@@ -40,8 +40,8 @@
 namespace jfkv {
 
 constexpr int DTOK = 32;      // positions per pipeline stage (one chunk)
-constexpr int DWARPS = 4;     // warps per split CTA
-constexpr int DSTAGES = 3;    // stages per warp
+constexpr int DWARPS = 6;     // warps per split CTA (2 CTAs per SM)
+constexpr int DSTAGES = 2;    // stages per warp
 constexpr int MIN_CPS = 16;   // minimum chunks per split (512 positions)
 constexpr float DTAU = 4.f;   // log2 headroom before the reference maximum moves
 
@@ -130,8 +130,11 @@ struct DecodeSmem {
   static constexpr int NBUF = DWARPS * DSTAGES;
   static constexpr int CODES_BYTES = NBUF * 2 * CODE_BUF;
   static constexpr int SB_BYTES = NBUF * 2 * SB_BUF;
+  static constexpr int QF_BYTES = NG * 2 * 32 * 16;   // query fragments [g][half][lane][4]
   static constexpr int BAR_BYTES = NBUF * 8;
-  static constexpr int TOTAL = 1024 + CODES_BYTES + SB_BYTES + BAR_BYTES;
+  // The dynamic shared window starts 1024-byte aligned (checked at run time),
+  // which the 128-byte TMA swizzle of the code buffers needs.
+  static constexpr int TOTAL = CODES_BYTES + SB_BYTES + QF_BYTES + BAR_BYTES;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
   static_assert(DWARPS * 8 * D * 4 <= CODES_BYTES, "combine buffer must fit");
   static_assert(DWARPS * 8 * (2 + NG) * 4 <= SB_BYTES, "combine ml/bias buffer must fit");
@@ -161,7 +164,7 @@ struct DecodeState {
 
 template <int NG>
 struct ChunkCtx {
-  const uint32_t (&qf)[NG][4][2];
+  const uint4* qf;   // this lane's query fragments: qf[2 g + half] = k-steps 2 half, 2 half + 1
   uint32_t bq;   // B fragment of the QK bias MMA: (Q_g high | low parts) for head r
   float cA, cB;
   int r, c, ld_t, ld_ch;
@@ -201,14 +204,15 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
     float acc[NG][4];
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
+      const uint4 qa = cc.qf[(2 * g) * 32], qb = cc.qf[(2 * g + 1) * 32];
       uint32_t w0, w1, w2, w3;
       ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
       acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
       const uint32_t h0 = shr8(w0), h1 = shr8(w1), h2 = shr8(w2), h3 = shr8(w3);
-      mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), cc.qf[g][0][0], cc.qf[g][0][1]);
-      mma_f16(acc[g], nib0(h0), nib0(h1), nib1(h0), nib1(h1), cc.qf[g][1][0], cc.qf[g][1][1]);
-      mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), cc.qf[g][2][0], cc.qf[g][2][1]);
-      mma_f16(acc[g], nib0(h2), nib0(h3), nib1(h2), nib1(h3), cc.qf[g][3][0], cc.qf[g][3][1]);
+      mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), qa.x, qa.y);
+      mma_f16(acc[g], nib0(h0), nib0(h1), nib1(h0), nib1(h1), qa.z, qa.w);
+      mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), qb.x, qb.y);
+      mma_f16(acc[g], nib0(h2), nib0(h3), nib1(h2), nib1(h3), qb.z, qb.w);
     }
     uint32_t wa[NG], wb[NG];
     load_sb_words<NG>(ksb + ta * SBB, wa);
@@ -352,12 +356,11 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   constexpr int SBB = L::SBB;
   constexpr float NEG_INF = -INFINITY;
 
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                             ~static_cast<uintptr_t>(1023));
-  uint8_t* codes = smem;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* codes = smem_raw;
   uint8_t* sbuf = codes + L::CODES_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES);
+  uint4* qsm = reinterpret_cast<uint4*>(sbuf + L::SB_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES + L::QF_BYTES);
 
   const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -381,6 +384,10 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const int c_end = min(c_begin + cps, nch);
   const int my_n = (c_end - c_begin > warp) ? (c_end - c_begin - warp + DWARPS - 1) / DWARPS : 0;
 
+  if (smem_u32(smem_raw) & 1023) {   // the swizzled TMA boxes need 1024-byte alignment
+    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
+    return;
+  }
   if (threadIdx.x == 0) prefetch_tensormap(&tmap);
   if (lane == 0) {
     for (int s = 0; s < DSTAGES; ++s) mbar_init(&bars[warp * DSTAGES + s], 1);
@@ -520,7 +527,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   // ldmatrix row address pieces: matrix m = lane>>3 -> (position half, chunk)
   const int ld_t = (lane & 7) + 8 * ((lane >> 3) & 1);
   const int ld_ch = lane >> 4;
-  const ChunkCtx<NG> cc{qf, bq, cA, cB, r, c, ld_t, ld_ch};
+  if (warp == 0) {
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      qsm[(2 * g) * 32 + lane] = make_uint4(qf[g][0][0], qf[g][0][1], qf[g][1][0], qf[g][1][1]);
+      qsm[(2 * g + 1) * 32 + lane] = make_uint4(qf[g][2][0], qf[g][2][1], qf[g][3][0], qf[g][3][1]);
+    }
+  }
+  __syncthreads();
+  const ChunkCtx<NG> cc{qsm + lane, bq, cA, cB, r, c, ld_t, ld_ch};
 
   int done = 0;
   for (int it = 0; it < my_n; ++it) {
