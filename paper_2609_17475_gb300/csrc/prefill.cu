@@ -13,17 +13,23 @@
 //   warp 0      TMEM allocation; lane 0 issues every tcgen05.mma:
 //                 S_j  = Q  K_j^T   (A = Q smem, B = K_j smem, both K-major)
 //                 O   += P_j V_j    (A = P_j in TMEM, B = V_j smem, MN-major)
-//   warps 1-4   dequantize 64-position K/V tiles from the pool (page-table
+//   warps 1-8   dequantize 64-position K/V tiles from the pool (page-table
 //               lookup, 4-bit codes -> fp16 via an e4m3 convert, then
 //               x = code * scale + bias with one fused multiply-add) into
-//               double-buffered 128B-swizzled tiles;
-//   warps 5-8   one thread per row: online softmax on S (tcgen05.ld), P back
+//               double-buffered 128B-swizzled tiles; each thread owns one
+//               position's 32 contiguous code bytes per 64-wide block, loads
+//               run two tiles ahead, and the 8 lanes of a quarter-warp store
+//               8 different positions (distinct swizzled chunks, no bank
+//               conflicts);
+//   warps 9-12  one thread per row: online softmax on S (tcgen05.ld), P back
 //               to TMEM as fp16 (tcgen05.st); the running maximum is moved
 //               only when it grows by more than 2^8, and then O is rescaled
 //               in TMEM; finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
 // 0,2,4,6,1,3,5,7 (what the two-nibble convert produces); Q uses the same
-// order, so Q K^T is unchanged, and the epilogue undoes it for O.
+// order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
+// stored pre-multiplied by softmax_scale * log2(e), so S arrives in the log2
+// domain.
 #include <cmath>
 
 #include "tc.cuh"
@@ -32,7 +38,7 @@ namespace jfkv {
 
 constexpr int PF_BM = 128;   // MMA rows per CTA
 constexpr int PF_BN = 64;    // positions per K/V tile
-constexpr int PF_DQ_WARPS = 4;
+constexpr int PF_DQ_WARPS = 8;
 constexpr int PF_SM_WARPS = 4;
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
@@ -100,10 +106,25 @@ __device__ __forceinline__ uint4 dequant8(uint32_t w, uint32_t s2, uint32_t b2) 
   return o;
 }
 
-// bf16 (scale | bias << 16) word -> f16x2 broadcasts of scale and bias
-__device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2) {
+// Same with the *512 folded into the scale (scale * 512 must fit fp16).
+__device__ __forceinline__ uint4 dequant8_fast(uint32_t w, uint32_t s512, uint32_t b2) {
+  const uint32_t lo = w & 0x0F0F0F0Fu;
+  const uint32_t hi = (w >> 4) & 0x0F0F0F0Fu;
+  uint4 o;
+  o.x = hfma2(cvt_e4m3x2_f16x2(lo & 0xFFFFu), s512, b2);
+  o.y = hfma2(cvt_e4m3x2_f16x2(lo >> 16), s512, b2);
+  o.z = hfma2(cvt_e4m3x2_f16x2(hi & 0xFFFFu), s512, b2);
+  o.w = hfma2(cvt_e4m3x2_f16x2(hi >> 16), s512, b2);
+  return o;
+}
+
+// bf16 (scale | bias << 16) word -> f16x2 broadcasts of scale (or scale*512
+// when that fits fp16: fast = true) and bias
+__device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2, bool& fast) {
   const float s = bf16lo_to_f32(w), b = bf16hi_to_f32(w);
-  s2 = pack_f16x2(s, s);
+  fast = fabsf(s) <= 120.f;
+  const float sc = fast ? s * 512.f : s;
+  s2 = pack_f16x2(sc, sc);
   b2 = pack_f16x2(b, b);
 }
 
@@ -113,10 +134,8 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   constexpr int NKB = D / 64;           // 64-wide d blocks
   constexpr int CB = D / 2;
   constexpr int SBB = D / 16;
-  constexpr int HPK = D / 32;           // 16-byte code items per position
-  constexpr int ITEMS = PF_BN * HPK;    // per tile, for K or V
-  constexpr int IPT = ITEMS / (32 * PF_DQ_WARPS);
-  static_assert(ITEMS % (32 * PF_DQ_WARPS) == 0, "items per thread");
+  constexpr int UPI = (D == 256) ? 2 : 1;   // 16-byte code units per dequant item
+  static_assert(PF_BN * NKB * 2 / UPI == 32 * PF_DQ_WARPS, "one item per dequant thread");
   constexpr uint32_t IDQK = tc::idesc_f16_f32(PF_BM, PF_BN, 0, 0);
   constexpr uint32_t IDPV = tc::idesc_f16_f32(PF_BM, D, 0, 1);
 
@@ -158,14 +177,15 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   __syncthreads();
 
   // ---- Q tile -> fp16, 128B-swizzled K-major, d order 0,2,4,6,1,3,5,7 ------
-  const int ltid = (int)threadIdx.x - 32;          // 0..255 for warps 1..8
+  const int ltid = (int)threadIdx.x - 32;          // 0..383 for warps 1..12
+  constexpr int QTHREADS = PF_THREADS - 32;
   constexpr int QITEMS = PF_BM * (D / 8);
   auto q_src = [&](int r) -> const uint16_t* {
     return a.q + ((int64_t)(q0 + r / a.G) * a.Hq + kvh * a.G + r % a.G) * D;
   };
   if (warp > 0) {
     float mx = 0.f;
-    for (int it = ltid; it < QITEMS; it += 256) {
+    for (int it = ltid; it < QITEMS; it += QTHREADS) {
       const int r = it / (D / 8), c8 = it % (D / 8);
       if (r < rows) {
         const uint4 w = *reinterpret_cast<const uint4*>(q_src(r) + 8 * c8);
@@ -180,11 +200,13 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     if (lane == 0) atomicMax(qmax_slot, __float_as_uint(mx));
   }
   __syncthreads();
-  const float qmax = __uint_as_float(*qmax_slot);
+  // Q enters fp16 pre-multiplied by softmax_scale * log2(e); a power of two
+  // keeps it below 2^14 and is multiplied back onto S.
+  const float qmax = __uint_as_float(*qmax_slot) * a.scale_log2;
   const int qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
   if (warp > 0) {
-    const float qs = ldexpf(1.f, -qe);
-    for (int it = ltid; it < QITEMS; it += 256) {
+    const float qs = ldexpf(a.scale_log2, -qe);
+    for (int it = ltid; it < QITEMS; it += QTHREADS) {
       const int r = it / (D / 8), c8 = it % (D / 8);
       uint4 o = make_uint4(0, 0, 0, 0);
       if (r < rows) {
@@ -250,76 +272,76 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     __syncwarp();
   } else if (warp <= PF_DQ_WARPS) {
     // ================= dequantization =================
-    const int dt = (int)threadIdx.x - 32;   // 0..127
-    uint4 kc[IPT], vc[IPT], kn[IPT], vn[IPT];
-    uint32_t ks[IPT], vs[IPT], ksn[IPT], vsn[IPT];
-    bool page_ok = true, page_okn = true;
-    auto load_tile = [&](int j, uint4 (&kx)[IPT], uint4 (&vx)[IPT], uint32_t (&ksx)[IPT],
-                         uint32_t (&vsx)[IPT], bool& pok) {
+    // item = (position t, 64-wide block kb[, half u]): UPI 16-byte code units
+    const int dt = (int)threadIdx.x - 32;   // 0 .. 32*PF_DQ_WARPS-1
+    const int t = dt % PF_BN;
+    const int rest = dt / PF_BN;
+    const int kb = (UPI == 2) ? rest : rest >> 1;
+    const int u0 = (UPI == 2) ? 0 : (rest & 1);
+    struct Tile {
+      uint4 k[UPI], v[UPI];
+      uint32_t ks, vs;
+      bool valid;
+    };
+    auto load_tile = [&](int j, Tile& x) {
       const int key0 = j * PF_BN;
       const int page = __ldg(a.pt + key0 / a.P);
-      const int slot0 = key0 % a.P;
-      pok = page >= 0 && page < a.num_pages;
-      const uint8_t* base = a.pool + (int64_t)(pok ? page : 0) * a.page_bytes;
+      const bool pok = page >= 0 && page < a.num_pages;
+      if (!pok && dt == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+      x.valid = pok && (key0 + t < kmax);
+      if (x.valid) {
+        const uint8_t* base = a.pool + (int64_t)page * a.page_bytes;
+        const int64_t row = (int64_t)kvh * a.P + key0 % a.P + t;
+        const uint8_t* kp = base + row * CB + kb * 32 + u0 * 16;
 #pragma unroll
-      for (int u = 0; u < IPT; ++u) {
-        const int i = dt + 32 * PF_DQ_WARPS * u;
-        const int t = i / HPK, h = i % HPK;
-        const int64_t row = (int64_t)kvh * a.P + slot0 + t;
-        if (pok && key0 + t < kmax) {
-          kx[u] = __ldg(reinterpret_cast<const uint4*>(base + row * CB + h * 16));
-          vx[u] = __ldg(reinterpret_cast<const uint4*>(base + a.codes_region + row * CB + h * 16));
-          ksx[u] = __ldg(reinterpret_cast<const uint32_t*>(base + a.sb_base + row * SBB + (h >> 1) * 4));
-          vsx[u] = __ldg(reinterpret_cast<const uint32_t*>(base + a.sb_base + a.sb_region +
-                                                           row * SBB + (h >> 1) * 4));
+        for (int u = 0; u < UPI; ++u) {
+          x.k[u] = __ldg(reinterpret_cast<const uint4*>(kp + 16 * u));
+          x.v[u] = __ldg(reinterpret_cast<const uint4*>(kp + a.codes_region + 16 * u));
+        }
+        const uint8_t* sp = base + a.sb_base + row * SBB + kb * 4;
+        x.ks = __ldg(reinterpret_cast<const uint32_t*>(sp));
+        x.vs = __ldg(reinterpret_cast<const uint32_t*>(sp + a.sb_region));
+      }
+    };
+    auto store_half = [&](uint8_t* tile, const uint4 (&codes)[UPI], uint32_t sbw, bool valid) {
+      uint32_t s2, b2;
+      bool fast;
+      sb_to_h2(sbw, s2, b2, fast);
+      uint4 o[UPI][4];
+#pragma unroll
+      for (int u = 0; u < UPI; ++u) {
+        const uint32_t cw[4] = {codes[u].x, codes[u].y, codes[u].z, codes[u].w};
+        if (fast) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w) o[u][w] = dequant8_fast(cw[w], s2, b2);
         } else {
-          kx[u] = vx[u] = make_uint4(0, 0, 0, 0);
-          ksx[u] = vsx[u] = 0;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
         }
       }
-    };
-    auto store_tile = [&](int j, const uint4 (&kx)[IPT], const uint4 (&vx)[IPT],
-                          const uint32_t (&ksx)[IPT], const uint32_t (&vsx)[IPT]) {
-      const int b = j & 1;
-      uint8_t* kt = sK + b * L::T_BYTES;
-      uint8_t* vt = sV + b * L::T_BYTES;
 #pragma unroll
-      for (int u = 0; u < IPT; ++u) {
-        const int i = dt + 32 * PF_DQ_WARPS * u;
-        const int t = i / HPK, h = i % HPK;
-        const int kb = h >> 1;
-        uint32_t s2, b2;
-        const uint32_t kw[4] = {kx[u].x, kx[u].y, kx[u].z, kx[u].w};
-        const uint32_t vw[4] = {vx[u].x, vx[u].y, vx[u].z, vx[u].w};
-        sb_to_h2(ksx[u], s2, b2);
+      for (int u = 0; u < UPI; ++u)
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
-          const int cc = (h & 1) * 4 + w;
-          *reinterpret_cast<uint4*>(kt + kb * (PF_BN * 128) + t * 128 + ((cc ^ (t & 7)) << 4)) =
-              dequant8(kw[w], s2, b2);
+          const int cc = (u0 + u) * 4 + w;
+          *reinterpret_cast<uint4*>(tile + kb * (PF_BN * 128) + t * 128 + ((cc ^ (t & 7)) << 4)) =
+              valid ? o[u][w] : make_uint4(0, 0, 0, 0);
         }
-        sb_to_h2(vsx[u], s2, b2);
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const int cc = (h & 1) * 4 + w;
-          *reinterpret_cast<uint4*>(vt + kb * (PF_BN * 128) + t * 128 + ((cc ^ (t & 7)) << 4)) =
-              dequant8(vw[w], s2, b2);
-        }
-      }
     };
-    load_tile(0, kc, vc, ks, vs, page_ok);
+    Tile cur, nxt, nn;
+    load_tile(0, cur);
+    if (ntiles > 1) load_tile(1, nxt);
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
-      if (j + 1 < ntiles) load_tile(j + 1, kn, vn, ksn, vsn, page_okn);
-      if (!page_ok && dt == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+      if (j + 2 < ntiles) load_tile(j + 2, nn);
       if (j >= 2 && !mbar_wait_bounded(&pv_done[j & 1], ((j - 2) >> 1) & 1)) { ok = false; break; }
-      store_tile(j, kc, vc, ks, vs);
+      store_half(sK + (j & 1) * L::T_BYTES, cur.k, cur.ks, cur.valid);
+      store_half(sV + (j & 1) * L::T_BYTES, cur.v, cur.vs, cur.valid);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&kv_full[j & 1]);
-#pragma unroll
-      for (int u = 0; u < IPT; ++u) { kc[u] = kn[u]; vc[u] = vn[u]; ks[u] = ksn[u]; vs[u] = vsn[u]; }
-      page_ok = page_okn;
+      cur = nxt;
+      nxt = nn;
     }
     if (!ok && dt == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
   } else {
@@ -330,7 +352,7 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     const int qi = row_ok ? r / a.G : 0;
     const int limit = !row_ok ? -1 : (a.causal ? a.q_start + q0 + qi : total - 1);
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const float cs = a.scale_log2 * ldexpf(1.f, qe);
+    const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
@@ -344,11 +366,20 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
       const int key0 = j * PF_BN;
       float x[PF_BN];
       float mt = -INFINITY;
+      if (key0 + PF_BN - 1 <= limit) {       // every position of the tile visible
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) * cs : -INFINITY;
-        x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) * cs : -INFINITY;
-        mt = fmaxf(mt, fmaxf(x[c], x[c + 32]));
+        for (int c = 0; c < 32; ++c) {
+          x[c] = __uint_as_float(s0[c]) * smul;
+          x[c + 32] = __uint_as_float(s1[c]) * smul;
+          mt = fmaxf(mt, fmaxf(x[c], x[c + 32]));
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) * smul : -INFINITY;
+          x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) * smul : -INFINITY;
+          mt = fmaxf(mt, fmaxf(x[c], x[c + 32]));
+        }
       }
       const bool need = mt > m_ref + PF_TAU;
       if (__any_sync(0xffffffffu, need)) {
