@@ -11,17 +11,20 @@
 // (query, head) pairs r = i * G + j of the G query heads that share the KV
 // head, so every dequantized K/V tile is reused by all of them.  Warp roles:
 //   warp 0      TMEM allocation; lane 0 issues every tcgen05.mma:
-//                 S_j  = Q  K_j^T   (A = Q smem, B = K_j smem, both K-major)
+//                 S_j  = Q  K_j^T   (A = Q in TMEM, B = K_j smem, K-major)
 //                 O   += P_j V_j    (A = P_j in TMEM, B = V_j smem, MN-major)
+//               TMEM columns: O [0, D), two S/P buffers of 64, Q [D + 128, +D/2);
+//               P_j (fp16) overwrites the first half of S_j once it is read.
 //   warps 1-8   dequantize 64-position K/V tiles from the pool (page-table
 //               lookup, 4-bit codes -> fp16 via an e4m3 convert, then
 //               x = code * scale + bias with one fused multiply-add) into
-//               double-buffered 128B-swizzled tiles; each thread owns one
+//               three 128B-swizzled tile buffers; each thread owns one
 //               position's 32 contiguous code bytes per 64-wide block, loads
 //               run two tiles ahead, and the 8 lanes of a quarter-warp store
 //               8 different positions (distinct swizzled chunks, no bank
 //               conflicts);
-//   warps 9-12  one thread per row: online softmax on S (tcgen05.ld), P back
+//   warps 9-12  one thread per row: Q row -> TMEM at the start; online
+//               softmax on S (tcgen05.ld), P back
 //               to TMEM as fp16 (tcgen05.st); the running maximum is moved
 //               only when it grows by more than 2^8, and then O is rescaled
 //               in TMEM; finally O / l -> bf16 output.
@@ -41,6 +44,7 @@ constexpr int PF_BN = 64;    // positions per K/V tile
 constexpr int PF_DQ_WARPS = 8;
 constexpr int PF_SM_WARPS = 4;
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
+constexpr int PF_KVBUF = 3;     // K/V tile buffers in shared memory
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
 
 struct PrefillArgs {
@@ -62,13 +66,11 @@ struct PrefillArgs {
 
 template <int D>
 struct PfSmem {
-  static constexpr int Q_BYTES = PF_BM * D * 2;
   static constexpr int T_BYTES = PF_BN * D * 2;
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = Q_BYTES;
-  static constexpr int OFF_V = OFF_K + 2 * T_BYTES;
-  static constexpr int OFF_BAR = OFF_V + 2 * T_BYTES;
-  static constexpr int TOTAL = 1024 + OFF_BAR + 128;
+  static constexpr int OFF_K = 0;
+  static constexpr int OFF_V = PF_KVBUF * T_BYTES;
+  static constexpr int OFF_BAR = 2 * PF_KVBUF * T_BYTES;
+  static constexpr int TOTAL = 1024 + OFF_BAR + 256;
 };
 
 __device__ __forceinline__ uint32_t cvt_e4m3x2_f16x2(uint32_t two_bytes) {
@@ -142,16 +144,14 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) &
                                            ~static_cast<uintptr_t>(1023));
-  uint8_t* sQ = sm + L::OFF_Q;
   uint8_t* sK = sm + L::OFF_K;
   uint8_t* sV = sm + L::OFF_V;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::OFF_BAR);
-  uint64_t* kv_full = bars + 0;
-  uint64_t* s_full = bars + 2;
-  uint64_t* p_full = bars + 4;
-  uint64_t* pv_done = bars + 6;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
-  uint32_t* qmax_slot = tmem_slot + 1;
+  uint64_t* kv_full = bars + 0;                // [PF_KVBUF]
+  uint64_t* pv_done = bars + PF_KVBUF;         // [PF_KVBUF]
+  uint64_t* s_full = bars + 2 * PF_KVBUF;      // [2]
+  uint64_t* p_full = bars + 2 * PF_KVBUF + 2;  // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * PF_KVBUF + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = a.n_qtiles - 1 - (int)blockIdx.x;   // latest (longest) query tiles first
@@ -165,105 +165,98 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
 
   if (warp == 0) tc::alloc(tmem_slot, 512);
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < PF_KVBUF; ++i) {
       mbar_init(&kv_full[i], PF_DQ_WARPS);
-      mbar_init(&s_full[i], 1);
-      mbar_init(&p_full[i], PF_SM_WARPS);
       mbar_init(&pv_done[i], 1);
     }
-    *qmax_slot = 0;
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], PF_SM_WARPS);
+    }
     fence_barrier_init();
-  }
-  __syncthreads();
-
-  // ---- Q tile -> fp16, 128B-swizzled K-major, d order 0,2,4,6,1,3,5,7 ------
-  const int ltid = (int)threadIdx.x - 32;          // 0..383 for warps 1..12
-  constexpr int QTHREADS = PF_THREADS - 32;
-  constexpr int QITEMS = PF_BM * (D / 8);
-  auto q_src = [&](int r) -> const uint16_t* {
-    return a.q + ((int64_t)(q0 + r / a.G) * a.Hq + kvh * a.G + r % a.G) * D;
-  };
-  if (warp > 0) {
-    float mx = 0.f;
-    for (int it = ltid; it < QITEMS; it += QTHREADS) {
-      const int r = it / (D / 8), c8 = it % (D / 8);
-      if (r < rows) {
-        const uint4 w = *reinterpret_cast<const uint4*>(q_src(r) + 8 * c8);
-        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          mx = fmaxf(mx, fmaxf(fabsf(bf16lo_to_f32(ws[i])), fabsf(bf16hi_to_f32(ws[i]))));
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    if (lane == 0) atomicMax(qmax_slot, __float_as_uint(mx));
-  }
-  __syncthreads();
-  // Q enters fp16 pre-multiplied by softmax_scale * log2(e); a power of two
-  // keeps it below 2^14 and is multiplied back onto S.
-  const float qmax = __uint_as_float(*qmax_slot) * a.scale_log2;
-  const int qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
-  if (warp > 0) {
-    const float qs = ldexpf(a.scale_log2, -qe);
-    for (int it = ltid; it < QITEMS; it += QTHREADS) {
-      const int r = it / (D / 8), c8 = it % (D / 8);
-      uint4 o = make_uint4(0, 0, 0, 0);
-      if (r < rows) {
-        const uint4 w = *reinterpret_cast<const uint4*>(q_src(r) + 8 * c8);
-        float e[8];
-        e[0] = bf16lo_to_f32(w.x) * qs; e[1] = bf16hi_to_f32(w.x) * qs;
-        e[2] = bf16lo_to_f32(w.y) * qs; e[3] = bf16hi_to_f32(w.y) * qs;
-        e[4] = bf16lo_to_f32(w.z) * qs; e[5] = bf16hi_to_f32(w.z) * qs;
-        e[6] = bf16lo_to_f32(w.w) * qs; e[7] = bf16hi_to_f32(w.w) * qs;
-        o.x = pack_f16x2(e[0], e[2]);
-        o.y = pack_f16x2(e[4], e[6]);
-        o.z = pack_f16x2(e[1], e[3]);
-        o.w = pack_f16x2(e[5], e[7]);
-      }
-      const int kb = c8 / 8, cc = c8 % 8;
-      *reinterpret_cast<uint4*>(sQ + kb * (PF_BM * 128) + r * 128 + ((cc ^ (r & 7)) << 4)) = o;
-    }
-    fence_proxy_async_smem();
   }
   tc::fence_before();
   __syncthreads();
   tc::fence_after();
   const uint32_t tbase = *tmem_slot;
   const uint32_t tO = tbase;
-  const uint32_t tS = tbase + D;
-  const uint32_t tP = tbase + D + 2 * PF_BN;
+  const uint32_t tS = tbase + D;               // two buffers of PF_BN columns
+  const uint32_t tQ = tbase + D + 2 * PF_BN;   // D/2 columns of f16 pairs
+
+  // ---- softmax warps: their Q row -> TMEM (fp16, pre-multiplied by
+  // softmax_scale * log2(e), d order 0,2,4,6,1,3,5,7 in every 8) ------------
+  const int quarter = warp & 3;                // TMEM lanes this warp may access
+  const int r = quarter * 32 + lane;
+  const bool row_ok = r < rows;
+  const int qi = row_ok ? r / a.G : 0;
+  const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+  int qe = 0;                                  // per-row power of two kept out of fp16
+  if (warp > PF_DQ_WARPS) {
+    const uint16_t* qrow = a.q + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
+    float qmax = 0.f;
+    if (row_ok) {
+      for (int c8 = 0; c8 < D / 8; ++c8) {
+        const uint4 w = *reinterpret_cast<const uint4*>(qrow + 8 * c8);
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          qmax = fmaxf(qmax, fmaxf(fabsf(bf16lo_to_f32(ws[k])), fabsf(bf16hi_to_f32(ws[k]))));
+      }
+    }
+    qmax *= a.scale_log2;
+    qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
+    const float qs = ldexpf(a.scale_log2, -qe);
+#pragma unroll 1
+    for (int c0 = 0; c0 < D / 2; c0 += 32) {   // 32 TMEM columns = 64 values = 8 blocks of 8
+      uint32_t v[32];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        uint4 w = make_uint4(0, 0, 0, 0);
+        if (row_ok) w = *reinterpret_cast<const uint4*>(qrow + 2 * c0 + 8 * k);
+        const float e0 = bf16lo_to_f32(w.x) * qs, e1 = bf16hi_to_f32(w.x) * qs;
+        const float e2 = bf16lo_to_f32(w.y) * qs, e3 = bf16hi_to_f32(w.y) * qs;
+        const float e4 = bf16lo_to_f32(w.z) * qs, e5 = bf16hi_to_f32(w.z) * qs;
+        const float e6 = bf16lo_to_f32(w.w) * qs, e7 = bf16hi_to_f32(w.w) * qs;
+        v[4 * k + 0] = pack_f16x2(e0, e2);
+        v[4 * k + 1] = pack_f16x2(e4, e6);
+        v[4 * k + 2] = pack_f16x2(e1, e3);
+        v[4 * k + 3] = pack_f16x2(e5, e7);
+      }
+      tc::st32(tQ + c0 + lane_off, v);
+    }
+    tc::wait_st();
+  }
+  tc::fence_before();
+  __syncthreads();
+  tc::fence_after();
 
   if (warp == 0) {
     // ================= MMA issuer =================
     if (lane == 0) {
-      const uint32_t qaddr = smem_u32(sQ), kaddr = smem_u32(sK), vaddr = smem_u32(sV);
+      const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV);
       bool ok = true;
       auto pv = [&](int j) {
-        const int b = j & 1;
-        if (!mbar_wait_bounded(&p_full[b], (j >> 1) & 1)) { ok = false; return; }
+        const int sb = j & 1, kb = j % PF_KVBUF;
+        if (!mbar_wait_bounded(&p_full[sb], (j >> 1) & 1)) { ok = false; return; }
         tc::fence_after();
 #pragma unroll
         for (int k = 0; k < PF_BN / 16; ++k)
-          tc::mma_ts(tO, tP + b * (PF_BN / 2) + 8 * k,
-                     tc::sdesc_sw128(vaddr + b * L::T_BYTES + k * 2048, PF_BN * 128, 1024), IDPV,
+          tc::mma_ts(tO, tS + sb * PF_BN + 8 * k,
+                     tc::sdesc_sw128(vaddr + kb * L::T_BYTES + k * 2048, PF_BN * 128, 1024), IDPV,
                      (j > 0 || k > 0) ? 1u : 0u);
-        tc::commit(&pv_done[b]);
+        tc::commit(&pv_done[kb]);
       };
       for (int j = 0; j < ntiles && ok; ++j) {
-        const int b = j & 1;
-        if (!mbar_wait_bounded(&kv_full[b], (j >> 1) & 1)) { ok = false; break; }
+        const int sb = j & 1, kb = j % PF_KVBUF;
+        if (!mbar_wait_bounded(&kv_full[kb], (j / PF_KVBUF) & 1)) { ok = false; break; }
         tc::fence_after();
 #pragma unroll
-        for (int kb = 0; kb < NKB; ++kb)
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            tc::mma_ss(tS + b * PF_BN,
-                       tc::sdesc_sw128(qaddr + kb * (PF_BM * 128) + 32 * k, 16, 1024),
-                       tc::sdesc_sw128(kaddr + b * L::T_BYTES + kb * (PF_BN * 128) + 32 * k, 16,
-                                       1024),
-                       IDQK, (kb | k) ? 1u : 0u);
-        tc::commit(&s_full[b]);
+        for (int ks = 0; ks < D / 16; ++ks)
+          tc::mma_ts(tS + sb * PF_BN, tQ + 8 * ks,
+                     tc::sdesc_sw128(kaddr + kb * L::T_BYTES + (ks >> 2) * (PF_BN * 128) +
+                                         (ks & 3) * 32, 16, 1024),
+                     IDQK, ks ? 1u : 0u);
+        tc::commit(&s_full[sb]);
         if (j >= 1) pv(j - 1);
       }
       if (ok) pv(ntiles - 1);
@@ -328,30 +321,36 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
               valid ? o[u][w] : make_uint4(0, 0, 0, 0);
         }
     };
-    Tile cur, nxt, nn;
-    load_tile(0, cur);
-    if (ntiles > 1) load_tile(1, nxt);
+    // Three register tiles rotate by name (the loop is unrolled by 3), so the
+    // loads for tile j + 2 stay in flight while tile j is converted; copying
+    // registers instead would wait for those loads.
+    Tile ta, tb, tcur;
     bool ok = true;
-    for (int j = 0; j < ntiles; ++j) {
-      if (j + 2 < ntiles) load_tile(j + 2, nn);
-      if (j >= 2 && !mbar_wait_bounded(&pv_done[j & 1], ((j - 2) >> 1) & 1)) { ok = false; break; }
-      store_half(sK + (j & 1) * L::T_BYTES, cur.k, cur.ks, cur.valid);
-      store_half(sV + (j & 1) * L::T_BYTES, cur.v, cur.vs, cur.valid);
+    auto step = [&](int j, const Tile& cur, Tile& dst) {
+      if (j + 2 < ntiles) load_tile(j + 2, dst);
+      const int kbuf = j % PF_KVBUF;
+      if (j >= PF_KVBUF &&
+          !mbar_wait_bounded(&pv_done[kbuf], ((j - PF_KVBUF) / PF_KVBUF) & 1)) { ok = false; return; }
+      store_half(sK + kbuf * L::T_BYTES, cur.k, cur.ks, cur.valid);
+      store_half(sV + kbuf * L::T_BYTES, cur.v, cur.vs, cur.valid);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&kv_full[j & 1]);
-      cur = nxt;
-      nxt = nn;
+      if (lane == 0) mbar_arrive(&kv_full[kbuf]);
+    };
+    load_tile(0, ta);
+    if (ntiles > 1) load_tile(1, tb);
+    for (int j = 0; j < ntiles && ok; j += 3) {
+      step(j, ta, tcur);
+      if (j + 1 < ntiles && ok) step(j + 1, tb, ta);
+      if (j + 2 < ntiles && ok) step(j + 2, tcur, tb);
     }
     if (!ok && dt == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
   } else {
     // ================= softmax + epilogue =================
-    const int quarter = warp & 3;                 // TMEM lanes this warp may access
-    const int r = quarter * 32 + lane;
-    const bool row_ok = r < rows;
-    const int qi = row_ok ? r / a.G : 0;
-    const int limit = !row_ok ? -1 : (a.causal ? a.q_start + q0 + qi : total - 1);
-    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    // Rows past the chunk (padding) see every position: their Q rows are zero
+    // and their outputs are never stored, and keeping them unmasked keeps the
+    // warp on the same (mask-free) path as its real rows.
+    const int limit = (row_ok && a.causal) ? a.q_start + q0 + qi : kmax - 1;
     const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
@@ -366,27 +365,38 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
       const int key0 = j * PF_BN;
       float x[PF_BN];
       float mt = -INFINITY;
-      if (key0 + PF_BN - 1 <= limit) {       // every position of the tile visible
+      {
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        if (key0 + PF_BN - 1 <= limit) {       // every position of the tile visible
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          x[c] = __uint_as_float(s0[c]) * smul;
-          x[c + 32] = __uint_as_float(s1[c]) * smul;
-          mt = fmaxf(mt, fmaxf(x[c], x[c + 32]));
-        }
-      } else {
+          for (int c = 0; c < 32; ++c) {
+            x[c] = __uint_as_float(s0[c]);
+            x[c + 32] = __uint_as_float(s1[c]);
+          }
+        } else {
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) * smul : -INFINITY;
-          x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) * smul : -INFINITY;
-          mt = fmaxf(mt, fmaxf(x[c], x[c + 32]));
+          for (int c = 0; c < 32; ++c) {
+            x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) : -INFINITY;
+            x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) : -INFINITY;
+          }
         }
+        if (qe != 0) {
+#pragma unroll
+          for (int c = 0; c < PF_BN; ++c) x[c] *= smul;
+        }
+#pragma unroll
+        for (int c = 0; c < PF_BN; ++c) m4[c & 3] = fmaxf(m4[c & 3], x[c]);
+        mt = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       }
       const bool need = mt > m_ref + PF_TAU;
       if (__any_sync(0xffffffffu, need)) {
         const float nref = need ? mt : m_ref;
         const float f = (need && m_ref != -INFINITY) ? fast_exp2(m_ref - nref) : 1.f;
         if (j > 0) {
-          if (!mbar_wait_bounded(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1)) { ok = false; break; }
+          if (!mbar_wait_bounded(&pv_done[(j - 1) % PF_KVBUF], ((j - 1) / PF_KVBUF) & 1)) {
+            ok = false;
+            break;
+          }
           tc::fence_after();
 #pragma unroll 1
           for (int c0 = 0; c0 < D; c0 += 32) {
@@ -402,21 +412,25 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
         m_ref = nref;
       }
       uint32_t p[32];
+      float l4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < 32; ++c) {
-        const float p0 = (x[2 * c] == -INFINITY) ? 0.f : fast_exp2(x[2 * c] - m_ref);
-        const float p1 = (x[2 * c + 1] == -INFINITY) ? 0.f : fast_exp2(x[2 * c + 1] - m_ref);
-        l += p0 + p1;
+        // -inf - m_ref -> exp2 = 0; m_ref is finite once any position was visible
+        const float p0 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c] - m_ref);
+        const float p1 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c + 1] - m_ref);
+        l4[c & 3] += p0 + p1;
         p[c] = pack_f16x2(p0, p1);
       }
-      tc::st32(tP + b * (PF_BN / 2) + lane_off, p);
+      l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+      tc::st32(tS + b * PF_BN + lane_off, p);   // P_j overwrites the S_j columns just read
       tc::wait_st();
       tc::fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[b]);
     }
     // epilogue: O / l -> bf16, undoing the d order 0,2,4,6,1,3,5,7
-    if (ok && mbar_wait_bounded(&pv_done[(ntiles - 1) & 1], ((ntiles - 1) >> 1) & 1)) {
+    if (ok && mbar_wait_bounded(&pv_done[(ntiles - 1) % PF_KVBUF],
+                                ((ntiles - 1) / PF_KVBUF) & 1)) {
       tc::fence_after();
       const float inv = l > 0.f ? 1.f / l : 0.f;
       uint16_t* orow = a.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
