@@ -36,6 +36,22 @@ METRIC = "4-bit paged decode attention KV positions/s and HBM GB/s vs GB300 peak
 UNIT = "positions/s"
 
 
+def measured_traffic(kernel):
+    """DRAM bytes per launch of `kernel` from the committed ncu record, or None
+    when the kernel source changed since the capture."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    rec = json.load(open(p)).get(kernel)
+    if not rec:
+        return None
+    src = os.path.join(ROOT, rec["source"])
+    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != rec["sha256"]:
+        return None
+    return rec["dram_read"] + rec["dram_write"]
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -284,7 +300,8 @@ def run_ours(args, world, rank, local):
         "hbm_gbs_step": positions_per_step * bytes_per_pos / (ms_per_step / 1e3) / 1e9,
         "roofline": {"bound": "hbm", "kernel": "jf_paged_decode_attn (split + merge launches)",
                      "achieved": achieved, "peak": hbm, "peak_source": src, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": None,
+                     "frac": achieved / hbm,
+                     "traffic": measured_traffic("decode_split_kernel<256>"),
                      "alg_bytes_per_launch": alg_bytes, "avg_call_us": decode_ms * 1e3,
                      "frac_of_8tbs": achieved / 8000.0},
         "e2e": {"value": positions_per_step * world / (e2e_ms / 1e3), "unit": UNIT,
@@ -383,7 +400,10 @@ def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
     flops = 4 * Hq * D * (chunk * q_last + chunk * (chunk + 1) // 2)
     out["a4_prefill_chunk_2048_at_30720"] = {
         "ms": t_pf, "TFLOPs": flops / (t_pf / 1e3) / 1e12,
-        "frac_tensor": flops / (t_pf / 1e3) / 1e12 / peak_tf, "flops": flops}
+        "frac_tensor": flops / (t_pf / 1e3) / 1e12 / peak_tf, "flops": flops,
+        "roofline": {"bound": "tensor", "achieved": flops / (t_pf / 1e3) / 1e12, "peak": peak_tf,
+                     "unit": "TFLOP/s", "frac": flops / (t_pf / 1e3) / 1e12 / peak_tf,
+                     "traffic": measured_traffic("prefill_kernel<256>")}}
     out["a1a4_prompt_32k_16_chunks"] = {
         "ms": t_pf_all, "TFLOPs_attention": flops_all / (t_pf_all / 1e3) / 1e12,
         "prompt_positions_per_s": prompt / (t_pf_all / 1e3)}
@@ -519,13 +539,11 @@ def cpu_baseline(args, sample_heads=1):
 
 
 def run_reference(args, world, rank):
+    """The CPU oracle on a bounded sample of the benchmark workload (rank 0)."""
     if rank != 0:
         return None
-    import numpy as np  # noqa: F401
     samples = []
     base = None
-    for _ in range(args.warmup):
-        pass
     t0 = time.perf_counter()
     for _ in range(max(1, min(args.steps, 3))):
         base = cpu_baseline(args)
