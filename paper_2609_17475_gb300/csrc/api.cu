@@ -16,6 +16,7 @@ int launch_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int3
                   const int32_t*, int32_t, const void*, int32_t, float, void*, void*, int32_t,
                   cudaStream_t);
 size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S);
+int decode_box_rows();
 int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
                    const void*, int32_t, int32_t, int32_t, float, int32_t, void*, void*,
                    cudaStream_t);
@@ -134,7 +135,7 @@ int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int3
   if (workspace_bytes < need) return JF_ERR_WORKSPACE_TOO_SMALL;
   const Geom g = make_geom(*pool);
   CUtensorMap tmap;
-  st = make_codes_map(g, pool->base, 32, &tmap);
+  st = make_codes_map(g, pool->base, decode_box_rows(), &tmap);
   if (st) return st;
   return launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q,
                        num_q_heads, softmax_scale, out, workspace, num_splits,
@@ -246,7 +247,7 @@ int jf_paged_decode_attn_noalloc(const jf_kv_pool* pool, const int32_t* page_tab
   if (cudaMemsetAsync(ws, 0, sizeof(int32_t), s) != cudaSuccess) return JF_ERR_CUDA;
   const Geom g = make_geom(*pool);
   CUtensorMap tmap;
-  st = make_codes_map(g, pool->base, 32, &tmap);
+  st = make_codes_map(g, pool->base, decode_box_rows(), &tmap);
   if (st) return st;
   st = launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q, num_q_heads,
                      softmax_scale, out, ws, num_splits, s);

@@ -43,6 +43,11 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
   const int64_t vec = warp_id * VPW + lane / LPV;
   const int64_t total = (int64_t)a.n_rows * a.Hkv * 2;
   const bool active = vec < total;
+  // programmatic dependent launch: the next kernel may be scheduled now (it
+  // waits for this grid before reading the pool); this grid waits for the
+  // previous kernel before it reads the rows, the table or the pool
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
   int64_t row = 0;
   int kind = 0, head = 0;
@@ -140,11 +145,18 @@ int launch_append(const Geom& g, const jf_kv_pool& pool, const int32_t* page_tab
   const int64_t warps = (vectors + vpw - 1) / vpw;
   const int64_t blocks = (warps + 7) / 8;
   if (blocks > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
-  if (g.D == 256)
-    append_kernel<256><<<(unsigned)blocks, 256, 0, stream>>>(a);
-  else
-    append_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(a);
-  return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cfg.attrs = pdl;
+  cfg.numAttrs = 1;
+  const cudaError_t e = (g.D == 256) ? cudaLaunchKernelEx(&cfg, append_kernel<256>, a)
+                                     : cudaLaunchKernelEx(&cfg, append_kernel<128>, a);
+  return e == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }
 
 }  // namespace jfkv

@@ -52,6 +52,7 @@ struct DecodeArgs {
   int64_t sb_base;     // offset of the K scale/bias region in a page record
   int64_t sb_region;   // bytes of one scale/bias region (K or V)
   int32_t P, Hkv, Hq, G;
+  int32_t log2P;        // P is a power of two
   const int32_t* page_table;
   int32_t pt_stride;
   const int32_t* ctx;
@@ -195,11 +196,12 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
   constexpr float NEG_INF = -INFINITY;
   const uint32_t vc = kc + DTOK * CB;
   const uint8_t* vsb = ksb + SB_BUF;
+  constexpr int NJ = DTOK / 16;   // 16-position MMA tiles per chunk
   const int r = cc.r;
 
-  float sc[2][4];
+  float sc[NJ][4];
 #pragma unroll
-  for (int j = 0; j < 2; ++j) {
+  for (int j = 0; j < NJ; ++j) {
     const int ta = 16 * j + r, tb = ta + 8;
     float acc[NG][4];
 #pragma unroll
@@ -248,8 +250,13 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
   }
 
   // ---- online softmax with a lazily moved reference maximum -------------
-  float mx0 = fmaxf(fmaxf(sc[0][0], sc[0][2]), fmaxf(sc[1][0], sc[1][2]));
-  float mx1 = fmaxf(fmaxf(sc[0][1], sc[0][3]), fmaxf(sc[1][1], sc[1][3]));
+  float mx0 = fmaxf(sc[0][0], sc[0][2]);
+  float mx1 = fmaxf(sc[0][1], sc[0][3]);
+#pragma unroll
+  for (int j = 1; j < NJ; ++j) {
+    mx0 = fmaxf(mx0, fmaxf(sc[j][0], sc[j][2]));
+    mx1 = fmaxf(mx1, fmaxf(sc[j][1], sc[j][3]));
+  }
   if (__any_sync(0xffffffffu, (mx0 > st.m0 + DTAU) || (mx1 > st.m1 + DTAU))) {
 #pragma unroll
     for (int o = 4; o < 32; o <<= 1) {
@@ -274,9 +281,9 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
     st.m0 = nm0;
     st.m1 = nm1;
   }
-  float p[2][4];
+  float p[NJ][4];
 #pragma unroll
-  for (int j = 0; j < 2; ++j) {
+  for (int j = 0; j < NJ; ++j) {
     if constexpr (FULL) {
       p[j][0] = fast_exp2(sc[j][0] - st.m0);
       p[j][1] = fast_exp2(sc[j][1] - st.m1);
@@ -294,7 +301,7 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
 
   // ---- PV ---------------------------------------------------------------
 #pragma unroll
-  for (int j = 0; j < 2; ++j) {
+  for (int j = 0; j < NJ; ++j) {
     const int ta = 16 * j + r, tb = ta + 8;
     uint32_t wa[NG], wb[NG];
     load_sb_words<NG>(vsb + ta * SBB, wa);
@@ -366,6 +373,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
   const bool direct = (a.num_splits == 1);
+  // the swizzled TMA boxes need a 1024-byte aligned window
+  const bool aligned = (smem_u32(smem_raw) & 1023) == 0;
+  if (aligned) {   // setup that reads nothing a previous kernel writes
+    if (threadIdx.x == 0) prefetch_tensormap(&tmap);
+    if (lane == 0) {
+      for (int s = 0; s < DSTAGES; ++s) mbar_init(&bars[warp * DSTAGES + s], 1);
+      fence_barrier_init();
+    }
+  }
   // launched with programmatic dependent launch: wait for the previous
   // kernel (e.g. the append that wrote the newest position) before any read
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
@@ -384,14 +400,9 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const int c_end = min(c_begin + cps, nch);
   const int my_n = (c_end - c_begin > warp) ? (c_end - c_begin - warp + DWARPS - 1) / DWARPS : 0;
 
-  if (smem_u32(smem_raw) & 1023) {   // the swizzled TMA boxes need 1024-byte alignment
+  if (!aligned) {
     if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
     return;
-  }
-  if (threadIdx.x == 0) prefetch_tensormap(&tmap);
-  if (lane == 0) {
-    for (int s = 0; s < DSTAGES; ++s) mbar_init(&bars[warp * DSTAGES + s], 1);
-    fence_barrier_init();
   }
   __syncwarp();
 
@@ -478,7 +489,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const int it = blk * 32 + lane;
     int page = -1;
     if (it < my_n) {
-      const int pidx = ((c_begin + warp + it * DWARPS) * DTOK) / a.P;
+      const int pidx = ((c_begin + warp + it * DWARPS) * DTOK) >> a.log2P;
       if (pidx < a.pt_stride) page = __ldg(a.page_table + (int64_t)b * a.pt_stride + pidx);
     }
     return page;
@@ -497,7 +508,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const int page = __shfl_sync(0xffffffffu, pg_cur, it & 31);
     const bool ok = page >= 0 && page < a.num_pages;
     if (lane == 0) {
-      const int inp = ((c_begin + warp + it * DWARPS) * DTOK) % a.P;
+      const int inp = ((c_begin + warp + it * DWARPS) * DTOK) & (a.P - 1);
       uint64_t* bar = &bars[warp * DSTAGES + s];
       if (!ok) {
         flag_error(a.status, JF_DEV_ERR_PAGE_ID);
@@ -650,53 +661,95 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
 
 // One CTA per (32-wide slice of head_dim, query head, request); its 8 warps
 // take interleaved splits and reduce through shared memory, so the merge is
-// spread over the whole GPU and each thread issues only a few loads.
+// spread over the whole GPU.  The kernel is a chain of dependent loads, so it
+// issues them all at once: the context length, every (m, l) row and this
+// thread's partial outputs for up to MERGE_BATCH splits are loaded before any
+// is used; rows past the split plan are loaded (the workspace holds
+// num_splits rows) and then ignored.
 constexpr int MERGE_THREADS = 256;
 constexpr int MERGE_DSLICE = 32;
+constexpr int MERGE_NSG = MERGE_THREADS / MERGE_DSLICE;   // split groups
+constexpr int MERGE_BATCH = 16;                           // splits per thread per batch
+constexpr int MERGE_MLB = MERGE_BATCH * MERGE_NSG / 32;   // (m, l) rows per lane per batch
 
 template <int D>
 __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const DecodeArgs a) {
-  constexpr int NSG = MERGE_THREADS / MERGE_DSLICE;   // split groups
-  __shared__ float red[NSG][MERGE_DSLICE];
-  __shared__ float sM, sL;
+  __shared__ float red[MERGE_NSG][MERGE_DSLICE];
+  // the next kernel in the stream may be scheduled now; it waits for this
+  // grid to complete before it reads anything
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   // the split kernel's partials must be complete and visible
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   const int d0 = blockIdx.x * MERGE_DSLICE, hq = blockIdx.y, b = blockIdx.z;
   const int t = threadIdx.x, dd = t % MERGE_DSLICE, sg = t / MERGE_DSLICE;
-  const int ctx = checked_ctx(a, b);
+  const int lane = t & 31;
+  const int S = a.num_splits;
+  const int64_t row0 = ((int64_t)b * a.Hq + hq) * S;
+  const float2* ml = reinterpret_cast<const float2*>(a.part_ml) + row0;
+  const float* po = a.part_o + row0 * D + d0 + dd;
+
+  const int ctx_raw = a.ctx[b];
+  float2 mlv[MERGE_MLB];
+  float ov[MERGE_BATCH], mv[MERGE_BATCH];
+#pragma unroll
+  for (int k = 0; k < MERGE_MLB; ++k) {
+    const int s = lane + 32 * k;
+    mlv[k] = (s < S) ? ml[s] : make_float2(-INFINITY, 0.f);
+  }
+#pragma unroll
+  for (int u = 0; u < MERGE_BATCH; ++u) {
+    const int s = sg + MERGE_NSG * u;
+    ov[u] = (s < S) ? po[(int64_t)s * D] : 0.f;
+    mv[u] = (s < S) ? ml[s].x : -INFINITY;
+  }
+  int ctx = ctx_raw;
+  const int64_t cap = (int64_t)a.pt_stride * a.P;
+  if (ctx < 0) ctx = 0;
+  if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
-  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  split_plan(ctx, S, nch, cps, nsplit);
   uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D + d0;
   if (nsplit == 0) {
     if (t < MERGE_DSLICE) orow[t] = 0;
     return;
   }
-  const int64_t row0 = ((int64_t)b * a.Hq + hq) * a.num_splits;
-  const float2* ml = reinterpret_cast<const float2*>(a.part_ml) + row0;
-  if (t < 32) {   // warp 0: global max and normalizer
-    float M = -INFINITY;
-    for (int s = t; s < nsplit; s += 32) M = fmaxf(M, ml[s].x);
+
+  // global maximum (every warp finds it itself)
+  float M = -INFINITY;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float L = 0.f;
-    if (M != -INFINITY)
-      for (int s = t; s < nsplit; s += 32) {
-        const float2 v = ml[s];
-        if (v.x != -INFINITY) L = fmaf(fast_exp2(v.x - M), v.y, L);
-      }
+  for (int k = 0; k < MERGE_MLB; ++k)
+    if (lane + 32 * k < nsplit) M = fmaxf(M, mlv[k].x);
+  for (int s = lane + 32 * MERGE_MLB; s < nsplit; s += 32) M = fmaxf(M, ml[s].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+
+  float L = 0.f, acc = 0.f;
+  if (M != -INFINITY) {
+#pragma unroll
+    for (int k = 0; k < MERGE_MLB; ++k)
+      if (lane + 32 * k < nsplit && mlv[k].x != -INFINITY)
+        L = fmaf(fast_exp2(mlv[k].x - M), mlv[k].y, L);
+    for (int s = lane + 32 * MERGE_MLB; s < nsplit; s += 32) {
+      const float2 v = ml[s];
+      if (v.x != -INFINITY) L = fmaf(fast_exp2(v.x - M), v.y, L);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    if (t == 0) { sM = M; sL = L; }
-  }
-  __syncthreads();
-  const float M = sM;
-  float acc = 0.f;
-  if (M != -INFINITY) {
-#pragma unroll 4
-    for (int s = sg; s < nsplit; s += NSG) {
-      const float ms = ml[s].x;
-      if (ms == -INFINITY) continue;
-      acc = fmaf(fast_exp2(ms - M), a.part_o[(row0 + s) * D + d0 + dd], acc);
+#pragma unroll
+    for (int u = 0; u < MERGE_BATCH; ++u)
+      if (sg + MERGE_NSG * u < nsplit && mv[u] != -INFINITY)
+        acc = fmaf(fast_exp2(mv[u] - M), ov[u], acc);
+    // more splits than one batch covers
+    for (int s0 = sg + MERGE_NSG * MERGE_BATCH; s0 < nsplit; s0 += MERGE_NSG * MERGE_BATCH) {
+#pragma unroll
+      for (int u = 0; u < MERGE_BATCH; ++u) {
+        const int s = s0 + MERGE_NSG * u;
+        ov[u] = (s < nsplit) ? po[(int64_t)s * D] : 0.f;
+        mv[u] = (s < nsplit) ? ml[s].x : -INFINITY;
+      }
+#pragma unroll
+      for (int u = 0; u < MERGE_BATCH; ++u)
+        if (mv[u] != -INFINITY) acc = fmaf(fast_exp2(mv[u] - M), ov[u], acc);
     }
   }
   red[sg][dd] = acc;
@@ -704,8 +757,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   if (t < MERGE_DSLICE) {
     float o = 0.f;
 #pragma unroll
-    for (int k = 0; k < NSG; ++k) o += red[k][t];
-    const float L = sL;
+    for (int k = 0; k < MERGE_NSG; ++k) o += red[k][t];
     orow[t] = __bfloat16_as_ushort(__float2bfloat16_rn(L > 0.f ? o / L : 0.f));
   }
 }
@@ -713,6 +765,9 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+// rows (positions) of one TMA box of the decode code tensor map
+int decode_box_rows() { return DTOK; }
+
 size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S) {
   const int64_t rows = B * Hq * S;
   const int64_t ml = (rows * 8 + 255) / 256 * 256;
@@ -768,6 +823,7 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.sb_base = 2 * g.codes_region;
   a.sb_region = g.sb_region;
   a.P = g.P;
+  a.log2P = __builtin_ctz((unsigned)g.P);
   a.Hkv = g.Hkv;
   a.Hq = Hq;
   a.G = Hq / g.Hkv;

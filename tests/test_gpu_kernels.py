@@ -40,6 +40,7 @@ def gpu_decode(case, pool, splits, ctx=None, q=None, scale=None, page_table=None
     B = len(ctx)
     out = torch.full((B, case.Hq, case.D), float("nan"), dtype=torch.bfloat16, device=DEV)
     ws = jf.decode_workspace(B, case.Hq, case.Hkv, case.D, splits, device=DEV)
+    ws[256:] = 0xFF    # NaN partials: rows past the split plan must never be used
     scale = 1 / math.sqrt(case.D) if scale is None else scale
     jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor(ctx, dtype=torch.int32, device=DEV),
                             q.to(DEV), scale, out, ws, splits)
@@ -151,6 +152,7 @@ def test_checkpoint_and_restore_bit_exact(Hkv, D, P, ctx):
     (4, 4, 256, 64, [1500], 2, False),             # G = 1
     (16, 2, 256, 256, [2500], 5, False),           # G = 8
     (12, 2, 128, 128, [999], 64, False),           # more splits than needed
+    (8, 2, 128, 256, [70000, 3000], 150, False),   # > 128 live splits: merge loops
 ])
 def test_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
     case = make_case(200 + Hq + sum(ctx), Hq, Hkv, D, P, ctx, outliers=outliers)
