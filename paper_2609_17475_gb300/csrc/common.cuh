@@ -145,6 +145,17 @@ __device__ __forceinline__ uint32_t movm_t(uint32_t x) {
 }
 
 // D += A(16x16, f16, row) * B(16x8, f16, col), fp32 accumulate.
+// d = A B (the accumulator input is the zero register, not four zeroed registers)
+__device__ __forceinline__ void mma_f16_zc(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                           uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "{\n.reg .f32 z;\nmov.f32 z, 0f00000000;\n"
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {z,z,z,z};\n}\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 __device__ __forceinline__ void mma_f16(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
                                         uint32_t a3, uint32_t b0, uint32_t b1) {
   asm volatile(

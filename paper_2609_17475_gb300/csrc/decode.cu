@@ -110,6 +110,17 @@ __device__ __forceinline__ void mma_bf16(float* d, uint32_t a0, uint32_t a1, uin
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// d = A B in bf16 (zero accumulator input)
+__device__ __forceinline__ void mma_bf16_zc(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
+                                            uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "{\n.reg .f32 z;\nmov.f32 z, 0f00000000;\n"
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {z,z,z,z};\n}\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   uint32_t r;
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
@@ -168,7 +179,11 @@ struct ChunkCtx {
   const uint4* qf;   // this lane's query fragments: qf[2 g + half] = k-steps 2 half, 2 half + 1
   uint32_t bq;   // B fragment of the QK bias MMA: (Q_g high | low parts) for head r
   float cA, cB;
-  int r, c, ld_t, ld_ch;
+  int r, c;
+  // this lane's ldmatrix row address within a stage buffer for group g's two
+  // 16-byte chunks (16-position tile 0; tile j adds 16 j rows, which keeps
+  // the swizzle phase)
+  uint32_t koff[NG];
 };
 
 template <int NG>
@@ -208,10 +223,9 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
     for (int g = 0; g < NG; ++g) {
       const uint4 qa = cc.qf[(2 * g) * 32], qb = cc.qf[(2 * g + 1) * 32];
       uint32_t w0, w1, w2, w3;
-      ldsm_x4(w0, w1, w2, w3, kc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
-      acc[g][0] = acc[g][1] = acc[g][2] = acc[g][3] = 0.f;
+      ldsm_x4(w0, w1, w2, w3, kc + cc.koff[g] + 16 * j * CB);
       const uint32_t h0 = shr8(w0), h1 = shr8(w1), h2 = shr8(w2), h3 = shr8(w3);
-      mma_f16(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), qa.x, qa.y);
+      mma_f16_zc(acc[g], nib0(w0), nib0(w1), nib1(w0), nib1(w1), qa.x, qa.y);
       mma_f16(acc[g], nib0(h0), nib0(h1), nib1(h0), nib1(h1), qa.z, qa.w);
       mma_f16(acc[g], nib0(w2), nib0(w3), nib1(w2), nib1(w3), qb.x, qb.y);
       mma_f16(acc[g], nib0(h2), nib0(h3), nib1(h2), nib1(h3), qb.z, qb.w);
@@ -220,7 +234,7 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
     load_sb_words<NG>(ksb + ta * SBB, wa);
     load_sb_words<NG>(ksb + tb * SBB, wb);
     // bias term sum_g bias_{t,g} Q_g: A rows = positions, k-slots = groups x (Q high, Q low)
-    float t2[4] = {0.f, 0.f, 0.f, 0.f};
+    float t2[4];
     {
       uint32_t aa, ab;
       if constexpr (NG == 4) {
@@ -230,7 +244,7 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
         aa = (cc.c < 2) ? hi_halves(wa[0], wa[1]) : 0u;
         ab = (cc.c < 2) ? hi_halves(wb[0], wb[1]) : 0u;
       }
-      mma_bf16(t2, aa, ab, 0u, 0u, cc.bq, 0u);
+      mma_bf16_zc(t2, aa, ab, 0u, 0u, cc.bq, 0u);
     }
     float t1[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
@@ -345,7 +359,7 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
       const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
       const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
       uint32_t v0, v1, v2, v3;
-      ldsm_x4_t(v0, v1, v2, v3, vc + swz<CB>(16 * j + cc.ld_t, 2 * g + cc.ld_ch));
+      ldsm_x4_t(v0, v1, v2, v3, vc + cc.koff[g] + 16 * j * CB);
       const uint32_t h0 = shr8(v0), h1 = shr8(v1), h2 = shr8(v2), h3 = shr8(v3);
       mma_f16(st.O[g][0], nib0(v0), nib0(v2), nib0(v1), nib0(v3), b0, b1);
       mma_f16(st.O[g][1], nib1(v0), nib1(v2), nib1(v1), nib1(v3), b0, b1);
@@ -546,9 +560,13 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     }
   }
   __syncthreads();
-  const ChunkCtx<NG> cc{qsm + lane, bq, cA, cB, r, c, ld_t, ld_ch};
+  ChunkCtx<NG> cc{qsm + lane, bq, cA, cB, r, c, {}};
+#pragma unroll
+  for (int g = 0; g < NG; ++g) cc.koff[g] = swz<L::CB>(ld_t, 2 * g + ld_ch);
 
   int done = 0;
+  // unrolled by the ring depth, so every stage address is a constant offset
+#pragma unroll DSTAGES
   for (int it = 0; it < my_n; ++it) {
     const int s = it % DSTAGES;
     const uint32_t par = (it / DSTAGES) & 1;
