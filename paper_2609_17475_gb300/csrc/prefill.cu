@@ -16,8 +16,9 @@
 //               TMEM columns: O [0, D), two S/P buffers of 64, Q [D + 128, +D/2);
 //               P_j (fp16) overwrites the first half of S_j once it is read.
 //   warps 1-8   dequantize 64-position K/V tiles from the pool (page-table
-//               lookup, 4-bit codes -> fp16 via an e4m3 convert, then
-//               x = code * scale + bias with one fused multiply-add) into
+//               lookup, 4-bit codes -> fp16 integers through the mantissa of
+//               fp16 1024, then x = code * scale + bias with one fused
+//               multiply-add) into
 //               three 128B-swizzled tile buffers; each thread owns one
 //               position's 32 contiguous code bytes per 64-wide block, loads
 //               run two tiles ahead, and the 8 lanes of a quarter-warp store
@@ -29,7 +30,7 @@
 //               only when it grows by more than 2^8, and then O is rescaled
 //               in TMEM; finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
-// 0,2,4,6,1,3,5,7 (what the two-nibble convert produces); Q uses the same
+// 0,4,1,5,2,6,3,7 (the pairs one 32-bit word of codes yields); Q uses the same
 // order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
 // stored pre-multiplied by softmax_scale * log2(e), so S arrives in the log2
 // domain.
@@ -73,16 +74,9 @@ struct PfSmem {
   static constexpr int TOTAL = 1024 + OFF_BAR + 256;
 };
 
-__device__ __forceinline__ uint32_t cvt_e4m3x2_f16x2(uint32_t two_bytes) {
+__device__ __forceinline__ uint32_t hadd2(uint32_t a, uint32_t b) {
   uint32_t r;
-  asm("{\n\t.reg .b16 t;\n\tcvt.u16.u32 t, %1;\n\tcvt.rn.f16x2.e4m3x2 %0, t;\n\t}\n"
-      : "=r"(r) : "r"(two_bytes));
-  return r;
-}
-
-__device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
-  uint32_t r;
-  asm("mul.rn.f16x2 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
+  asm("add.rn.f16x2 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
   return r;
 }
 
@@ -92,41 +86,29 @@ __device__ __forceinline__ uint32_t hfma2(uint32_t a, uint32_t b, uint32_t c) {
   return r;
 }
 
-// 8 packed 4-bit codes (d0..d7) -> 8 fp16 values code*scale + bias in the
-// order d0,d2,d4,d6,d1,d3,d5,d7.  A byte 0..15 read as e4m3 is exactly
-// code * 2^-9 (subnormal for < 8, exponent 1 for >= 8), so the convert plus an
-// exact *512 yields the integer code; the fma rounds once.
+// 8 packed 4-bit codes (d0..d7) -> 8 fp16 values code * scale + bias, stored
+// in the order d0,d4,d1,d5,d2,d6,d3,d7.  A nibble OR-ed into the mantissa of
+// fp16 1024 (exponent 2^10, unit mantissa step) gives 1024 + n, or 1024 + 16 n
+// for a high nibble; subtracting 1024 (or scaling by 1/16 and subtracting 64)
+// recovers the integer code exactly, and one fused multiply-add rounds once.
 __device__ __forceinline__ uint4 dequant8(uint32_t w, uint32_t s2, uint32_t b2) {
-  const uint32_t lo = w & 0x0F0F0F0Fu;
-  const uint32_t hi = (w >> 4) & 0x0F0F0F0Fu;
-  const uint32_t k512 = 0x60006000u;   // (512, 512) in f16
+  constexpr uint32_t K1024 = 0x64006400u;    // (1024, 1024)
+  constexpr uint32_t KM1024 = 0xE400E400u;   // (-1024, -1024)
+  constexpr uint32_t K1_16 = 0x2C002C00u;    // (1/16, 1/16)
+  constexpr uint32_t KM64 = 0xD400D400u;     // (-64, -64)
+  const uint32_t w8 = __umulhi(w, 0x01000000u);   // w >> 8 on the FMA pipe
   uint4 o;
-  o.x = hfma2(hmul2(cvt_e4m3x2_f16x2(lo & 0xFFFFu), k512), s2, b2);
-  o.y = hfma2(hmul2(cvt_e4m3x2_f16x2(lo >> 16), k512), s2, b2);
-  o.z = hfma2(hmul2(cvt_e4m3x2_f16x2(hi & 0xFFFFu), k512), s2, b2);
-  o.w = hfma2(hmul2(cvt_e4m3x2_f16x2(hi >> 16), k512), s2, b2);
+  o.x = hfma2(hadd2((w & 0x000F000Fu) | K1024, KM1024), s2, b2);           // (d0, d4)
+  o.y = hfma2(hfma2((w & 0x00F000F0u) | K1024, K1_16, KM64), s2, b2);      // (d1, d5)
+  o.z = hfma2(hadd2((w8 & 0x000F000Fu) | K1024, KM1024), s2, b2);          // (d2, d6)
+  o.w = hfma2(hfma2((w8 & 0x00F000F0u) | K1024, K1_16, KM64), s2, b2);     // (d3, d7)
   return o;
 }
 
-// Same with the *512 folded into the scale (scale * 512 must fit fp16).
-__device__ __forceinline__ uint4 dequant8_fast(uint32_t w, uint32_t s512, uint32_t b2) {
-  const uint32_t lo = w & 0x0F0F0F0Fu;
-  const uint32_t hi = (w >> 4) & 0x0F0F0F0Fu;
-  uint4 o;
-  o.x = hfma2(cvt_e4m3x2_f16x2(lo & 0xFFFFu), s512, b2);
-  o.y = hfma2(cvt_e4m3x2_f16x2(lo >> 16), s512, b2);
-  o.z = hfma2(cvt_e4m3x2_f16x2(hi & 0xFFFFu), s512, b2);
-  o.w = hfma2(cvt_e4m3x2_f16x2(hi >> 16), s512, b2);
-  return o;
-}
-
-// bf16 (scale | bias << 16) word -> f16x2 broadcasts of scale (or scale*512
-// when that fits fp16: fast = true) and bias
-__device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2, bool& fast) {
+// bf16 (scale | bias << 16) word -> f16x2 broadcasts of scale and bias
+__device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2) {
   const float s = bf16lo_to_f32(w), b = bf16hi_to_f32(w);
-  fast = fabsf(s) <= 120.f;
-  const float sc = fast ? s * 512.f : s;
-  s2 = pack_f16x2(sc, sc);
+  s2 = pack_f16x2(s, s);
   b2 = pack_f16x2(b, b);
 }
 
@@ -184,7 +166,7 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   const uint32_t tQ = tbase + D + 2 * PF_BN;   // D/2 columns of f16 pairs
 
   // ---- softmax warps: their Q row -> TMEM (fp16, pre-multiplied by
-  // softmax_scale * log2(e), d order 0,2,4,6,1,3,5,7 in every 8) ------------
+  // softmax_scale * log2(e), d order 0,4,1,5,2,6,3,7 in every 8) ------------
   const int quarter = warp & 3;                // TMEM lanes this warp may access
   const int r = quarter * 32 + lane;
   const bool row_ok = r < rows;
@@ -217,10 +199,10 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
         const float e2 = bf16lo_to_f32(w.y) * qs, e3 = bf16hi_to_f32(w.y) * qs;
         const float e4 = bf16lo_to_f32(w.z) * qs, e5 = bf16hi_to_f32(w.z) * qs;
         const float e6 = bf16lo_to_f32(w.w) * qs, e7 = bf16hi_to_f32(w.w) * qs;
-        v[4 * k + 0] = pack_f16x2(e0, e2);
-        v[4 * k + 1] = pack_f16x2(e4, e6);
-        v[4 * k + 2] = pack_f16x2(e1, e3);
-        v[4 * k + 3] = pack_f16x2(e5, e7);
+        v[4 * k + 0] = pack_f16x2(e0, e4);
+        v[4 * k + 1] = pack_f16x2(e1, e5);
+        v[4 * k + 2] = pack_f16x2(e2, e6);
+        v[4 * k + 3] = pack_f16x2(e3, e7);
       }
       tc::st32(tQ + c0 + lane_off, v);
     }
@@ -298,19 +280,13 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     };
     auto store_half = [&](uint8_t* tile, const uint4 (&codes)[UPI], uint32_t sbw, bool valid) {
       uint32_t s2, b2;
-      bool fast;
-      sb_to_h2(sbw, s2, b2, fast);
+      sb_to_h2(sbw, s2, b2);
       uint4 o[UPI][4];
 #pragma unroll
       for (int u = 0; u < UPI; ++u) {
         const uint32_t cw[4] = {codes[u].x, codes[u].y, codes[u].z, codes[u].w};
-        if (fast) {
 #pragma unroll
-          for (int w = 0; w < 4; ++w) o[u][w] = dequant8_fast(cw[w], s2, b2);
-        } else {
-#pragma unroll
-          for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
-        }
+        for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
       }
 #pragma unroll
       for (int u = 0; u < UPI; ++u)
@@ -428,7 +404,7 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[b]);
     }
-    // epilogue: O / l -> bf16, undoing the d order 0,2,4,6,1,3,5,7
+    // epilogue: O / l -> bf16, undoing the d order 0,4,1,5,2,6,3,7
     if (ok && mbar_wait_bounded(&pv_done[(ntiles - 1) % PF_KVBUF],
                                 ((ntiles - 1) / PF_KVBUF) & 1)) {
       tc::fence_after();
@@ -445,12 +421,12 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
             const float* v = reinterpret_cast<const float*>(o + 8 * k);
             uint4 w;
             w.x = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[0] * inv)) |
-                  ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[4] * inv)) << 16);
-            w.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[1] * inv)) |
-                  ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[5] * inv)) << 16);
-            w.z = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[2] * inv)) |
+                  ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[2] * inv)) << 16);
+            w.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[4] * inv)) |
                   ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[6] * inv)) << 16);
-            w.w = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[3] * inv)) |
+            w.z = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[1] * inv)) |
+                  ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[3] * inv)) << 16);
+            w.w = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[5] * inv)) |
                   ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v[7] * inv)) << 16);
             *reinterpret_cast<uint4*>(orow + c0 + 8 * k) = w;
           }
