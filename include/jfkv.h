@@ -148,6 +148,30 @@ int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int3
                          size_t workspace_bytes, int32_t num_splits, void* stream);
 
 /*
+ * Append-then-attend decode step in one launch pair (Sec. 3.3: the step's
+ * pending cache write lands before its attention reads the pool; Sec. 3.1
+ * decode).  For every request b with context_lens[b] >= 1 the bf16 vectors
+ * k_new[b, h, :] and v_new[b, h, :] are quantized exactly as
+ * jf_kv_quantize_append does and written to position context_lens[b] - 1,
+ * then out is computed exactly as jf_paged_decode_attn computes it over
+ * positions [0, context_lens[b]).  The result (pool bytes and out) equals
+ * jf_kv_quantize_append with row_req = b, row_pos = context_lens[b] - 1
+ * followed by jf_paged_decode_attn; the fused form saves one launch and one
+ * grid-wide dependency per step.  Each new row is written by the split that
+ * owns its position, before that split reads it.
+ *   k_new, v_new  bf16 [batch, Hkv, D], 16-byte aligned
+ * Other arguments, limits and errors as for jf_paged_decode_attn; a bad page
+ * id for the new row sets JF_DEV_ERR_PAGE_ID in the status word and skips
+ * that write.
+ */
+int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_table,
+                                int32_t pt_stride, const int32_t* context_lens, int32_t batch,
+                                const void* k_new, const void* v_new, const void* q,
+                                int32_t num_q_heads, float softmax_scale, void* out,
+                                void* workspace, size_t workspace_bytes, int32_t num_splits,
+                                void* stream);
+
+/*
  * Prefill-chunk attention for one request (Sec. 3.1 "decode and prefill need
  * different kernels"; Eq. 5).  chunk_len queries q[i] at absolute positions
  * q_start + i attend positions [0, q_start + i] (causal != 0) or

@@ -31,7 +31,7 @@ EXPORTS = [
     "jf_kv_page_bytes", "jf_attn_workspace_bytes", "jf_prefill_workspace_bytes",
     "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
-    "jf_paged_decode_attn_noalloc",
+    "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -75,6 +75,8 @@ def lib() -> ctypes.CDLL:
             "jf_kv_restore": (ctypes.c_int, [PP, P, I32, P, SZ, P, P]),
             "jf_paged_decode_attn_noalloc": (ctypes.c_int, [PP, P, I32, P, I32, P, I32, F32, P,
                                                             I32, P, P]),
+            "jf_paged_decode_append_attn": (ctypes.c_int, [PP, P, I32, P, I32, P, P, P, I32, F32,
+                                                           P, P, SZ, I32, P]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -211,6 +213,34 @@ def jf_paged_decode_attn(pool: KVPool, page_table: torch.Tensor, context_lens: t
                                      float(softmax_scale), _ptr(out), _ptr(workspace),
                                      workspace.numel(), int(num_splits), _stream(stream))
     _check("jf_paged_decode_attn", st)
+
+
+def jf_paged_decode_append_attn(pool: KVPool, page_table: torch.Tensor,
+                                context_lens: torch.Tensor, k_new: torch.Tensor,
+                                v_new: torch.Tensor, q: torch.Tensor, softmax_scale: float,
+                                out: torch.Tensor, workspace: torch.Tensor, num_splits: int,
+                                stream=None) -> None:
+    """Append the step's K/V row of every request at position context_lens[b] - 1,
+    then decode: the same pool bytes and output as jf_kv_quantize_append followed
+    by jf_paged_decode_attn, in one launch pair."""
+    _need(page_table, torch.int32, "page_table")
+    _need(context_lens, torch.int32, "context_lens")
+    _need(k_new, torch.bfloat16, "k_new")
+    _need(v_new, torch.bfloat16, "v_new")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    _need(workspace, torch.uint8, "workspace")
+    B, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim or page_table.shape[0] != B or context_lens.numel() != B:
+        raise ValueError("shape mismatch")
+    if tuple(k_new.shape) != (B, pool.num_kv_heads, D) or v_new.shape != k_new.shape:
+        raise ValueError("k_new / v_new must be [batch, Hkv, D]")
+    st = lib().jf_paged_decode_append_attn(ctypes.byref(pool.c_struct()), _ptr(page_table),
+                                            page_table.shape[1], _ptr(context_lens), B,
+                                            _ptr(k_new), _ptr(v_new), _ptr(q), Hq,
+                                            float(softmax_scale), _ptr(out), _ptr(workspace),
+                                            workspace.numel(), int(num_splits), _stream(stream))
+    _check("jf_paged_decode_append_attn", st)
 
 
 def jf_paged_decode_attn_noalloc(pool: KVPool, page_table: torch.Tensor,

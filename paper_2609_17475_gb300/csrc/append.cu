@@ -5,10 +5,8 @@
 // One vector (row, KV head, K|V) of D bf16 elements is handled by D/8 lanes,
 // each loading 16 bytes (8 elements), so a warp reads 512 contiguous bytes at
 // D = 256 and writes one 128-byte code row plus four 4-byte scale/bias words.
-// A 64-element group spans 8 consecutive lanes; its min/max is reduced with
-// three xor-shuffles.  All arithmetic is IEEE fp32 with explicit rounding
-// intrinsics (no contraction) so the codes match the CPU oracle bit for bit.
-#include "common.cuh"
+// The quantizer itself (quant.cuh) is shared with the fused decode.
+#include "quant.cuh"
 
 namespace jfkv {
 
@@ -35,8 +33,6 @@ template <int D>
 __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
   constexpr int LPV = D / 8;        // lanes per vector
   constexpr int VPW = 32 / LPV;     // vectors per warp
-  constexpr int CB = D / 2;
-  constexpr int SBB = D / 16;       // 4 bytes per 64-group
   const int lane = threadIdx.x & 31;
   const int64_t warp_id = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int li = lane % LPV;
@@ -51,49 +47,17 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
 
   int64_t row = 0;
   int kind = 0, head = 0;
-  float x[8];
+  float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   if (active) {
     row = vec / (2 * a.Hkv);
     const int rem = (int)(vec % (2 * a.Hkv));
     kind = rem / a.Hkv;
     head = rem % a.Hkv;
-    const uint16_t* src = (kind ? a.v : a.k) + (row * a.Hkv + head) * D + li * 8;
-    const uint4 w = *reinterpret_cast<const uint4*>(src);
-    x[0] = bf16lo_to_f32(w.x); x[1] = bf16hi_to_f32(w.x);
-    x[2] = bf16lo_to_f32(w.y); x[3] = bf16hi_to_f32(w.y);
-    x[4] = bf16lo_to_f32(w.z); x[5] = bf16hi_to_f32(w.z);
-    x[6] = bf16lo_to_f32(w.w); x[7] = bf16hi_to_f32(w.w);
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) x[i] = 0.f;
+    load8_bf16((kind ? a.v : a.k) + (row * a.Hkv + head) * D + li * 8, x);
   }
-
-  // group min / max over 8 lanes x 8 elements (exact)
-  float mn = x[0], mx = x[0];
-#pragma unroll
-  for (int i = 1; i < 8; ++i) { mn = fminf(mn, x[i]); mx = fmaxf(mx, x[i]); }
-#pragma unroll
-  for (int o = 1; o < 8; o <<= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  }
+  __nv_bfloat16 scale_h, bias_h;
+  const uint32_t word = quantize8(x, scale_h, bias_h);
   if (!active) return;
-
-  const float bias = __fadd_rn(mn, 0.0f);                 // -0 -> +0
-  const float range = __fsub_rn(mx, mn);
-  const __nv_bfloat16 scale_h = __float2bfloat16_rn(__fdiv_rn(range, 15.0f));
-  const float scale = __bfloat162float(scale_h);
-  uint32_t word = 0;
-  if (scale != 0.0f) {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const float r = __fdiv_rn(__fsub_rn(x[i], bias), scale);
-      // code = number of thresholds k + 1/2 (k = 0..14) that r strictly exceeds
-      int c = (int)ceilf(__fsub_rn(r, 0.5f));
-      c = min(max(c, 0), 15);
-      word |= (uint32_t)c << (4 * i);
-    }
-  }
 
   // destination slot
   const int32_t req = a.row_req[row];
@@ -107,16 +71,8 @@ __global__ void __launch_bounds__(256) append_kernel(const AppendArgs a) {
     if (li == 0) flag_error(a.err, JF_DEV_ERR_PAGE_ID);
     return;
   }
-  const int slot = pos % a.P;
-  uint8_t* base = a.pool + (int64_t)page * a.page_bytes;
-  const int64_t vrow = (int64_t)head * a.P + slot;
-  *reinterpret_cast<uint32_t*>(base + kind * a.codes_region + vrow * CB + li * 4) = word;
-  if ((li & 7) == 0) {
-    const uint32_t sb = (uint32_t)__bfloat16_as_ushort(scale_h) |
-                        ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(bias)) << 16);
-    *reinterpret_cast<uint32_t*>(base + 2 * a.codes_region + kind * a.sb_region + vrow * SBB +
-                                 (li >> 3) * 4) = sb;
-  }
+  store_quantized<D>(a.pool + (int64_t)page * a.page_bytes, a.codes_region, a.sb_region, a.P,
+                     head, pos % a.P, kind, li, word, scale_h, bias_h);
 }
 
 int launch_append(const Geom& g, const jf_kv_pool& pool, const int32_t* page_table,

@@ -35,7 +35,7 @@
 #include <cmath>
 #include <cfloat>
 
-#include "common.cuh"
+#include "quant.cuh"
 
 namespace jfkv {
 
@@ -49,6 +49,7 @@ struct DecodeArgs {
   const uint8_t* pool;
   int64_t num_pages;
   int64_t page_bytes;
+  int64_t codes_region;   // bytes of one code region (K or V) in a page record
   int64_t sb_base;     // offset of the K scale/bias region in a page record
   int64_t sb_region;   // bytes of one scale/bias region (K or V)
   int32_t P, Hkv, Hq, G;
@@ -57,6 +58,8 @@ struct DecodeArgs {
   int32_t pt_stride;
   const int32_t* ctx;
   const uint16_t* q;
+  const uint16_t* knew;   // fused append: new K/V rows [B, Hkv, D], or null
+  const uint16_t* vnew;
   uint16_t* out;
   float* part_ml;      // [B, Hq, S, 2]
   float* part_o;       // [B, Hq, S, D]
@@ -369,6 +372,34 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
   }
 }
 
+// Fused append: the split that owns position pos of request b quantizes the
+// step's new K and V vectors of its KV head (one vector per D/8 lanes, the
+// quantizer the append kernel uses) and stores them before any of its reads.
+template <int D>
+__device__ __forceinline__ void append_new_row(const DecodeArgs& a, int b, int kvh, int pos,
+                                               int warp, int lane) {
+  constexpr int LPV = D / 8;        // lanes per vector
+  constexpr int VPW = 32 / LPV;     // vectors per warp
+  if (warp * VPW >= 2) return;      // warp-uniform: the K and V vectors only
+  const int vec = warp * VPW + lane / LPV;   // 0: K, 1: V
+  const int li = lane % LPV;
+  const bool active = vec < 2;
+  float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (active) load8_bf16((vec ? a.vnew : a.knew) + ((int64_t)b * a.Hkv + kvh) * D + li * 8, x);
+  __nv_bfloat16 sh, bh;
+  const uint32_t word = quantize8(x, sh, bh);
+  if (!active) return;
+  const int pidx = pos >> a.log2P;
+  const int page = (pidx < a.pt_stride) ? a.page_table[(int64_t)b * a.pt_stride + pidx] : -1;
+  if (page < 0 || page >= a.num_pages) {
+    if (li == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+    return;
+  }
+  store_quantized<D>(const_cast<uint8_t*>(a.pool) + (int64_t)page * a.page_bytes,
+                     a.codes_region, a.sb_region, a.P, kvh, pos & (a.P - 1), vec, li, word, sh,
+                     bh);
+}
+
 template <int D>
 __global__ void __launch_bounds__(DWARPS * 32, 2)
 decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
@@ -417,6 +448,13 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   if (!aligned) {
     if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
     return;
+  }
+  if (a.knew != nullptr && split == nsplit - 1) {   // CTA-uniform
+    // the new row goes to the pool before this split's TMA reads it
+    append_new_row<D>(a, b, kvh, ctx - 1, warp, lane);
+    fence_proxy_async_global();
+    __syncthreads();
+    fence_proxy_async_global();
   }
   __syncwarp();
 
@@ -833,11 +871,13 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
 int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
                   const int32_t* page_table, int32_t pt_stride, const int32_t* context_lens,
                   int32_t batch, const void* q, int32_t Hq, float softmax_scale, void* out,
-                  void* workspace, int32_t num_splits, cudaStream_t stream) {
+                  void* workspace, int32_t num_splits, cudaStream_t stream, const void* k_new,
+                  const void* v_new) {
   DecodeArgs a;
   a.pool = static_cast<const uint8_t*>(pool.base);
   a.num_pages = g.num_pages;
   a.page_bytes = g.page_bytes;
+  a.codes_region = g.codes_region;
   a.sb_base = 2 * g.codes_region;
   a.sb_region = g.sb_region;
   a.P = g.P;
@@ -849,6 +889,8 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.pt_stride = pt_stride;
   a.ctx = context_lens;
   a.q = static_cast<const uint16_t*>(q);
+  a.knew = static_cast<const uint16_t*>(k_new);
+  a.vnew = static_cast<const uint16_t*>(v_new);
   a.out = static_cast<uint16_t*>(out);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   const int64_t rows = (int64_t)batch * Hq * num_splits;

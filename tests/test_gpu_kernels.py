@@ -164,6 +164,70 @@ def test_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,splits", [
+    (24, 4, 256, 256, [5000, 257, 1], 76),   # new rows mid-page, at slot 0 of a page, alone
+    (8, 2, 128, 64, [64, 65, 999], 4),
+    (16, 2, 256, 128, [3000], 1),            # one split writes and reads directly
+])
+def test_fused_append_decode_equals_append_then_decode(Hq, Hkv, D, P, ctx, splits):
+    """jf_paged_decode_append_attn leaves the same pool bytes and output as
+    jf_kv_quantize_append of each request's newest row followed by
+    jf_paged_decode_attn, and both match the oracle."""
+    case = make_case(900 + sum(ctx), Hq, Hkv, D, P, ctx)
+    req, pos = case.req.numpy(), case.pos.numpy()
+    last = np.array([np.nonzero(req == b)[0].max() for b in range(len(ctx))])
+    keep = np.setdiff1d(np.arange(len(req)), last)
+    prefix = OA.new_pool(case.layout, case.num_pages, fill=0xFF)
+    OA.append(prefix, case.layout, case.page_table.numpy(), req[keep], pos[keep],
+              bits(case.k[keep]), bits(case.v[keep]))
+    full = case.oracle_pool(fill=0xFF)
+    k_new = case.k[last].contiguous()
+    v_new = case.v[last].contiguous()
+    B = len(ctx)
+    pt = case.page_table.to(DEV)
+    ctx_t = torch.tensor(ctx, dtype=torch.int32, device=DEV)
+    scale = 1 / math.sqrt(D)
+
+    pool_a = pool_from_numpy(case, prefix)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool_a, pt, torch.arange(B, dtype=torch.int32, device=DEV),
+                             (ctx_t - 1).contiguous(), k_new.to(DEV), v_new.to(DEV), err)
+    out_a = torch.full((B, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws_a = jf.decode_workspace(B, Hq, Hkv, D, splits, device=DEV)
+    jf.jf_paged_decode_attn(pool_a, pt, ctx_t, case.q.to(DEV), scale, out_a, ws_a, splits)
+
+    pool_b = pool_from_numpy(case, prefix)
+    out_b = torch.full((B, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws_b = jf.decode_workspace(B, Hq, Hkv, D, splits, device=DEV)
+    ws_b[256:] = 0xFF
+    jf.jf_paged_decode_append_attn(pool_b, pt, ctx_t, k_new.to(DEV), v_new.to(DEV),
+                                   case.q.to(DEV), scale, out_b, ws_b, splits)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws_a) == 0 and jf.workspace_status(ws_b) == 0
+    assert torch.equal(pool_a.data, pool_b.data)
+    assert np.array_equal(pool_b.data.cpu().numpy(), full)       # bit-exact quantize-append
+    assert torch.equal(out_a, out_b)
+    ref = OT.paged_decode(full, case.layout, case.page_table.numpy(), ctx, bits(case.q), scale)
+    assert_attention_close(out_b, ref)
+
+
+def test_fused_append_decode_reports_bad_page_id():
+    case = make_case(911, 8, 2, 128, 64, [100])
+    pool = pool_from_numpy(case, case.oracle_pool())
+    pt = case.page_table.clone()
+    pt[0, 1] = 10 ** 6                      # the page of position 99 (and 64..98)
+    out = torch.zeros((1, 8, 128), dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(1, 8, 2, 128, 2, device=DEV)
+    before = pool.data.clone()
+    ctx_t = torch.tensor([100], dtype=torch.int32, device=DEV)
+    jf.jf_paged_decode_append_attn(pool, pt.to(DEV), ctx_t, case.k[99:100].contiguous().to(DEV),
+                                   case.v[99:100].contiguous().to(DEV), case.q.to(DEV), 0.1, out,
+                                   ws, 2)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) & jf.binding.JF_DEV_ERR_PAGE_ID
+    assert torch.equal(pool.data, before)    # nothing written anywhere
+
+
 def test_decode_edge_contexts():
     case = make_case(5, 8, 2, 128, 64, [0, 1, 64, 65])
     ref_pool = case.oracle_pool()
