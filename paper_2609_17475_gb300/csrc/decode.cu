@@ -2,8 +2,9 @@
 // decode reads the compressed pages where they are used; Sec. 2, Eq. 3: never
 // size temporaries by the history length; Eq. 5: contiguous GQA head groups).
 //
-// Kernel 1 (split phase).  CTA = (split s, KV head, request b), 6 warps.  The
-// split's 32-position chunks are dealt round-robin to the warps; each warp owns
+// Kernel 1 (split phase).  CTA = (split s, KV head, request b), 6 warps.  A
+// split takes a contiguous range of the context's 32-position chunks and
+// deals them round-robin to its warps; each warp owns
 // a private ring of DSTAGES shared-memory stages that it refills itself with
 // TMA: a 5-D tiled copy (128-byte swizzle) for the K and V code rows of the
 // chunk and two 1-D bulk copies for their scale/bias words.
@@ -151,8 +152,8 @@ struct DecodeSmem {
   // which the 128-byte TMA swizzle of the code buffers needs.
   static constexpr int TOTAL = CODES_BYTES + SB_BYTES + QF_BYTES + BAR_BYTES;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
-  static_assert(DWARPS * 8 * D * 4 <= CODES_BYTES, "combine buffer must fit");
-  static_assert(DWARPS * 8 * (2 + NG) * 4 <= SB_BYTES, "combine ml/bias buffer must fit");
+  static_assert(DWARPS * 8 * (D + 4) * 4 <= CODES_BYTES, "combine buffer must fit");
+  static_assert((DWARPS * 8 * 3 + 16) * 4 <= SB_BYTES, "combine (m, l), weights must fit");
 };
 
 // Per-warp online-softmax state.  Thread (r, c) of the warp owns query heads
@@ -443,13 +444,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   }
   const int c_begin = split * cps;
   const int c_end = min(c_begin + cps, nch);
-  const int my_n = (c_end - c_begin > warp) ? (c_end - c_begin - warp + DWARPS - 1) / DWARPS : 0;
+  const int n_cta = c_end - c_begin;
+  const int my_n = (n_cta > warp) ? (n_cta - warp + DWARPS - 1) / DWARPS : 0;
+  auto chunk_of = [&](int it) { return c_begin + warp + it * DWARPS; };
 
   if (!aligned) {
     if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
     return;
   }
-  if (a.knew != nullptr && split == nsplit - 1) {   // CTA-uniform
+  if (a.knew != nullptr && split == nsplit - 1) {   // owns the last chunk
     // the new row goes to the pool before this split's TMA reads it
     append_new_row<D>(a, b, kvh, ctx - 1, warp, lane);
     fence_proxy_async_global();
@@ -541,7 +544,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const int it = blk * 32 + lane;
     int page = -1;
     if (it < my_n) {
-      const int pidx = ((c_begin + warp + it * DWARPS) * DTOK) >> a.log2P;
+      const int pidx = (chunk_of(it) * DTOK) >> a.log2P;
       if (pidx < a.pt_stride) page = __ldg(a.page_table + (int64_t)b * a.pt_stride + pidx);
     }
     return page;
@@ -560,7 +563,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const int page = __shfl_sync(0xffffffffu, pg_cur, it & 31);
     const bool ok = page >= 0 && page < a.num_pages;
     if (lane == 0) {
-      const int inp = ((c_begin + warp + it * DWARPS) * DTOK) & (a.P - 1);
+      const int inp = (chunk_of(it) * DTOK) & (a.P - 1);
       uint64_t* bar = &bars[warp * DSTAGES + s];
       if (!ok) {
         flag_error(a.status, JF_DEV_ERR_PAGE_ID);
@@ -614,7 +617,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     }
     done = it + 1;
     const bool ok = (valid >> s) & 1u;
-    const int tokbase = (c_begin + warp + it * DWARPS) * DTOK;
+    const int tokbase = chunk_of(it) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF);
     const uint8_t* ksb = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
     if (ok && tokbase + DTOK <= ctx)
@@ -656,21 +659,29 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
   }
   __syncthreads();   // every warp is past its last stage: reuse the rings
-  float* so = reinterpret_cast<float*>(codes);    // [DWARPS][8][D]
+  // Each warp's O (rows padded by 4 floats: the 128-bit stores of one
+  // quarter-warp hit 8 distinct bank groups) and (m, l) per head.
+  constexpr int SROW = D + 4;
+  float* so = reinterpret_cast<float*>(codes);    // [DWARPS][8][SROW]
   float* sml = reinterpret_cast<float*>(sbuf);    // [DWARPS][8][2]
+  float* swt = sml + DWARPS * 8 * 2;              // [DWARPS][8] combine weights
+  float* shl = swt + DWARPS * 8;                  // [8][2] (M, L) per head
   {
-    float* w0 = so + (warp * 8 + 2 * c) * D;
-    float* w1 = w0 + D;
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float fe = (e & 1) ? 1048576.f : 16777216.f;   // 2^24, or 2^24/16 for hi nibbles
-        const int d0 = 64 * g + 4 * r + e, d1 = d0 + 32;
-        w0[d0] = fmaf(O[g][e][0], fe, Bs[g][0]);
-        w1[d0] = fmaf(O[g][e][1], fe, Bs[g][1]);
-        w0[d1] = fmaf(O[g][e][2], fe, Bs[g][0]);
-        w1[d1] = fmaf(O[g][e][3], fe, Bs[g][1]);
+      for (int hf = 0; hf < 2; ++hf) {          // d block 64g + 32 hf + 4r + e
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {        // head 2c + hh
+          float4 v;
+          // 2^24 undoes the fp16 subnormal codes (2^20 for the hi nibbles)
+          v.x = fmaf(O[g][0][2 * hf + hh], 16777216.f, Bs[g][hh]);
+          v.y = fmaf(O[g][1][2 * hf + hh], 1048576.f, Bs[g][hh]);
+          v.z = fmaf(O[g][2][2 * hf + hh], 16777216.f, Bs[g][hh]);
+          v.w = fmaf(O[g][3][2 * hf + hh], 1048576.f, Bs[g][hh]);
+          *reinterpret_cast<float4*>(so + (warp * 8 + 2 * c + hh) * SROW + 64 * g + 32 * hf +
+                                     4 * r) = v;
+        }
       }
     }
     if (r == 0) {
@@ -683,37 +694,61 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   __syncthreads();
 
   // ---- combine the warps of this CTA --------------------------------------
-  for (int idx = threadIdx.x; idx < a.G * D; idx += blockDim.x) {
-    const int h = idx / D, d = idx % D;
+  // per head: M = max_w m_w, weights 2^(m_w - M) (divided by L when this CTA
+  // writes the final output), L = sum_w 2^(m_w - M) l_w
+  if (threadIdx.x < a.G) {
+    const int h = threadIdx.x;
     float M = NEG_INF;
 #pragma unroll
     for (int w = 0; w < DWARPS; ++w) M = fmaxf(M, sml[(w * 8 + h) * 2]);
-    float Lsum = 0.f, Osum = 0.f;
-    if (M != NEG_INF) {
+    float f[DWARPS];
+    float L = 0.f;
 #pragma unroll
-      for (int w = 0; w < DWARPS; ++w) {
-        const float mw = sml[(w * 8 + h) * 2];
-        if (mw != NEG_INF) {
-          const float f = fast_exp2(mw - M);
-          Lsum = fmaf(f, sml[(w * 8 + h) * 2 + 1], Lsum);
-          Osum = fmaf(f, so[(w * 8 + h) * D + d], Osum);
-        }
+    for (int w = 0; w < DWARPS; ++w) {
+      const float mw = sml[(w * 8 + h) * 2];
+      f[w] = (mw != NEG_INF) ? fast_exp2(mw - M) : 0.f;
+      L = fmaf(f[w], sml[(w * 8 + h) * 2 + 1], L);
+    }
+    const float inv = direct ? (L > 0.f ? 1.f / L : 0.f) : 1.f;
+#pragma unroll
+    for (int w = 0; w < DWARPS; ++w) swt[w * 8 + h] = f[w] * inv;
+    shl[h * 2 + 0] = M;
+    shl[h * 2 + 1] = L;
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < a.G * (D / 4); idx += blockDim.x) {
+    const int h = idx / (D / 4), d = 4 * (idx % (D / 4));
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < DWARPS; ++w) {
+      const float f = swt[w * 8 + h];
+      const float4 v = *reinterpret_cast<const float4*>(so + (w * 8 + h) * SROW + d);
+      if (f != 0.f) {
+        acc.x = fmaf(f, v.x, acc.x);
+        acc.y = fmaf(f, v.y, acc.y);
+        acc.z = fmaf(f, v.z, acc.z);
+        acc.w = fmaf(f, v.w, acc.w);
       }
     }
     const int hq = hq0 + h;
     if (direct) {
-      a.out[((int64_t)b * a.Hq + hq) * D + d] =
-          __bfloat16_as_ushort(__float2bfloat16_rn(Lsum > 0.f ? Osum / Lsum : 0.f));
+      uint2 o;
+      o.x = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.x)) |
+            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.y)) << 16);
+      o.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.z)) |
+            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.w)) << 16);
+      *reinterpret_cast<uint2*>(a.out + ((int64_t)b * a.Hq + hq) * D + d) = o;
     } else {
       const int64_t row = ((int64_t)b * a.Hq + hq) * a.num_splits + split;
-      a.part_o[row * D + d] = Osum;
+      *reinterpret_cast<float4*>(a.part_o + row * D + d) = acc;
       if (d == 0) {
-        a.part_ml[row * 2 + 0] = M;
-        a.part_ml[row * 2 + 1] = Lsum;
+        a.part_ml[row * 2 + 0] = shl[h * 2 + 0];
+        a.part_ml[row * 2 + 1] = shl[h * 2 + 1];
       }
     }
   }
 }
+
 
 // One CTA per (32-wide slice of head_dim, query head, request); its 8 warps
 // take interleaved splits and reduce through shared memory, so the merge is
