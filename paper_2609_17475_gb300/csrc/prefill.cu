@@ -9,26 +9,32 @@
 //
 // CTA = (tile of QPC = 128 / G queries, KV head); its 128 MMA rows are the
 // (query, head) pairs r = i * G + j of the G query heads that share the KV
-// head, so every dequantized K/V tile is reused by all of them.  Warp roles:
-//   warp 0      TMEM allocation; lane 0 issues every tcgen05.mma:
+// head, so every dequantized K/V tile is reused by all of them.  Two CTAs on
+// two SMs form a pair (a cluster of 2, tcgen05 cta_group::2): the pair runs
+// M = 256 MMAs over the same K/V tiles, and each CTA dequantizes only half of
+// every tile -- 32 of its 64 K rows (the N half of S = Q K^T it supplies) and
+// D/2 of the V columns (its N half of O += P V) -- so the dequantization work
+// per SM is halved while each SM's tensor core still does its 128 rows.
+// Warp roles (each CTA):
+//   warp 0      TMEM allocation (512 columns, pair-wide); in CTA 0, lane 0
+//               issues every tcgen05.mma.cta_group::2 of the pair:
 //                 S_j  = Q  K_j^T   (A = Q in TMEM, B = K_j smem, K-major)
 //                 O   += P_j V_j    (A = P_j in TMEM, B = V_j smem, MN-major)
+//               and commits to the barrier of both CTAs (multicast).
 //               TMEM columns: O [0, D), two S/P buffers of 64, Q [D + 128, +D/2);
 //               P_j (fp16) overwrites the first half of S_j once it is read.
-//   warps 1-8   dequantize 64-position K/V tiles from the pool (page-table
-//               lookup, 4-bit codes -> fp16 integers through the mantissa of
-//               fp16 1024, then x = code * scale + bias with one fused
-//               multiply-add) into
-//               three 128B-swizzled tile buffers; each thread owns one
-//               position's 32 contiguous code bytes per 64-wide block, loads
-//               run two tiles ahead, and the 8 lanes of a quarter-warp store
-//               8 different positions (distinct swizzled chunks, no bank
-//               conflicts);
+//   warps 1-8   dequantize this CTA's halves of 64-position K/V tiles from
+//               the pool (page-table lookup, 4-bit codes -> fp16 integers
+//               through the mantissa of fp16 1024, then x = code * scale +
+//               bias with one fused multiply-add) into four 128B-swizzled
+//               half-tile buffers, one item (one position's code bytes of a
+//               64-wide block) per thread, loads running two tiles ahead;
+//               each warp then arrives on CTA 0's tile barrier.
 //   warps 9-12  one thread per row: Q row -> TMEM at the start; online
-//               softmax on S (tcgen05.ld), P back
-//               to TMEM as fp16 (tcgen05.st); the running maximum is moved
-//               only when it grows by more than 2^8, and then O is rescaled
-//               in TMEM; finally O / l -> bf16 output.
+//               softmax on S (tcgen05.ld), P back to TMEM as fp16
+//               (tcgen05.st) and an arrive on CTA 0's P barrier; the running
+//               maximum is moved only when it grows by more than 2^8, and
+//               then O is rescaled in TMEM; finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
 // 0,4,1,5,2,6,3,7 (the pairs one 32-bit word of codes yields); Q uses the same
 // order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
@@ -40,12 +46,12 @@
 
 namespace jfkv {
 
-constexpr int PF_BM = 128;   // MMA rows per CTA
+constexpr int PF_BM = 128;   // MMA rows per CTA (256 per CTA pair)
 constexpr int PF_BN = 64;    // positions per K/V tile
 constexpr int PF_DQ_WARPS = 8;
 constexpr int PF_SM_WARPS = 4;
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
-constexpr int PF_KVBUF = 3;     // K/V tile buffers in shared memory
+constexpr int PF_KVBUF = 4;     // K/V half-tile buffers in shared memory
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
 
 struct PrefillArgs {
@@ -62,15 +68,19 @@ struct PrefillArgs {
   int32_t q_start, C, causal;
   float scale_log2;
   int32_t* status;
-  int32_t n_qtiles;
+  int32_t n_tiles2;   // query tiles, rounded up to pairs
 };
 
+// Each CTA of a pair holds half of every K/V tile: K rows 32 r .. 32 r + 31
+// (all of head_dim, K-major) and V columns D/2 r .. D/2 (r + 1) (all 64
+// positions, MN-major), r = its rank in the pair.
 template <int D>
 struct PfSmem {
-  static constexpr int T_BYTES = PF_BN * D * 2;
+  static constexpr int KT_BYTES = (PF_BN / 2) * D * 2;   // [D/64][32 rows][128 B]
+  static constexpr int VT_BYTES = PF_BN * (D / 2) * 2;   // [D/128][64 rows][128 B]
   static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = PF_KVBUF * T_BYTES;
-  static constexpr int OFF_BAR = 2 * PF_KVBUF * T_BYTES;
+  static constexpr int OFF_V = PF_KVBUF * KT_BYTES;
+  static constexpr int OFF_BAR = OFF_V + PF_KVBUF * VT_BYTES;
   static constexpr int TOTAL = 1024 + OFF_BAR + 256;
 };
 
@@ -113,15 +123,19 @@ __device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2)
 }
 
 template <int D>
-__global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArgs a) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PF_THREADS, 1)
+prefill_kernel(const PrefillArgs a) {
   using L = PfSmem<D>;
   constexpr int NKB = D / 64;           // 64-wide d blocks
-  constexpr int CB = D / 2;
-  constexpr int SBB = D / 16;
   constexpr int UPI = (D == 256) ? 2 : 1;   // 16-byte code units per dequant item
-  static_assert(PF_BN * NKB * 2 / UPI == 32 * PF_DQ_WARPS, "one item per dequant thread");
-  constexpr uint32_t IDQK = tc::idesc_f16_f32(PF_BM, PF_BN, 0, 0);
-  constexpr uint32_t IDPV = tc::idesc_f16_f32(PF_BM, D, 0, 1);
+  constexpr int SBB = D / 16;
+  constexpr int CB = D / 2;
+  // 128 K items (32 positions x NKB blocks x 2/UPI units) + 128 V items
+  // (64 positions x NKB/2 blocks x 2/UPI units): one per dequant thread
+  static_assert((PF_BN / 2) * NKB * 2 / UPI == 128 && PF_BN * (NKB / 2) * 2 / UPI == 128,
+                "one item per dequant thread");
+  constexpr uint32_t IDQK = tc::idesc_f16_f32(2 * PF_BM, PF_BN, 0, 0);
+  constexpr uint32_t IDPV = tc::idesc_f16_f32(2 * PF_BM, D, 0, 1);
 
   extern __shared__ uint8_t smraw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) &
@@ -129,36 +143,47 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   uint8_t* sK = sm + L::OFF_K;
   uint8_t* sV = sm + L::OFF_V;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::OFF_BAR);
-  uint64_t* kv_full = bars + 0;                // [PF_KVBUF]
-  uint64_t* pv_done = bars + PF_KVBUF;         // [PF_KVBUF]
-  uint64_t* s_full = bars + 2 * PF_KVBUF;      // [2]
-  uint64_t* p_full = bars + 2 * PF_KVBUF + 2;  // [2]
+  uint64_t* kv_full = bars + 0;                // [PF_KVBUF] on CTA 0: both CTAs' halves stored
+  uint64_t* pv_done = bars + PF_KVBUF;         // [PF_KVBUF] both CTAs: P V of the tile done
+  uint64_t* s_full = bars + 2 * PF_KVBUF;      // [2] both CTAs: S ready
+  uint64_t* p_full = bars + 2 * PF_KVBUF + 2;  // [2] on CTA 0: both CTAs' P stored
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * PF_KVBUF + 4);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qt = a.n_qtiles - 1 - (int)blockIdx.x;   // latest (longest) query tiles first
+  const uint32_t rank = tc::cluster_rank();
+  // query tile of this CTA and of its partner: latest (longest) tiles first
+  const int qt = a.n_tiles2 - 1 - (int)blockIdx.x;
+  const int qt_partner = a.n_tiles2 - 1 - (int)(blockIdx.x ^ 1u);
   const int kvh = blockIdx.y;
   const int q0 = qt * a.QPC;
-  const int nq = min(a.QPC, a.C - q0);
+  const int nq = max(0, min(a.QPC, a.C - q0));
   const int rows = nq * a.G;
   const int total = a.q_start + a.C;
-  const int kmax = a.causal ? a.q_start + q0 + nq : total;
-  const int ntiles = (kmax + PF_BN - 1) / PF_BN;
+  // positions a query tile attends (0 for the padding tile of an odd count)
+  auto kmax_of = [&](int t) {
+    const int first = t * a.QPC;
+    const int n = max(0, min(a.QPC, a.C - first));
+    return n == 0 ? 0 : (a.causal ? a.q_start + first + n : total);
+  };
+  const int kmax = kmax_of(qt);
+  const int kmax_pair = max(kmax, kmax_of(qt_partner));
+  const int ntiles = (kmax_pair + PF_BN - 1) / PF_BN;   // the pair walks the same tiles
 
-  if (warp == 0) tc::alloc(tmem_slot, 512);
   if (threadIdx.x == 0) {
     for (int i = 0; i < PF_KVBUF; ++i) {
-      mbar_init(&kv_full[i], PF_DQ_WARPS);
+      mbar_init(&kv_full[i], 2 * PF_DQ_WARPS);
       mbar_init(&pv_done[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_full[i], PF_SM_WARPS);
+      mbar_init(&p_full[i], 2 * PF_SM_WARPS);
     }
     fence_barrier_init();
   }
+  if (warp == 0) tc::alloc2(tmem_slot, 512);
   tc::fence_before();
   __syncthreads();
+  tc::cluster_sync();   // both CTAs: barriers initialized, TMEM allocated
   tc::fence_after();
   const uint32_t tbase = *tmem_slot;
   const uint32_t tO = tbase;
@@ -210,35 +235,36 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
   }
   tc::fence_before();
   __syncthreads();
+  tc::cluster_sync();   // both CTAs' Q rows are in TMEM before the first MMA
   tc::fence_after();
 
   if (warp == 0) {
-    // ================= MMA issuer =================
-    if (lane == 0) {
+    // ================= MMA issuer (CTA 0 of the pair) =================
+    if (rank == 0 && lane == 0) {
       const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV);
       bool ok = true;
       auto pv = [&](int j) {
         const int sb = j & 1, kb = j % PF_KVBUF;
-        if (!mbar_wait_bounded(&p_full[sb], (j >> 1) & 1)) { ok = false; return; }
+        if (!tc::wait_cluster(&p_full[sb], (j >> 1) & 1)) { ok = false; return; }
         tc::fence_after();
 #pragma unroll
         for (int k = 0; k < PF_BN / 16; ++k)
-          tc::mma_ts(tO, tS + sb * PF_BN + 8 * k,
-                     tc::sdesc_sw128(vaddr + kb * L::T_BYTES + k * 2048, PF_BN * 128, 1024), IDPV,
-                     (j > 0 || k > 0) ? 1u : 0u);
-        tc::commit(&pv_done[kb]);
+          tc::mma2_ts(tO, tS + sb * PF_BN + 8 * k,
+                      tc::sdesc_sw128(vaddr + kb * L::VT_BYTES + k * 2048, PF_BN * 128, 1024),
+                      IDPV, (j > 0 || k > 0) ? 1u : 0u);
+        tc::commit2_both(&pv_done[kb]);
       };
       for (int j = 0; j < ntiles && ok; ++j) {
         const int sb = j & 1, kb = j % PF_KVBUF;
-        if (!mbar_wait_bounded(&kv_full[kb], (j / PF_KVBUF) & 1)) { ok = false; break; }
+        if (!tc::wait_cluster(&kv_full[kb], (j / PF_KVBUF) & 1)) { ok = false; break; }
         tc::fence_after();
 #pragma unroll
         for (int ks = 0; ks < D / 16; ++ks)
-          tc::mma_ts(tS + sb * PF_BN, tQ + 8 * ks,
-                     tc::sdesc_sw128(kaddr + kb * L::T_BYTES + (ks >> 2) * (PF_BN * 128) +
-                                         (ks & 3) * 32, 16, 1024),
-                     IDQK, ks ? 1u : 0u);
-        tc::commit(&s_full[sb]);
+          tc::mma2_ts(tS + sb * PF_BN, tQ + 8 * ks,
+                      tc::sdesc_sw128(kaddr + kb * L::KT_BYTES + (ks >> 2) * ((PF_BN / 2) * 128) +
+                                          (ks & 3) * 32, 16, 1024),
+                      IDQK, ks ? 1u : 0u);
+        tc::commit2_both(&s_full[sb]);
         if (j >= 1) pv(j - 1);
       }
       if (ok) pv(ntiles - 1);
@@ -246,45 +272,52 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     }
     __syncwarp();
   } else if (warp <= PF_DQ_WARPS) {
-    // ================= dequantization =================
-    // item = (position t, 64-wide block kb[, half u]): UPI 16-byte code units
-    const int dt = (int)threadIdx.x - 32;   // 0 .. 32*PF_DQ_WARPS-1
-    const int t = dt % PF_BN;
-    const int rest = dt / PF_BN;
-    const int kb = (UPI == 2) ? rest : rest >> 1;
-    const int u0 = (UPI == 2) ? 0 : (rest & 1);
+    // ================= dequantization (this CTA's halves) =================
+    // threads 0..127: K item (position 32 rank + t of the tile, block kb, unit u0)
+    // threads 128..255: V item (position t, block D/128 * rank + kbl, unit u0)
+    const int dt = (int)threadIdx.x - 32;
+    const bool is_v = dt >= 128;
+    const int e = is_v ? dt - 128 : dt;
+    const int t = is_v ? (e % PF_BN) : (e % (PF_BN / 2));
+    const int rest = is_v ? (e / PF_BN) : (e / (PF_BN / 2));
+    const int kbl = (UPI == 2) ? rest : (is_v ? 0 : rest >> 1);
+    const int u0 = (UPI == 2) ? 0 : (is_v ? rest : rest & 1);
+    const int kb = is_v ? (NKB / 2) * (int)rank + kbl : kbl;
+    const int tpos = is_v ? t : (PF_BN / 2) * (int)rank + t;   // position within the tile
+    uint8_t* dst_base = is_v ? sV + kbl * (PF_BN * 128) + t * 128
+                             : sK + kbl * ((PF_BN / 2) * 128) + t * 128;
+    const int tile_bytes = is_v ? L::VT_BYTES : L::KT_BYTES;
+    const int64_t code_off = (is_v ? a.codes_region : 0) + kb * 32 + u0 * 16;
+    const int64_t sb_off = a.sb_base + (is_v ? a.sb_region : 0) + kb * 4;
     struct Tile {
-      uint4 k[UPI], v[UPI];
-      uint32_t ks, vs;
+      uint4 c[UPI];
+      uint32_t sbw;
       bool valid;
     };
-    auto load_tile = [&](int j, Tile& x) {
+    // page id of tile j (P >= 64, so a tile lies in one page); it is loaded a
+    // step before its tile's code loads need it
+    auto page_of = [&](int j) -> int { return j < ntiles ? __ldg(a.pt + (j * PF_BN) / a.P) : -1; };
+    auto load_tile = [&](int j, int page, Tile& x) {
       const int key0 = j * PF_BN;
-      const int page = __ldg(a.pt + key0 / a.P);
       const bool pok = page >= 0 && page < a.num_pages;
       if (!pok && dt == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
-      x.valid = pok && (key0 + t < kmax);
+      x.valid = pok && (key0 + tpos < kmax_pair);
       if (x.valid) {
         const uint8_t* base = a.pool + (int64_t)page * a.page_bytes;
-        const int64_t row = (int64_t)kvh * a.P + key0 % a.P + t;
-        const uint8_t* kp = base + row * CB + kb * 32 + u0 * 16;
+        const int64_t row = (int64_t)kvh * a.P + key0 % a.P + tpos;
+        const uint8_t* cp = base + code_off + row * CB;
 #pragma unroll
-        for (int u = 0; u < UPI; ++u) {
-          x.k[u] = __ldg(reinterpret_cast<const uint4*>(kp + 16 * u));
-          x.v[u] = __ldg(reinterpret_cast<const uint4*>(kp + a.codes_region + 16 * u));
-        }
-        const uint8_t* sp = base + a.sb_base + row * SBB + kb * 4;
-        x.ks = __ldg(reinterpret_cast<const uint32_t*>(sp));
-        x.vs = __ldg(reinterpret_cast<const uint32_t*>(sp + a.sb_region));
+        for (int u = 0; u < UPI; ++u) x.c[u] = __ldg(reinterpret_cast<const uint4*>(cp + 16 * u));
+        x.sbw = __ldg(reinterpret_cast<const uint32_t*>(base + sb_off + row * SBB));
       }
     };
-    auto store_half = [&](uint8_t* tile, const uint4 (&codes)[UPI], uint32_t sbw, bool valid) {
+    auto store = [&](uint8_t* tile, const Tile& x) {
       uint32_t s2, b2;
-      sb_to_h2(sbw, s2, b2);
+      sb_to_h2(x.sbw, s2, b2);
       uint4 o[UPI][4];
 #pragma unroll
       for (int u = 0; u < UPI; ++u) {
-        const uint32_t cw[4] = {codes[u].x, codes[u].y, codes[u].z, codes[u].w};
+        const uint32_t cw[4] = {x.c[u].x, x.c[u].y, x.c[u].z, x.c[u].w};
 #pragma unroll
         for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
       }
@@ -293,28 +326,28 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
           const int cc = (u0 + u) * 4 + w;
-          *reinterpret_cast<uint4*>(tile + kb * (PF_BN * 128) + t * 128 + ((cc ^ (t & 7)) << 4)) =
-              valid ? o[u][w] : make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(tile + ((cc ^ (t & 7)) << 4)) =
+              x.valid ? o[u][w] : make_uint4(0, 0, 0, 0);
         }
     };
     // Three register tiles rotate by name (the loop is unrolled by 3), so the
-    // loads for tile j + 2 stay in flight while tile j is converted; copying
-    // registers instead would wait for those loads.
+    // loads for tile j + 2 stay in flight while tile j is converted.
     Tile ta, tb, tcur;
     bool ok = true;
-    auto step = [&](int j, const Tile& cur, Tile& dst) {
-      if (j + 2 < ntiles) load_tile(j + 2, dst);
+    int pg_next = page_of(2);
+    auto step = [&](int j, const Tile& cur, Tile& nxt) {
+      if (j + 2 < ntiles) load_tile(j + 2, pg_next, nxt);
+      pg_next = page_of(j + 3);
       const int kbuf = j % PF_KVBUF;
       if (j >= PF_KVBUF &&
-          !mbar_wait_bounded(&pv_done[kbuf], ((j - PF_KVBUF) / PF_KVBUF) & 1)) { ok = false; return; }
-      store_half(sK + kbuf * L::T_BYTES, cur.k, cur.ks, cur.valid);
-      store_half(sV + kbuf * L::T_BYTES, cur.v, cur.vs, cur.valid);
+          !tc::wait_cluster(&pv_done[kbuf], ((j - PF_KVBUF) / PF_KVBUF) & 1)) { ok = false; return; }
+      store(dst_base + kbuf * tile_bytes, cur);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&kv_full[kbuf]);
+      if (lane == 0) tc::arrive_cluster(&kv_full[kbuf], 0);
     };
-    load_tile(0, ta);
-    if (ntiles > 1) load_tile(1, tb);
+    load_tile(0, page_of(0), ta);
+    if (ntiles > 1) load_tile(1, page_of(1), tb);
     for (int j = 0; j < ntiles && ok; j += 3) {
       step(j, ta, tcur);
       if (j + 1 < ntiles && ok) step(j + 1, tb, ta);
@@ -322,17 +355,17 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     }
     if (!ok && dt == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
   } else {
-    // ================= softmax + epilogue =================
+    // ================= softmax + epilogue (this CTA's 128 rows) =================
     // Rows past the chunk (padding) see every position: their Q rows are zero
     // and their outputs are never stored, and keeping them unmasked keeps the
     // warp on the same (mask-free) path as its real rows.
-    const int limit = (row_ok && a.causal) ? a.q_start + q0 + qi : kmax - 1;
+    const int limit = (row_ok && a.causal) ? a.q_start + q0 + qi : kmax_pair - 1;
     const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
       const int b = j & 1;
-      if (!mbar_wait_bounded(&s_full[b], (j >> 1) & 1)) { ok = false; break; }
+      if (!tc::wait_cluster(&s_full[b], (j >> 1) & 1)) { ok = false; break; }
       tc::fence_after();
       uint32_t s0[32], s1[32];
       tc::ld32(tS + b * PF_BN + lane_off, s0);
@@ -369,7 +402,7 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
         const float nref = need ? mt : m_ref;
         const float f = (need && m_ref != -INFINITY) ? fast_exp2(m_ref - nref) : 1.f;
         if (j > 0) {
-          if (!mbar_wait_bounded(&pv_done[(j - 1) % PF_KVBUF], ((j - 1) / PF_KVBUF) & 1)) {
+          if (!tc::wait_cluster(&pv_done[(j - 1) % PF_KVBUF], ((j - 1) / PF_KVBUF) & 1)) {
             ok = false;
             break;
           }
@@ -402,10 +435,10 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
       tc::wait_st();
       tc::fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[b]);
+      if (lane == 0) tc::arrive_cluster(&p_full[b], 0);
     }
     // epilogue: O / l -> bf16, undoing the d order 0,4,1,5,2,6,3,7
-    if (ok && mbar_wait_bounded(&pv_done[(ntiles - 1) % PF_KVBUF],
+    if (ok && tc::wait_cluster(&pv_done[(ntiles - 1) % PF_KVBUF],
                                 ((ntiles - 1) / PF_KVBUF) & 1)) {
       tc::fence_after();
       const float inv = l > 0.f ? 1.f / l : 0.f;
@@ -438,11 +471,13 @@ __global__ void __launch_bounds__(PF_THREADS, 1) prefill_kernel(const PrefillArg
     if (!ok && lane == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
   }
 
+  // neither CTA may release TMEM or exit while its partner can still reach it
   tc::fence_before();
   __syncthreads();
+  tc::cluster_sync();
   if (warp == 0) {
     tc::fence_after();
-    tc::dealloc(tbase, 512);
+    tc::dealloc2(tbase, 512);
   }
 }
 
@@ -471,9 +506,10 @@ int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
   a.causal = causal ? 1 : 0;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.status = static_cast<int32_t*>(workspace);
-  a.n_qtiles = (chunk_len + a.QPC - 1) / a.QPC;
+  const int n_qtiles = (chunk_len + a.QPC - 1) / a.QPC;
+  a.n_tiles2 = (n_qtiles + 1) & ~1;   // CTA pairs
   if (g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
-  dim3 grid((unsigned)a.n_qtiles, (unsigned)g.Hkv);
+  dim3 grid((unsigned)a.n_tiles2, (unsigned)g.Hkv);
   if (g.D == 256) {
     static bool attr = false;
     if (!attr) {
