@@ -343,16 +343,21 @@ def _event_time(fn, reps, stream):
     return e0.elapsed_time(e1) / reps
 
 
-def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
-    """Append, prefill chunk, checkpoint, two-request and mixed-batch decode.
-    Every tensor is allocated on `stream`, the stream the kernels run on, so the
-    caching allocator never hands a buffer back out while a kernel still reads it."""
+ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed")
+
+
+def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
+    """Tiny decode, append, prefill chunk, decode loop, checkpoint, two-request and
+    mixed-batch decode (`only` selects one group of ROW_GROUPS).  Every tensor is
+    allocated on `stream`, the stream the kernels run on, so the caching allocator
+    never hands a buffer back out while a kernel still reads it."""
     with torch.cuda.stream(stream):
-        return _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf)
+        return _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only)
 
 
-def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
+def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
     out = {}
+    want = lambda name: only is None or only == name
 
     def check(section, *words):
         stream.synchronize()
@@ -364,6 +369,31 @@ def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
     g = torch.Generator(device=dev)
     g.manual_seed(4242)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
+    if want("tiny"):
+        # ---- tiny workload: 8/2/128, P 256, one request of 4,096 positions in
+        # 16 shuffled pages (L2-resident: a latency figure, not a bandwidth one)
+        gt = synth.generator(1)
+        geo = synth.WORKLOADS["tiny"]["geometry"]
+        kt, vt = synth.kv_rows(gt, 4096, geo.num_kv_heads, geo.head_dim)
+        ptt, npt = synth.page_tables(gt, [4096], geo.page_size)
+        poolt = jf.KVPool.allocate(npt, geo.page_size, geo.num_kv_heads, geo.head_dim, device=dev)
+        jf.jf_kv_quantize_append(poolt, ptt.to(dev), torch.zeros(4096, dtype=torch.int32, device=dev),
+                                 torch.arange(4096, dtype=torch.int32, device=dev), kt.to(dev),
+                                 vt.to(dev), err, stream=stream)
+        qt = synth.normal_bf16(gt, (1, geo.num_q_heads, geo.head_dim)).to(dev)
+        ot = torch.empty_like(qt)
+        st = jf.default_num_splits(1, geo.num_kv_heads)
+        wst = jf.decode_workspace(1, geo.num_q_heads, geo.num_kv_heads, geo.head_dim, st, device=dev)
+        ct = torch.tensor([4096], dtype=torch.int32, device=dev)
+        ptt = ptt.to(dev)
+        tt = _event_time(lambda: jf.jf_paged_decode_attn(poolt, ptt, ct, qt, 1 / math.sqrt(128), ot,
+                                                         wst, st, stream=stream), 50, stream)
+        check("tiny", wst)
+        out["tiny_4096_8q_2kv_128d"] = {"us": tt * 1e3, "positions_per_s": 4096 / (tt / 1e3)}
+        del poolt
+    if not want("prompt"):
+        return _bench_rows_rest(jf, synth, dev, stream, peaks_gbs, peak_tf, only, out, g, err,
+                                check, want)
     # ---- prefill-then-decode shapes: 24/4/256, P 256, 32K prompt + 6K decode
     Hq, Hkv, D, P = 24, 4, 256, 256
     prompt, chunk, steps = 32768, 2048, 6144
@@ -451,6 +481,16 @@ def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
                                       "frac_hbm": ck_bytes / (t_ck / 1e3) / 1e9 / peaks_gbs,
                                       "alg_bytes": ck_bytes}
     del pool, blob
+    return _bench_rows_rest(jf, synth, dev, stream, peaks_gbs, peak_tf, only, out, g, err, check,
+                            want)
+
+
+def _bench_rows_rest(jf, synth, dev, stream, peaks_gbs, peak_tf, only, out, g, err, check, want):
+    Hq, Hkv, D, P = 24, 4, 256, 256
+    scale = 1 / math.sqrt(D)
+    bpp = 2 * Hkv * (D // 2 + 4 * D // 64)
+    if not want("two_request"):
+        return _bench_rows_mixed(jf, synth, dev, stream, out, g, err, check, want)
     # ---- two requests, 196,608 + 131,072 positions, 1,280-page pool, 32 splits
     ctxs = [196608, 131072]
     gc = synth.generator(3)
@@ -474,6 +514,15 @@ def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf):
     out["two_request_320k_32_splits"] = {"us": t2 * 1e3, "positions_per_s": sum(ctxs) / (t2 / 1e3),
                                          "GBps": sum(ctxs) * bpp / (t2 / 1e3) / 1e9}
     del pool2
+    return _bench_rows_mixed(jf, synth, dev, stream, out, g, err, check, want)
+
+
+def _bench_rows_mixed(jf, synth, dev, stream, out, g, err, check, want):
+    if not want("mixed"):
+        return out
+    Hq, Hkv, D = 24, 4, 256
+    scale = 1 / math.sqrt(D)
+    bpp = 2 * Hkv * (D // 2 + 4 * D // 64)
     # ---- 32 requests, contexts uniform in [1,024, 65,536], page size sweep
     gm = synth.generator(5)
     ctxm = synth.context_lengths(gm, 32, 1024, 65536)
@@ -574,7 +623,21 @@ def main():
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
     ap.add_argument("--no-rows", dest="rows", action="store_false",
                     help="skip the append / prefill / checkpoint / multi-request measurements")
+    ap.add_argument("--row", choices=ROW_GROUPS, default=None,
+                    help="run only this group of the row measurements (for profiling) and "
+                         "print it; no bench line")
     args = ap.parse_args()
+    if args.row:
+        import paper_2609_17475_gb300 as jf
+        from paper_2609_17475_gb300 import synth
+        dev = torch.device("cuda", 0)
+        torch.cuda.set_device(dev)
+        hbm, _ = peaks()
+        pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+        peak_tf = float(json.load(open(pk))["bf16_tflops"]) if os.path.exists(pk) else 1900.0
+        stream = torch.cuda.Stream(device=dev)
+        print(json.dumps(bench_rows(jf, synth, dev, stream, hbm, peak_tf, only=args.row)))
+        return
     args.warmup = max(3, args.warmup)
     world, rank, local = dist_env()
     if world > 1 and args.impl == "ours":
