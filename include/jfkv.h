@@ -133,9 +133,15 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
  *                 Hkv, D, num_splits) bytes, 256-byte aligned.  Its first
  *                 int32 is the device status word (JF_DEV_* bits, ORed);
  *                 the caller zeroes it when it wants a fresh status.
- *   num_splits    >= 1: maximum number of split-K partitions per (request,
- *                 KV head).  Each partition keeps (max, sum, partial output)
- *                 in the workspace; a second kernel merges them.
+ *   num_splits    >= 1: split-K partitions per (request, KV head) that the
+ *                 workspace holds.  Each partition keeps (max, sum, partial
+ *                 output) in the workspace; a second kernel merges them.  A
+ *                 single request uses at most num_splits; a batch of 2 to
+ *                 1,024 requests shares its batch * num_splits partitions,
+ *                 cutting every request into pieces of one size chosen for
+ *                 the whole batch (so a long request may take more than
+ *                 num_splits and a short one fewer, and the split CTAs carry
+ *                 equal work).
  * Numerics: K codes and q enter fp16 tensor-core products with fp32
  * accumulation (q is rescaled by a power of two per KV head when max|q| >= 2^14,
  * so any finite bf16 q is accepted); the softmax runs in fp32 with the

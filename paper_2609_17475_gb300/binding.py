@@ -311,7 +311,11 @@ def jf_kv_restore(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
 
 
 def default_num_splits(batch: int, num_kv_heads: int, device=None) -> int:
-    """Splits per (request, KV head) so the split grid fills the GPU twice over."""
+    """Split cap per (request, KV head) so the split grid fills the GPU twice
+    over.  A batch plans its splits over all requests together, and its
+    workspace then needs room for about two more splits per request than an
+    even share (rounding up per request)."""
     props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
     target = 2 * props.multi_processor_count
-    return max(1, -(-target // (batch * num_kv_heads)))
+    per = -(-target // (batch * num_kv_heads))
+    return max(1, per if batch == 1 else per + 2)

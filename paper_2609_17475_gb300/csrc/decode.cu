@@ -67,6 +67,9 @@ struct DecodeArgs {
   int32_t* status;
   int32_t num_splits;
   float scale_log2;    // softmax_scale * log2(e)
+  int32_t B;           // requests
+  int32_t balanced;    // 1: batch split plan (balanced_plan), partial rows by global split
+  int32_t budget;      // balanced: target splits per KV head over the whole batch
 };
 
 __host__ __device__ inline void split_plan(int ctx, int num_splits, int& nch, int& cps,
@@ -76,6 +79,60 @@ __host__ __device__ inline void split_plan(int ctx, int num_splits, int& nch, in
   cps = (nch + num_splits - 1) / num_splits;
   if (cps < MIN_CPS) cps = MIN_CPS;
   nsplit = (nch + cps - 1) / cps;
+}
+
+// Batch split plan (B > 1).  Splits are sized for the whole batch, not per
+// request: with T the chunks of all requests, every request is cut into
+// pieces of cps = max(MIN_CPS, ceil(T / budget)) chunks, so each split CTA
+// streams about the same bytes however unequal the contexts are.  Request b
+// gets n_b = ceil(nch_b / cps) splits, numbered g0_b .. g0_b + n_b - 1 after
+// those of requests 0 .. b-1; the global number g names the split's partial
+// rows (g * Hq + hq).  Called by one whole warp; for a split CTA (x >= 0) it
+// finds the request and split of global split x (b = -1 when x is past the
+// last), for a merge CTA (want_b >= 0) the first global split and count of
+// request want_b.
+struct BalPlan {
+  int b, split, nsplit, g0, cps;
+};
+
+__device__ BalPlan balanced_plan(const DecodeArgs& a, int x, int want_b, int lane) {
+  const int64_t cap = (int64_t)a.pt_stride * a.P;
+  auto nch_of = [&](int bb) -> int {
+    int64_t c = a.ctx[bb];
+    c = c < 0 ? 0 : (c > cap ? cap : c);
+    return (int)((c + DTOK - 1) / DTOK);
+  };
+  long long T = 0;
+  for (int bb = lane; bb < a.B; bb += 32) T += nch_of(bb);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) T += __shfl_xor_sync(0xffffffffu, T, o);
+  int cps = (int)((T + a.budget - 1) / a.budget);
+  if (cps < MIN_CPS) cps = MIN_CPS;
+  BalPlan p{-1, 0, 0, 0, cps};
+  int base = 0;
+  for (int b0 = 0; b0 < a.B; b0 += 32) {
+    const int bb = b0 + lane;
+    const int n = (bb < a.B) ? (nch_of(bb) + cps - 1) / cps : 0;
+    int incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const int excl = base + incl - n;
+    const bool hit = (x >= 0) ? (bb < a.B && x >= excl && x < excl + n) : (bb == want_b);
+    const unsigned m = __ballot_sync(0xffffffffu, hit);
+    if (m) {
+      const int src = __ffs(m) - 1;
+      p.b = __shfl_sync(0xffffffffu, bb, src);
+      p.g0 = __shfl_sync(0xffffffffu, excl, src);
+      p.nsplit = __shfl_sync(0xffffffffu, n, src);
+      p.split = (x >= 0) ? x - p.g0 : 0;
+      return p;
+    }
+    base += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  return p;
 }
 
 __device__ __forceinline__ int checked_ctx(const DecodeArgs& a, int b) {
@@ -150,7 +207,8 @@ struct DecodeSmem {
   static constexpr int BAR_BYTES = NBUF * 8;
   // The dynamic shared window starts 1024-byte aligned (checked at run time),
   // which the 128-byte TMA swizzle of the code buffers needs.
-  static constexpr int TOTAL = CODES_BYTES + SB_BYTES + QF_BYTES + BAR_BYTES;
+  static constexpr int PLAN_BYTES = 16;                // batch plan broadcast
+  static constexpr int TOTAL = CODES_BYTES + SB_BYTES + QF_BYTES + BAR_BYTES + PLAN_BYTES;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
   static_assert(DWARPS * 8 * (D + 4) * 4 <= CODES_BYTES, "combine buffer must fit");
   static_assert((DWARPS * 8 * 3 + 16) * 4 <= SB_BYTES, "combine (m, l), weights must fit");
@@ -415,10 +473,11 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   uint4* qsm = reinterpret_cast<uint4*>(sbuf + L::SB_BYTES);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES + L::QF_BYTES);
 
-  const int split = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
+  const int kvh = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
   const bool direct = (a.num_splits == 1);
+  int* plan_sh = reinterpret_cast<int*>(sbuf + L::SB_BYTES + L::QF_BYTES + L::BAR_BYTES);
   // the swizzled TMA boxes need a 1024-byte aligned window
   const bool aligned = (smem_u32(smem_raw) & 1023) == 0;
   if (aligned) {   // setup that reads nothing a previous kernel writes
@@ -432,9 +491,37 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   // kernel (e.g. the append that wrote the newest position) before any read
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
-  const int ctx = checked_ctx(a, b);
-  int nch, cps, nsplit;
-  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  int split, b, ctx, nch, cps, nsplit;
+  int64_t prow;   // partial row of this split for query head hq: prow + hq * pstride
+  int pstride;
+  if (a.balanced) {
+    if (warp == 0) {
+      const BalPlan p = balanced_plan(a, (int)blockIdx.x, -1, lane);
+      if (lane == 0) {
+        plan_sh[0] = p.b;
+        plan_sh[1] = p.split;
+        plan_sh[2] = p.nsplit;
+        plan_sh[3] = p.cps;
+      }
+    }
+    __syncthreads();
+    b = plan_sh[0];
+    split = plan_sh[1];
+    nsplit = plan_sh[2];
+    cps = plan_sh[3];
+    if (b < 0) return;   // past the batch's last split
+    ctx = checked_ctx(a, b);
+    nch = (ctx + DTOK - 1) / DTOK;
+    prow = (int64_t)((int)blockIdx.x) * a.Hq;   // global split x = g0 + split
+    pstride = 1;
+  } else {
+    split = blockIdx.x;
+    b = blockIdx.z;
+    ctx = checked_ctx(a, b);
+    split_plan(ctx, a.num_splits, nch, cps, nsplit);
+    prow = (int64_t)b * a.Hq * a.num_splits + split;
+    pstride = a.num_splits;
+  }
   if (split >= nsplit) {
     if (direct && split == 0) {   // empty context: zero output
       for (int i = threadIdx.x; i < a.G * D; i += blockDim.x)
@@ -739,7 +826,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
             ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.w)) << 16);
       *reinterpret_cast<uint2*>(a.out + ((int64_t)b * a.Hq + hq) * D + d) = o;
     } else {
-      const int64_t row = ((int64_t)b * a.Hq + hq) * a.num_splits + split;
+      const int64_t row = prow + (int64_t)hq * pstride;
       *reinterpret_cast<float4*>(a.part_o + row * D + d) = acc;
       if (d == 0) {
         a.part_ml[row * 2 + 0] = shl[h * 2 + 0];
@@ -774,8 +861,29 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   const int d0 = blockIdx.x * MERGE_DSLICE, hq = blockIdx.y, b = blockIdx.z;
   const int t = threadIdx.x, dd = t % MERGE_DSLICE, sg = t / MERGE_DSLICE;
   const int lane = t & 31;
-  const int S = a.num_splits;
-  const int64_t row0 = ((int64_t)b * a.Hq + hq) * S;
+  // partials of split s: row row0 + s * rs.  Per-request plans put them at
+  // ((b Hq + hq) S + s) and are known only after the context is read, so all
+  // S rows are loaded speculatively; the batch plan numbers splits globally
+  // (row (g0 + s) Hq + hq) and is worked out first.
+  __shared__ int plan_sh[2];
+  int S = a.num_splits;
+  int64_t row0 = ((int64_t)b * a.Hq + hq) * S;
+  int64_t rs = 1;
+  int nsplit_bal = 0;
+  if (a.balanced) {
+    if (t < 32) {
+      const BalPlan p = balanced_plan(a, -1, b, lane);
+      if (lane == 0) {
+        plan_sh[0] = p.g0;
+        plan_sh[1] = p.nsplit;
+      }
+    }
+    __syncthreads();
+    row0 = (int64_t)plan_sh[0] * a.Hq + hq;
+    rs = a.Hq;
+    nsplit_bal = plan_sh[1];
+    S = nsplit_bal;
+  }
   const float2* ml = reinterpret_cast<const float2*>(a.part_ml) + row0;
   const float* po = a.part_o + row0 * D + d0 + dd;
 
@@ -785,20 +893,21 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 #pragma unroll
   for (int k = 0; k < MERGE_MLB; ++k) {
     const int s = lane + 32 * k;
-    mlv[k] = (s < S) ? ml[s] : make_float2(-INFINITY, 0.f);
+    mlv[k] = (s < S) ? ml[s * rs] : make_float2(-INFINITY, 0.f);
   }
 #pragma unroll
   for (int u = 0; u < MERGE_BATCH; ++u) {
     const int s = sg + MERGE_NSG * u;
-    ov[u] = (s < S) ? po[(int64_t)s * D] : 0.f;
-    mv[u] = (s < S) ? ml[s].x : -INFINITY;
+    ov[u] = (s < S) ? po[s * rs * D] : 0.f;
+    mv[u] = (s < S) ? ml[s * rs].x : -INFINITY;
   }
   int ctx = ctx_raw;
   const int64_t cap = (int64_t)a.pt_stride * a.P;
   if (ctx < 0) ctx = 0;
   if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
-  split_plan(ctx, S, nch, cps, nsplit);
+  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  if (a.balanced) nsplit = nsplit_bal;
   uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D + d0;
   if (nsplit == 0) {
     if (t < MERGE_DSLICE) orow[t] = 0;
@@ -810,7 +919,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 #pragma unroll
   for (int k = 0; k < MERGE_MLB; ++k)
     if (lane + 32 * k < nsplit) M = fmaxf(M, mlv[k].x);
-  for (int s = lane + 32 * MERGE_MLB; s < nsplit; s += 32) M = fmaxf(M, ml[s].x);
+  for (int s = lane + 32 * MERGE_MLB; s < nsplit; s += 32) M = fmaxf(M, ml[s * rs].x);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
 
@@ -821,7 +930,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
       if (lane + 32 * k < nsplit && mlv[k].x != -INFINITY)
         L = fmaf(fast_exp2(mlv[k].x - M), mlv[k].y, L);
     for (int s = lane + 32 * MERGE_MLB; s < nsplit; s += 32) {
-      const float2 v = ml[s];
+      const float2 v = ml[s * rs];
       if (v.x != -INFINITY) L = fmaf(fast_exp2(v.x - M), v.y, L);
     }
 #pragma unroll
@@ -835,8 +944,8 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 #pragma unroll
       for (int u = 0; u < MERGE_BATCH; ++u) {
         const int s = s0 + MERGE_NSG * u;
-        ov[u] = (s < nsplit) ? po[(int64_t)s * D] : 0.f;
-        mv[u] = (s < nsplit) ? ml[s].x : -INFINITY;
+        ov[u] = (s < nsplit) ? po[s * rs * D] : 0.f;
+        mv[u] = (s < nsplit) ? ml[s * rs].x : -INFINITY;
       }
 #pragma unroll
       for (int u = 0; u < MERGE_BATCH; ++u)
@@ -856,6 +965,22 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+constexpr int BAL_MAX_B = 1024;   // batch plan limit (each plan reads every context length)
+
+// SMs of the current device (cached per device)
+static int sm_count() {
+  static int cache[256] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return 152;
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+      n = 152;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
 // rows (positions) of one TMA box of the decode code tensor map
 int decode_box_rows() { return DTOK; }
 
@@ -883,7 +1008,10 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
+  // batch plan: a.budget + B CTAs per KV head cover every split (sum_b n_b <=
+  // T / cps + B <= budget + B); per-request plans: num_splits per request
+  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)a.Hkv, 1u)
+                           : dim3((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
   cfg.blockDim = dim3(DWARPS * 32);
   cfg.dynamicSmemBytes = L::TOTAL;
   cfg.stream = stream;
@@ -934,6 +1062,18 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
   a.num_splits = num_splits;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
+  a.B = batch;
+  // Batches of up to BAL_MAX_B requests size their splits for the whole batch
+  // (balanced_plan): about 2 CTAs per SM in all, fewer than B * num_splits
+  // (minus B/2 for rounding) so every split's partial row fits the workspace.
+  a.balanced = (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) ? 1 : 0;
+  a.budget = 1;
+  if (a.balanced) {
+    const int slots = (2 * sm_count() + g.Hkv - 1) / g.Hkv;
+    const int64_t fit = (int64_t)batch * num_splits - batch;
+    const int64_t cap = fit < slots ? fit : slots;
+    a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);
+  }
   if (g.D == 256) return launch_decode_t<256>(tmap, a, batch, stream);
   return launch_decode_t<128>(tmap, a, batch, stream);
 }

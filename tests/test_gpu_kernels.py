@@ -153,6 +153,9 @@ def test_checkpoint_and_restore_bit_exact(Hkv, D, P, ctx):
     (16, 2, 256, 256, [2500], 5, False),           # G = 8
     (12, 2, 128, 128, [999], 64, False),           # more splits than needed
     (8, 2, 128, 256, [70000, 3000], 150, False),   # > 128 live splits: merge loops
+    (8, 2, 128, 64, [20000, 70, 1, 3000], 8, False),   # batch plan: the long request
+                                                       # takes more than num_splits
+    (24, 4, 256, 128, [9000, 0, 40], 3, True),     # batch plan with an empty request
 ])
 def test_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
     case = make_case(200 + Hq + sum(ctx), Hq, Hkv, D, P, ctx, outliers=outliers)
