@@ -154,6 +154,29 @@ int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int3
                          size_t workspace_bytes, int32_t num_splits, void* stream);
 
 /*
+ * Packed multi-query verifier (Sec. 3.1, speculative verification of two to
+ * four proposed tokens at once; App. A.1 dispatch: causal masks, query
+ * lengths 2-4).  Each request b has q_len query tokens at absolute positions
+ * context_lens[b] - q_len + i (i < q_len), already appended to the pool;
+ * token i attends positions [0, context_lens[b] - q_len + i] causally:
+ *   out[b, i, h, :] = sum_t softmax_t(scale * <q[b, i, h], K_t>) V_t.
+ * The page reads are shared by the tokens: the split CTAs of a KV head each
+ * take 8 of its G * q_len (token, head) rows over the same chunk range.
+ *   q, out        bf16 [batch, q_len, Hq, D]
+ *   q_len         1..4 (1 is plain decode)
+ *   context_lens  int32 [batch], >= q_len for every request that has tokens
+ *                 (a shorter context gives each token the positions it has)
+ *   workspace     >= jf_attn_workspace_bytes(batch, q_len * Hq, Hkv, D,
+ *                 num_splits) bytes, 256-byte aligned
+ * Other arguments, limits, numerics and errors as for jf_paged_decode_attn.
+ */
+int jf_paged_verify_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                         const int32_t* context_lens, int32_t batch, const void* q,
+                         int32_t q_len, int32_t num_q_heads, float softmax_scale, void* out,
+                         void* workspace, size_t workspace_bytes, int32_t num_splits,
+                         void* stream);
+
+/*
  * Append-then-attend decode step in one launch pair (Sec. 3.3: the step's
  * pending cache write lands before its attention reads the pool; Sec. 3.1
  * decode).  For every request b with context_lens[b] >= 1 the bf16 vectors

@@ -7,6 +7,6 @@ from .binding import (  # noqa: F401
     KVPool, JfError, decode_workspace, default_num_splits, jf_attn_workspace_bytes,
     jf_kv_checkpoint, jf_kv_page_bytes, jf_kv_quantize_append, jf_kv_restore,
     jf_paged_decode_append_attn, jf_paged_decode_attn, jf_paged_decode_attn_noalloc,
-    jf_prefill_chunk_attn, jf_prefill_workspace_bytes, lib, status_string, version,
-    workspace_status,
+    jf_paged_verify_attn, jf_prefill_chunk_attn, jf_prefill_workspace_bytes, lib,
+    status_string, version, verify_workspace, default_verify_splits, workspace_status,
 )

@@ -31,7 +31,7 @@ EXPORTS = [
     "jf_kv_page_bytes", "jf_attn_workspace_bytes", "jf_prefill_workspace_bytes",
     "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
-    "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn",
+    "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -77,6 +77,8 @@ def lib() -> ctypes.CDLL:
                                                             I32, P, P]),
             "jf_paged_decode_append_attn": (ctypes.c_int, [PP, P, I32, P, I32, P, P, P, I32, F32,
                                                            P, P, SZ, I32, P]),
+            "jf_paged_verify_attn": (ctypes.c_int, [PP, P, I32, P, I32, P, I32, I32, F32, P, P,
+                                                    SZ, I32, P]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -241,6 +243,41 @@ def jf_paged_decode_append_attn(pool: KVPool, page_table: torch.Tensor,
                                             float(softmax_scale), _ptr(out), _ptr(workspace),
                                             workspace.numel(), int(num_splits), _stream(stream))
     _check("jf_paged_decode_append_attn", st)
+
+
+def jf_paged_verify_attn(pool: KVPool, page_table: torch.Tensor, context_lens: torch.Tensor,
+                         q: torch.Tensor, softmax_scale: float, out: torch.Tensor,
+                         workspace: torch.Tensor, num_splits: int, stream=None) -> None:
+    """Packed verifier: q, out are [batch, q_len, Hq, D]; token i of request b
+    sees positions up to context_lens[b] - q_len + i."""
+    _need(page_table, torch.int32, "page_table")
+    _need(context_lens, torch.int32, "context_lens")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    _need(workspace, torch.uint8, "workspace")
+    B, L, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim or page_table.shape[0] != B or context_lens.numel() != B:
+        raise ValueError("shape mismatch")
+    st = lib().jf_paged_verify_attn(ctypes.byref(pool.c_struct()), _ptr(page_table),
+                                     page_table.shape[1], _ptr(context_lens), B, _ptr(q), L, Hq,
+                                     float(softmax_scale), _ptr(out), _ptr(workspace),
+                                     workspace.numel(), int(num_splits), _stream(stream))
+    _check("jf_paged_verify_attn", st)
+
+
+def verify_workspace(batch, q_len, num_q_heads, num_kv_heads, head_dim, num_splits, device="cuda"):
+    return decode_workspace(batch, q_len * num_q_heads, num_kv_heads, head_dim, num_splits,
+                            device=device)
+
+
+def default_verify_splits(batch: int, q_len: int, num_q_heads: int, num_kv_heads: int,
+                          device=None) -> int:
+    """Split cap for the verifier: each split of a KV head runs
+    ceil(G * q_len / 8) CTAs, so fewer splits fill the GPU."""
+    nt = -(-(num_q_heads // num_kv_heads) * q_len // 8)
+    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
+    per = (2 * props.multi_processor_count) // (batch * num_kv_heads * nt)   # one full wave
+    return max(1, per if batch == 1 else per + 2)
 
 
 def jf_paged_decode_attn_noalloc(pool: KVPool, page_table: torch.Tensor,

@@ -14,7 +14,8 @@ int launch_page_copy(const Geom&, const jf_kv_pool&, const int32_t*, int32_t, vo
                      bool, cudaStream_t);
 int launch_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*, int32_t,
                   const int32_t*, int32_t, const void*, int32_t, float, void*, void*, int32_t,
-                  cudaStream_t, const void* k_new = nullptr, const void* v_new = nullptr);
+                  cudaStream_t, const void* k_new = nullptr, const void* v_new = nullptr,
+                  int32_t q_len = 1);
 size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S);
 int decode_box_rows();
 int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
@@ -121,7 +122,7 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
                          const int32_t* context_lens, int32_t batch, const void* k_new,
                          const void* v_new, const void* q, int32_t num_q_heads,
                          float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
-                         int32_t num_splits, void* stream) {
+                         int32_t num_splits, void* stream, int32_t q_len = 1) {
   int st = check_pool(pool);
   if (st) return st;
   if (!page_table || !context_lens || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
@@ -129,10 +130,11 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
   if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
   if (num_q_heads / pool->num_kv_heads > 8) return JF_ERR_UNSUPPORTED;
   if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
+  if (q_len < 1 || q_len > 4) return JF_ERR_INVALID_ARG;
   if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
   if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return JF_ERR_INVALID_ARG;
   if (k_new && (!aligned(k_new, 16) || !aligned(v_new, 16))) return JF_ERR_INVALID_ARG;
-  const size_t need = jf_attn_workspace_bytes(batch, num_q_heads, pool->num_kv_heads,
+  const size_t need = jf_attn_workspace_bytes(batch, q_len * num_q_heads, pool->num_kv_heads,
                                               pool->head_dim, num_splits);
   if (workspace_bytes < need) return JF_ERR_WORKSPACE_TOO_SMALL;
   const Geom g = make_geom(*pool);
@@ -141,7 +143,7 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
   if (st) return st;
   return launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q,
                        num_q_heads, softmax_scale, out, workspace, num_splits,
-                       static_cast<cudaStream_t>(stream), k_new, v_new);
+                       static_cast<cudaStream_t>(stream), k_new, v_new, q_len);
 }
 
 int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
@@ -151,6 +153,17 @@ int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int3
   return decode_common(pool, page_table, pt_stride, context_lens, batch, nullptr, nullptr, q,
                        num_q_heads, softmax_scale, out, workspace, workspace_bytes, num_splits,
                        stream);
+}
+
+int jf_paged_verify_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                         const int32_t* context_lens, int32_t batch, const void* q,
+                         int32_t q_len, int32_t num_q_heads, float softmax_scale, void* out,
+                         void* workspace, size_t workspace_bytes, int32_t num_splits,
+                         void* stream) {
+  if (q_len < 1 || q_len > 4) return JF_ERR_INVALID_ARG;
+  return decode_common(pool, page_table, pt_stride, context_lens, batch, nullptr, nullptr, q,
+                       num_q_heads, softmax_scale, out, workspace, workspace_bytes, num_splits,
+                       stream, q_len);
 }
 
 int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_table,

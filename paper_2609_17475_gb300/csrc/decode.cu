@@ -68,6 +68,9 @@ struct DecodeArgs {
   int32_t num_splits;
   float scale_log2;    // softmax_scale * log2(e)
   int32_t B;           // requests
+  int32_t L;           // query tokens per request (1: decode; 2-4: packed verifier)
+  int32_t NT;          // CTAs per KV head, each for 8 of its G * L (token, head) rows
+  int32_t HqL;         // L * Hq: rows of q, out and the partials per request
   int32_t balanced;    // 1: batch split plan (balanced_plan), partial rows by global split
   int32_t budget;      // balanced: target splits per KV head over the whole batch
 };
@@ -260,12 +263,16 @@ __device__ __forceinline__ void load_sb_words(const uint8_t* p, uint32_t (&w)[NG
 }
 
 // One 32-position chunk (two 16-position MMA tiles).  FULL: every position is
-// valid, so no masking work is done; otherwise positions >= nvalid are masked
-// (their logits become -inf and their scale/bias words are never used, so
-// whatever bytes sit in unused slots cannot leak into the result).
+// valid and visible to every row, so no masking work is done; otherwise
+// positions >= nvalid hold no data (their logits become -inf and their
+// scale/bias words are never used, so whatever bytes sit in unused slots
+// cannot leak into the result), and the rows of this thread's columns 2c and
+// 2c+1 see only positions < nv0 and < nv1 (causal limits of the verifier's
+// query tokens; both are nvalid for a single query).
 template <int D, bool FULL>
 __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const ChunkCtx<D / 64>& cc,
-                                              uint32_t kc, const uint8_t* ksb, int nvalid) {
+                                              uint32_t kc, const uint8_t* ksb, int nvalid,
+                                              int nv0, int nv1) {
   constexpr int NG = D / 64;
   constexpr int CB = D / 2;
   constexpr int SBB = 4 * NG;
@@ -320,8 +327,10 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
 #pragma unroll
     for (int i = 0; i < 4; ++i) sc[j][i] = fmaf(t1[i], cc.cA, t2[i] * cc.cB);
     if constexpr (!FULL) {
-      if (ta >= nvalid) sc[j][0] = sc[j][1] = NEG_INF;
-      if (tb >= nvalid) sc[j][2] = sc[j][3] = NEG_INF;
+      if (ta >= nv0) sc[j][0] = NEG_INF;
+      if (ta >= nv1) sc[j][1] = NEG_INF;
+      if (tb >= nv0) sc[j][2] = NEG_INF;
+      if (tb >= nv1) sc[j][3] = NEG_INF;
     }
   }
 
@@ -459,9 +468,10 @@ __device__ __forceinline__ void append_new_row(const DecodeArgs& a, int b, int k
                      bh);
 }
 
-template <int D>
+template <int D, bool VER>
 __global__ void __launch_bounds__(DWARPS * 32, 2)
 decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
+  // VER: packed verifier (a.L > 1, per-row causal limits); otherwise decode
   using L = DecodeSmem<D>;
   constexpr int NG = L::NG;
   constexpr int SBB = L::SBB;
@@ -473,7 +483,21 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   uint4* qsm = reinterpret_cast<uint4*>(sbuf + L::SB_BYTES);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES + L::QF_BYTES);
 
-  const int kvh = blockIdx.y;
+  // decode: one CTA per KV head holds its G query heads; verifier: NT CTAs
+  // each hold 8 of its G * L (token, head) rows
+  const int kvh = VER ? (int)blockIdx.y / a.NT : (int)blockIdx.y;
+  const int nt = VER ? (int)blockIdx.y % a.NT : 0;
+  const int rows = VER ? min(8, a.G * a.L - 8 * nt) : a.G;
+  // row k of this CTA: query token i = (8 nt + k) / G, head h = (8 nt + k) % G;
+  // its q, out and partial row within the request is i * Hq + kvh * G + h
+  auto row_of = [&](int k) {
+    if constexpr (VER) {
+      const int gr = 8 * nt + k;
+      return (gr / a.G) * a.Hq + kvh * a.G + gr % a.G;
+    } else {
+      return kvh * a.G + k;
+    }
+  };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
   const bool direct = (a.num_splits == 1);
@@ -492,8 +516,6 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
   int split, b, ctx, nch, cps, nsplit;
-  int64_t prow;   // partial row of this split for query head hq: prow + hq * pstride
-  int pstride;
   if (a.balanced) {
     if (warp == 0) {
       const BalPlan p = balanced_plan(a, (int)blockIdx.x, -1, lane);
@@ -512,20 +534,16 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     if (b < 0) return;   // past the batch's last split
     ctx = checked_ctx(a, b);
     nch = (ctx + DTOK - 1) / DTOK;
-    prow = (int64_t)((int)blockIdx.x) * a.Hq;   // global split x = g0 + split
-    pstride = 1;
   } else {
     split = blockIdx.x;
     b = blockIdx.z;
     ctx = checked_ctx(a, b);
     split_plan(ctx, a.num_splits, nch, cps, nsplit);
-    prow = (int64_t)b * a.Hq * a.num_splits + split;
-    pstride = a.num_splits;
   }
   if (split >= nsplit) {
     if (direct && split == 0) {   // empty context: zero output
-      for (int i = threadIdx.x; i < a.G * D; i += blockDim.x)
-        a.out[((int64_t)b * a.Hq + kvh * a.G + i / D) * D + i % D] = 0;
+      for (int i = threadIdx.x; i < rows * D; i += blockDim.x)
+        a.out[((int64_t)b * a.HqL + row_of(i / D)) * D + i % D] = 0;
     }
     return;
   }
@@ -549,9 +567,8 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   __syncwarp();
 
   // ---- query fragments (B operand of QK^T) ---------------------------------
-  const int hq0 = kvh * a.G;
-  const bool head_ok = r < a.G;
-  const uint16_t* qrow = a.q + ((int64_t)b * a.Hq + hq0 + (head_ok ? r : 0)) * D;
+  const bool head_ok = r < rows;
+  const uint16_t* qrow = a.q + ((int64_t)b * a.HqL + row_of(head_ok ? r : 0)) * D;
   uint4 qlo[NG], qhi[NG];
   float qmax = 0.f;
 #pragma unroll
@@ -692,6 +709,14 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
 #pragma unroll
   for (int g = 0; g < NG; ++g) cc.koff[g] = swz<L::CB>(ld_t, 2 * g + ld_ch);
 
+  // verifier causal limits: query token i of L sees positions < ctx - L + 1 + i;
+  // a chunk below ctx_all is visible to every row (decode: ctx_all = ctx)
+  int ctx_all = ctx, lim0 = ctx, lim1 = ctx;
+  if constexpr (VER) {
+    ctx_all = ctx - a.L + 1;
+    lim0 = min(ctx, ctx_all + (8 * nt + 2 * c) / a.G);
+    lim1 = min(ctx, ctx_all + (8 * nt + 2 * c + 1) / a.G);
+  }
   int done = 0;
   // unrolled by the ring depth, so every stage address is a constant offset
 #pragma unroll DSTAGES
@@ -707,10 +732,15 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     const int tokbase = chunk_of(it) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF);
     const uint8_t* ksb = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
-    if (ok && tokbase + DTOK <= ctx)
-      process_chunk<D, true>(st, cc, kc, ksb, 0);
-    else
-      process_chunk<D, false>(st, cc, kc, ksb, ok ? ctx - tokbase : 0);
+    if (ok && tokbase + DTOK <= (VER ? ctx_all : ctx)) {
+      process_chunk<D, true>(st, cc, kc, ksb, 0, 0, 0);
+    } else if constexpr (VER) {
+      process_chunk<D, false>(st, cc, kc, ksb, ok ? ctx - tokbase : 0,
+                              ok ? lim0 - tokbase : 0, ok ? lim1 - tokbase : 0);
+    } else {
+      const int nv = ok ? ctx - tokbase : 0;
+      process_chunk<D, false>(st, cc, kc, ksb, nv, nv, nv);
+    }
 
     __syncwarp();
     if (it + DSTAGES < my_n) {
@@ -783,7 +813,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   // ---- combine the warps of this CTA --------------------------------------
   // per head: M = max_w m_w, weights 2^(m_w - M) (divided by L when this CTA
   // writes the final output), L = sum_w 2^(m_w - M) l_w
-  if (threadIdx.x < a.G) {
+  if (threadIdx.x < rows) {
     const int h = threadIdx.x;
     float M = NEG_INF;
 #pragma unroll
@@ -803,7 +833,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     shl[h * 2 + 1] = L;
   }
   __syncthreads();
-  for (int idx = threadIdx.x; idx < a.G * (D / 4); idx += blockDim.x) {
+  for (int idx = threadIdx.x; idx < rows * (D / 4); idx += blockDim.x) {
     const int h = idx / (D / 4), d = 4 * (idx % (D / 4));
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -817,16 +847,20 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
         acc.w = fmaf(f, v.w, acc.w);
       }
     }
-    const int hq = hq0 + h;
+    const int fr = row_of(h);
     if (direct) {
       uint2 o;
       o.x = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.x)) |
             ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.y)) << 16);
       o.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.z)) |
             ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.w)) << 16);
-      *reinterpret_cast<uint2*>(a.out + ((int64_t)b * a.Hq + hq) * D + d) = o;
+      *reinterpret_cast<uint2*>(a.out + ((int64_t)blockIdx.z * a.HqL + fr) * D + d) = o;
     } else {
-      const int64_t row = prow + (int64_t)hq * pstride;
+      // partial row: global split x (batch plan) or (b, split) per request
+      // without the batch plan (b, split) = (blockIdx.z, blockIdx.x)
+      const int64_t row = a.balanced
+          ? (int64_t)blockIdx.x * a.HqL + fr
+          : ((int64_t)blockIdx.z * a.HqL + fr) * a.num_splits + blockIdx.x;
       *reinterpret_cast<float4*>(a.part_o + row * D + d) = acc;
       if (d == 0) {
         a.part_ml[row * 2 + 0] = shl[h * 2 + 0];
@@ -867,7 +901,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   // (row (g0 + s) Hq + hq) and is worked out first.
   __shared__ int plan_sh[2];
   int S = a.num_splits;
-  int64_t row0 = ((int64_t)b * a.Hq + hq) * S;
+  int64_t row0 = ((int64_t)b * a.HqL + hq) * S;
   int64_t rs = 1;
   int nsplit_bal = 0;
   if (a.balanced) {
@@ -879,8 +913,8 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
       }
     }
     __syncthreads();
-    row0 = (int64_t)plan_sh[0] * a.Hq + hq;
-    rs = a.Hq;
+    row0 = (int64_t)plan_sh[0] * a.HqL + hq;
+    rs = a.HqL;
     nsplit_bal = plan_sh[1];
     S = nsplit_bal;
   }
@@ -908,7 +942,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   int nch, cps, nsplit;
   split_plan(ctx, a.num_splits, nch, cps, nsplit);
   if (a.balanced) nsplit = nsplit_bal;
-  uint16_t* orow = a.out + ((int64_t)b * a.Hq + hq) * D + d0;
+  uint16_t* orow = a.out + ((int64_t)b * a.HqL + hq) * D + d0;
   if (nsplit == 0) {
     if (t < MERGE_DSLICE) orow[t] = 0;
     return;
@@ -996,7 +1030,9 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   using L = DecodeSmem<D>;
   static bool attr_done = false;
   if (!attr_done) {
-    if (cudaFuncSetAttribute(decode_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(decode_split_kernel<D, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) != cudaSuccess ||
+        cudaFuncSetAttribute(decode_split_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              L::TOTAL) != cudaSuccess)
       return JF_ERR_CUDA;
     attr_done = true;
@@ -1010,17 +1046,19 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   cudaLaunchConfig_t cfg = {};
   // batch plan: a.budget + B CTAs per KV head cover every split (sum_b n_b <=
   // T / cps + B <= budget + B); per-request plans: num_splits per request
-  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)a.Hkv, 1u)
-                           : dim3((unsigned)a.num_splits, (unsigned)a.Hkv, (unsigned)B);
+  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)(a.Hkv * a.NT), 1u)
+                           : dim3((unsigned)a.num_splits, (unsigned)(a.Hkv * a.NT), (unsigned)B);
   cfg.blockDim = dim3(DWARPS * 32);
   cfg.dynamicSmemBytes = L::TOTAL;
   cfg.stream = stream;
   cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, decode_split_kernel<D>, tmap, a) != cudaSuccess) return JF_ERR_CUDA;
+  const cudaError_t e = (a.L > 1) ? cudaLaunchKernelEx(&cfg, decode_split_kernel<D, true>, tmap, a)
+                                  : cudaLaunchKernelEx(&cfg, decode_split_kernel<D, false>, tmap, a);
+  if (e != cudaSuccess) return JF_ERR_CUDA;
   if (a.num_splits > 1) {
     cudaLaunchConfig_t mc = {};
-    mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.Hq, (unsigned)B);
+    mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.HqL, (unsigned)B);
     mc.blockDim = dim3(MERGE_THREADS);
     mc.dynamicSmemBytes = 0;
     mc.stream = stream;
@@ -1035,7 +1073,7 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
                   const int32_t* page_table, int32_t pt_stride, const int32_t* context_lens,
                   int32_t batch, const void* q, int32_t Hq, float softmax_scale, void* out,
                   void* workspace, int32_t num_splits, cudaStream_t stream, const void* k_new,
-                  const void* v_new) {
+                  const void* v_new, int32_t q_len) {
   DecodeArgs a;
   a.pool = static_cast<const uint8_t*>(pool.base);
   a.num_pages = g.num_pages;
@@ -1048,6 +1086,9 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.Hkv = g.Hkv;
   a.Hq = Hq;
   a.G = Hq / g.Hkv;
+  a.L = q_len;
+  a.NT = (a.G * q_len + 7) / 8;
+  a.HqL = q_len * Hq;
   a.page_table = page_table;
   a.pt_stride = pt_stride;
   a.ctx = context_lens;
@@ -1056,7 +1097,7 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.vnew = static_cast<const uint16_t*>(v_new);
   a.out = static_cast<uint16_t*>(out);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  const int64_t rows = (int64_t)batch * Hq * num_splits;
+  const int64_t rows = (int64_t)batch * q_len * Hq * num_splits;
   a.status = reinterpret_cast<int32_t*>(ws);
   a.part_ml = reinterpret_cast<float*>(ws + 256);
   a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
@@ -1069,7 +1110,7 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.balanced = (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) ? 1 : 0;
   a.budget = 1;
   if (a.balanced) {
-    const int slots = (2 * sm_count() + g.Hkv - 1) / g.Hkv;
+    const int slots = (2 * sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
     const int64_t fit = (int64_t)batch * num_splits - batch;
     const int64_t cap = fit < slots ? fit : slots;
     a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);

@@ -231,6 +231,51 @@ def test_fused_append_decode_reports_bad_page_id():
     assert torch.equal(pool.data, before)    # nothing written anywhere
 
 
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,L,splits", [
+    (24, 4, 256, 256, [5000], 2, None),          # 12 (token, head) rows: 2 CTAs per split
+    (24, 4, 256, 128, [3000, 777], 4, None),     # 24 rows, batch plan
+    (24, 4, 256, 256, [4096], 3, 1),             # one split: rows written directly
+    (8, 2, 128, 64, [3, 65, 300, 2001], 3, 5),   # a context equal to q_len, partial pages
+    (16, 2, 256, 64, [1000], 4, 7),              # G = 8: 32 rows
+])
+def test_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
+    """Token i of each request attends positions up to ctx - L + i; the oracle
+    is the causal prefill of those L queries (Sec. 3.1 packed verifier)."""
+    from paper_2609_17475_gb300 import synth
+    case = make_case(500 + sum(ctx) + L, Hq, Hkv, D, P, ctx)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    B = len(ctx)
+    q = synth.normal_bf16(synth.generator(600 + L), (B, L, Hq, D))
+    if splits is None:
+        splits = jf.default_verify_splits(B, L, Hq, Hkv)
+    ws = jf.verify_workspace(B, L, Hq, Hkv, D, splits, device=DEV)
+    ws[256:] = 0xFF
+    out = torch.full((B, L, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    scale = 1 / math.sqrt(D)
+    jf.jf_paged_verify_attn(pool, case.page_table.to(DEV), torch.tensor(ctx, dtype=torch.int32,
+                            device=DEV), q.to(DEV), scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    ref = np.stack([OT.prefill_chunk(ref_pool, case.layout, case.page_table[b].numpy(), bits(q[b]),
+                                     ctx[b] - L, scale) for b in range(B)])
+    assert_attention_close(out, ref)
+
+
+def test_verifier_with_one_token_is_decode():
+    case = make_case(77, 24, 4, 256, 256, [3333, 1234])
+    pool = pool_from_numpy(case, case.oracle_pool())
+    splits = 9
+    out_d = gpu_decode(case, pool, splits)
+    ws = jf.verify_workspace(2, 1, 24, 4, 256, splits, device=DEV)
+    out_v = torch.empty((2, 1, 24, 256), dtype=torch.bfloat16, device=DEV)
+    jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
+                            torch.tensor(case.ctx, dtype=torch.int32, device=DEV),
+                            case.q.view(2, 1, 24, 256).to(DEV), 1 / 16, out_v, ws, splits)
+    torch.cuda.synchronize()
+    assert torch.equal(out_v.view(2, 24, 256), out_d)
+
+
 def test_decode_edge_contexts():
     case = make_case(5, 8, 2, 128, 64, [0, 1, 64, 65])
     ref_pool = case.oracle_pool()
