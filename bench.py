@@ -343,7 +343,7 @@ def _event_time(fn, reps, stream):
     return e0.elapsed_time(e1) / reps
 
 
-ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed")
+ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify")
 
 
 def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
@@ -352,7 +352,50 @@ def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
     allocated on `stream`, the stream the kernels run on, so the caching allocator
     never hands a buffer back out while a kernel still reads it."""
     with torch.cuda.stream(stream):
-        return _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only)
+        out = _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only)
+        if only is None or only == "verify":
+            out["verify_256k"] = _bench_verify(jf, dev, stream)
+        return out
+
+
+def _bench_verify(jf, dev, stream):
+    """Packed verifier on one 262,144-position request (24/4/256, page 256):
+    q_len 2-4 tokens in one call against q_len separate decode calls."""
+    Hq, Hkv, D, P, ctx = 24, 4, 256, 256, 262144
+    g = torch.Generator(device=dev)
+    g.manual_seed(99)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    pt = torch.randperm(ctx // P, device=dev, generator=g).to(torch.int32).view(1, -1)
+    pool = jf.KVPool.allocate(ctx // P, P, Hkv, D, device=dev, fill=None)
+    for s0 in range(0, ctx, 65536):
+        kk = torch.randn(65536, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vv = torch.randn(65536, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        jf.jf_kv_quantize_append(pool, pt, torch.zeros(65536, dtype=torch.int32, device=dev),
+                                 torch.arange(s0, s0 + 65536, dtype=torch.int32, device=dev),
+                                 kk, vv, err, stream=stream)
+    c = torch.tensor([ctx], dtype=torch.int32, device=dev)
+    bpp = 2 * Hkv * (D // 2 + 4 * D // 64)
+    q1 = torch.randn(1, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o1 = torch.empty_like(q1)
+    s1 = jf.default_num_splits(1, Hkv)
+    w1 = jf.decode_workspace(1, Hq, Hkv, D, s1, device=dev)
+    t1 = _event_time(lambda: jf.jf_paged_decode_attn(pool, pt, c, q1, 1 / 16, o1, w1, s1,
+                                                     stream=stream), 20, stream)
+    res = {"decode_us": t1 * 1e3}
+    for L in (2, 3, 4):
+        qv = torch.randn(1, L, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        ov = torch.empty_like(qv)
+        sv = jf.default_verify_splits(1, L, Hq, Hkv)
+        wv = jf.verify_workspace(1, L, Hq, Hkv, D, sv, device=dev)
+        tv = _event_time(lambda: jf.jf_paged_verify_attn(pool, pt, c, qv, 1 / 16, ov, wv, sv,
+                                                         stream=stream), 20, stream)
+        stream.synchronize()
+        assert jf.workspace_status(wv) == 0 and int(err.item()) == 0
+        res[f"q_len_{L}"] = {"us": tv * 1e3, "splits": sv,
+                             "GBps_kv_once": ctx * bpp / (tv / 1e3) / 1e9,
+                             "speedup_vs_separate_decodes": L * t1 / tv}
+    del pool
+    return res
 
 
 def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
