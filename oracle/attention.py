@@ -1,5 +1,8 @@
 """Attention over the paged 4-bit KV pool, in fp64 (test infrastructure).
 
+Every function reads the pool through ``gather_head``, so it serves both KV
+formats: affine 4-bit group-64 and TQ4 (Sec. 3.1 Eq. 4).
+
 Only tests, smoke() and the bench CPU baseline use this module.
 
 * ``paged_decode`` is the plain definition of single-query attention read from
@@ -25,7 +28,16 @@ from __future__ import annotations
 
 import numpy as np
 
-from .affine4 import KIND_K, KIND_V, PoolLayout, bf16_to_f64, gather_head
+from . import affine4, tq4
+from .affine4 import KIND_K, KIND_V, bf16_to_f64
+
+
+def gather_head(pool, layout, page_table_row, ctx, head, kind):
+    """Reconstructed K or V of one KV head, fp64 [ctx, D], for either format:
+    an affine ``PoolLayout`` or a TQ4 ``Tq4Layout`` (which carries its codec)."""
+    if isinstance(layout, tq4.Tq4Layout):
+        return tq4.gather_head(pool, layout, page_table_row, ctx, head, kind)
+    return affine4.gather_head(pool, layout, page_table_row, ctx, head, kind)
 
 
 def _softmax_weighted(s: np.ndarray, v: np.ndarray) -> np.ndarray:
@@ -35,7 +47,7 @@ def _softmax_weighted(s: np.ndarray, v: np.ndarray) -> np.ndarray:
     return (p @ v) / p.sum(axis=-1, keepdims=True)
 
 
-def paged_decode(pool: np.ndarray, layout: PoolLayout, page_table: np.ndarray,
+def paged_decode(pool: np.ndarray, layout, page_table: np.ndarray,
                  context_lens, q_bits: np.ndarray, softmax_scale: float,
                  heads=None) -> np.ndarray:
     """Single-query paged decode attention.
@@ -86,7 +98,7 @@ def merge_partials(parts) -> np.ndarray:
     return num / den
 
 
-def paged_decode_split(pool: np.ndarray, layout: PoolLayout, page_table: np.ndarray,
+def paged_decode_split(pool: np.ndarray, layout, page_table: np.ndarray,
                        context_lens, q_bits: np.ndarray, softmax_scale: float,
                        num_splits: int) -> np.ndarray:
     """The same result as ``paged_decode`` through split partials + merge."""
@@ -107,7 +119,7 @@ def paged_decode_split(pool: np.ndarray, layout: PoolLayout, page_table: np.ndar
     return out
 
 
-def prefill_chunk(pool: np.ndarray, layout: PoolLayout, page_table_row: np.ndarray,
+def prefill_chunk(pool: np.ndarray, layout, page_table_row: np.ndarray,
                   q_bits: np.ndarray, q_start: int, softmax_scale: float,
                   causal: bool = True) -> np.ndarray:
     """Chunk attention.  q_bits [C, Hq, D] at absolute positions q_start + i.

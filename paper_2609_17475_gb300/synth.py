@@ -15,6 +15,8 @@ model; no dataset or weights are needed for the KV path):
 * Queries are drawn the same way, N(0, 1) bf16.
 * Physical page ids are a seeded random permutation of the pool, so logical
   token order never matches physical order.
+* The TQ4 random-sign vectors are NumPy draws (``tq4_signs``); both the
+  oracle and the CUDA path take them as inputs.
 
 The head geometry follows the paper's evaluated model (Sec. 2; App. A.1):
 24 query heads, 4 KV heads, head_dim 256, 256-position pages.
@@ -24,6 +26,7 @@ from __future__ import annotations
 import dataclasses
 from typing import List, Optional, Sequence
 
+import numpy as np
 import torch
 
 
@@ -133,6 +136,17 @@ def append_rows_for(context_lens: Sequence[int]):
     if not req:
         return torch.zeros(0, dtype=torch.int32), torch.zeros(0, dtype=torch.int32)
     return torch.cat(req), torch.cat(pos)
+
+
+def tq4_signs(seed: int, head_dim: int) -> np.ndarray:
+    """The random-sign diagonal S of the TQ4 rotation (App. A.1 Table 3):
+    NumPy ``default_rng(seed + d * 7919)`` drawing one of (-1, +1) per
+    coordinate, int8 [d].  K uses seed 0 and V seed 1 by default."""
+    rng = np.random.default_rng(int(seed) + int(head_dim) * 7919)
+    return rng.choice(np.array([-1, 1], dtype=np.int8), size=int(head_dim))
+
+
+TQ4_SEED_K, TQ4_SEED_V = 0, 1
 
 
 def context_lengths(gen: torch.Generator, batch: int, lo: int, hi: int) -> List[int]:

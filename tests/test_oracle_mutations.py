@@ -129,3 +129,74 @@ def test_unmutated_pins_pass():
     TQ.test_golden_packing()
     TA.test_decode_matches_sdpa_on_exact_values(8, 2, 128, 64, [300, 64, 1])
     TA.test_prefill_rows_equal_decode_and_sdpa(100, 70)
+
+
+# -- TQ4 (Sec. 3.1 Eq. 4; App. A.1 Table 3) -----------------------------------
+import oracle.tq4 as Q
+from tests import test_oracle_tq4 as TT
+
+
+def test_tq4_dropped_signs_are_caught(monkeypatch):
+    orig = Q.encode
+
+    def bad(x_bits, codec, kind):
+        ones = np.ones(codec.head_dim)
+        return orig(x_bits, Q.Codec(codec.head_dim, codec.centroids, ones, ones), kind)
+    monkeypatch.setattr(Q, "encode", bad)
+    assert _fails(TT.test_one_hot_vectors_get_the_gaussian_lloyd_max_indices)
+
+
+def test_tq4_wrong_density_exponent_is_caught(monkeypatch):
+    def bad(d):
+        x = np.linspace(-1.0 + Q.GRID_EPS, 1.0 - Q.GRID_EPS, Q.GRID_POINTS)
+        w = (1.0 - x * x) ** ((d - 1) / 2.0)
+        return x, w / w.sum()
+    monkeypatch.setattr(Q, "grid_and_weights", bad)
+    assert _fails(TT.test_lloyd_update_matches_the_continuous_conditional_means, 256)
+
+
+def test_tq4_unweighted_cell_means_are_caught(monkeypatch):
+    orig = Q.lloyd_update
+
+    def bad(x, w, c):
+        return orig(x, np.full_like(w, 1.0 / len(w)), c)
+    monkeypatch.setattr(Q, "lloyd_update", bad)
+    assert _fails(TT.test_lloyd_update_matches_the_continuous_conditional_means, 256)
+
+
+def test_tq4_thresholds_at_centroids_are_caught(monkeypatch):
+    monkeypatch.setattr(Q, "thresholds", lambda c32: np.asarray(c32, dtype=np.float32)[1:])
+    assert _fails(TT.test_indices_are_nearest_centroids)
+
+
+def test_tq4_missing_sqrt_d_in_decode_is_caught(monkeypatch):
+    orig = Q.decode
+
+    def bad(z, nb, codec, kind):
+        return orig(z, nb, codec, kind) * np.sqrt(codec.head_dim)
+    monkeypatch.setattr(Q, "decode", bad)
+    assert _fails(TT.test_round_trip_error_matches_the_codebook_distortion)
+
+
+def test_tq4_rotation_order_swapped_in_decode_is_caught(monkeypatch):
+    def bad(z, nb, codec, kind):
+        d = codec.head_dim
+        cz = codec.centroids.astype(np.float64)[np.asarray(z, dtype=np.int64)]
+        rot = (cz * codec.signs(kind)) @ Q.hadamard(d).T          # H S c instead of S H c
+        return Q.fp16_to_f64(nb)[..., None] * rot / np.sqrt(np.float64(d))
+    monkeypatch.setattr(Q, "decode", bad)
+    assert _fails(TT.test_round_trip_error_matches_the_codebook_distortion)
+
+
+def test_tq4_bf16_norm_is_caught(monkeypatch):
+    monkeypatch.setattr(Q, "norm_to_fp16",
+                        lambda rho: A.f32_to_bf16(np.asarray(rho, dtype=np.float32)))
+    assert _fails(TT.test_one_hot_vectors_get_the_gaussian_lloyd_max_indices)
+
+
+def test_tq4_quantile_offset_is_caught(monkeypatch):
+    def bad(x, w):
+        cdf = np.cumsum(w)
+        return np.array([x[np.searchsorted(cdf, k / 16.0)] for k in range(16)])
+    monkeypatch.setattr(Q, "quantile_init", bad)
+    assert _fails(TT.test_quantile_start_is_the_beta_quantile, 256)
