@@ -343,7 +343,7 @@ def _event_time(fn, reps, stream):
     return e0.elapsed_time(e1) / reps
 
 
-ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify")
+ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify", "tq4")
 
 
 def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
@@ -355,7 +355,68 @@ def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
         out = _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only)
         if only is None or only == "verify":
             out["verify_256k"] = _bench_verify(jf, dev, stream)
+        if only is None or only == "tq4":
+            out["tq4_256k"] = _bench_tq4(jf, synth, dev, stream, peaks_gbs)
         return out
+
+
+def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
+    """TQ4 format (Sec. 3.1 Eq. 4) on the 256K full-window shape (24/4/256,
+    page 256, random physical pages, 4 K channels per KV head x20): encode on
+    append of a 2,048-row chunk, and single-query decode over `copies`
+    independent caches taken in turn (2.2 GB in all, so no call finds the
+    previous one's pages in L2)."""
+    Hq, Hkv, D, P, ctx = 24, 4, 256, 256, 262144
+    g = torch.Generator(device=dev)
+    g.manual_seed(777)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    codec = jf.Tq4Codec(D, synth.tq4_signs(synth.TQ4_SEED_K, D), synth.tq4_signs(synth.TQ4_SEED_V, D))
+    ch = torch.randperm(D, device=dev, generator=g)[:4]
+    pools, tables = [], []
+    for _ in range(copies):
+        pt = torch.randperm(ctx // P, device=dev, generator=g).to(torch.int32).view(1, -1)
+        pool = jf.KVPool.allocate(ctx // P, P, Hkv, D, device=dev, fill=None,
+                                  format=jf.JF_FMT_TQ4, codec=codec)
+        for s0 in range(0, ctx, 65536):
+            kk = torch.randn(65536, Hkv, D, generator=g, device=dev)
+            kk[:, :, ch] *= 20.0
+            vv = torch.randn(65536, Hkv, D, generator=g, device=dev)
+            jf.jf_kv_quantize_append(pool, pt, torch.zeros(65536, dtype=torch.int32, device=dev),
+                                     torch.arange(s0, s0 + 65536, dtype=torch.int32, device=dev),
+                                     kk.to(torch.bfloat16), vv.to(torch.bfloat16), err,
+                                     stream=stream)
+        pools.append(pool)
+        tables.append(pt)
+    c = torch.tensor([ctx], dtype=torch.int32, device=dev)
+    q = torch.randn(1, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o = torch.empty_like(q)
+    splits = jf.default_num_splits(1, Hkv, format=jf.JF_FMT_TQ4)
+    ws = jf.decode_workspace(1, Hq, Hkv, D, splits, device=dev)
+    it = [0]
+
+    def call():
+        i = it[0] % copies
+        it[0] += 1
+        jf.jf_paged_decode_attn(pools[i], tables[i], c, q, 1 / 16, o, ws, splits, stream=stream)
+    t = _event_time(call, 8 * copies, stream)
+    # encode on append: one 2,048-row chunk (8,192 vectors) into the first cache
+    kk = torch.randn(2048, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    vv = torch.randn(2048, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+    rr = torch.zeros(2048, dtype=torch.int32, device=dev)
+    pp = torch.arange(0, 2048, dtype=torch.int32, device=dev)
+    ta = _event_time(lambda: jf.jf_kv_quantize_append(pools[0], tables[0], rr, pp, kk, vv, err,
+                                                      stream=stream), 20, stream)
+    stream.synchronize()
+    assert jf.workspace_status(ws) == 0 and int(err.item()) == 0
+    bpp = 2 * Hkv * (D // 2 + 2)
+    alg = ctx * bpp + 2 * Hq * D * 2 + (ctx // P) * 4
+    gbs = alg / (t / 1e3) / 1e9
+    res = {"decode_us": t * 1e3, "positions_per_s": ctx / (t / 1e3), "GBps": gbs,
+           "frac_of_measured": gbs / peaks_gbs, "splits": splits, "bytes_per_position": bpp,
+           "alg_bytes_per_call": alg, "append_2048_rows_us": ta * 1e3,
+           "append_GBps": (2048 * Hkv * D * 2 * 2 + 2048 * bpp) / (ta / 1e3) / 1e9}
+    del pools
+    return res
 
 
 def _bench_verify(jf, dev, stream):

@@ -22,9 +22,9 @@
  *     after the stream completes.
  *   - bf16 means IEEE bfloat16 bit patterns (uint16), row-major, contiguous.
  *
- * KV pool format (JF_FMT_AFFINE4_G64; the paper defines TQ4 for KV and only
+ * KV pool formats.  JF_FMT_AFFINE4_G64 (the paper defines TQ4 for KV and only
  * mentions affine Q4 groups for weights, so the affine group layout below is
- * this library's reading):
+ * this library's reading) and JF_FMT_TQ4 (documented with jf_tq4_codec):
  *   page record = [K codes: Hkv x P x D/2 bytes][V codes: same]
  *                 [K scale/bias: Hkv x P x D/64 x (bf16 scale, bf16 bias)]
  *                 [V scale/bias: same]
@@ -59,8 +59,33 @@ extern "C" {
 #define JF_DEV_ERR_TIMEOUT    4   /* a bounded wait on a copy gave up      */
 
 /* ---- formats -------------------------------------------------------- */
-#define JF_FMT_AFFINE4_G64 0      /* implemented                            */
-#define JF_FMT_TQ4         1      /* reserved (Eq. 4 codec); unsupported    */
+#define JF_FMT_AFFINE4_G64 0      /* affine 4-bit, 64-element groups (above) */
+#define JF_FMT_TQ4         1      /* TQ4 (Sec. 3.1 Eq. 4), see below         */
+
+/*
+ * TQ4 format (Sec. 3.1 Eq. 4; App. A.1 Table 3).  A vector x of D elements is
+ * stored as D 4-bit indices z into 16 shared centroids c and one fp16 norm:
+ *   rho   = fp32 rounding of ||x||_2 (from the fp64 sum of squares),
+ *   u     = H_D S x   (H_D the unnormalized Sylvester Hadamard matrix,
+ *                      H[i][j] = (-1)^popcount(i & j); S = diag(signs)),
+ *   z_j   = #{k in 0..14 : u_j > fp64(fp64(sqrt(D) rho) t_k)},
+ *           t_k = fp32(fp32(c_k + c_{k+1}) * 0.5)   (midpoints, strict >),
+ *   norm  = fp16 round-to-nearest of min(rho, 65504),
+ * and reconstructs as x_hat = norm S H_D c[z] / sqrt(D).  Indices are exact
+ * (bit for bit with the reference definition) for bf16 vectors whose
+ * nonzero magnitudes span less than 2^37 and whose norm lies in [1e-30, 1e36].
+ *   page record = [K indices: Hkv x P x D/2 bytes][V indices: same]
+ *                 [K norms: Hkv x P x fp16][V norms: same]
+ *   Index j of a vector is nibble j % 8 of little-endian 32-bit word j / 8
+ *   (element 2i in the low nibble of byte i).  page_bytes = 2*Hkv*P*(D/2 + 2):
+ *   1,040 bytes per position per layer at Hkv 4, D 256, i.e. Eq. 2's 16,640
+ *   bytes over 16 layers.
+ */
+typedef struct jf_tq4_codec {
+  float  centroids[16];   /* strictly ascending, |c| < 1 (jf_tq4_codebook)  */
+  int8_t signs_k[256];    /* diagonal of S for K: +1 or -1, first D used    */
+  int8_t signs_v[256];    /* diagonal of S for V                            */
+} jf_tq4_codec;
 
 typedef struct jf_kv_pool {
   void*   base;          /* device pointer to num_pages page records,
@@ -69,12 +94,31 @@ typedef struct jf_kv_pool {
   int32_t page_size;     /* P: 64, 128 or 256 positions                    */
   int32_t num_kv_heads;  /* Hkv >= 1                                       */
   int32_t head_dim;      /* D: 128 or 256                                  */
-  int32_t group_size;    /* must be 64                                     */
-  int32_t format;        /* JF_FMT_AFFINE4_G64                             */
+  int32_t group_size;    /* 64 (affine format; ignored for TQ4)            */
+  int32_t format;        /* JF_FMT_AFFINE4_G64 or JF_FMT_TQ4               */
+  const jf_tq4_codec* tq4;  /* host pointer, read during each call;
+                               required for JF_FMT_TQ4, else ignored       */
 } jf_kv_pool;
 
-/* Bytes of one page record (0 if the geometry is unsupported). */
+/* Bytes of one affine page record (0 if the geometry is unsupported). */
 size_t jf_kv_page_bytes(int32_t num_kv_heads, int32_t page_size, int32_t head_dim);
+
+/* Bytes of one page record of the given format (0 if unsupported). */
+size_t jf_kv_page_bytes_fmt(int32_t format, int32_t num_kv_heads, int32_t page_size,
+                            int32_t head_dim);
+
+/*
+ * TQ4 codebook for head dimension head_dim (App. A.1 Table 3), on the host:
+ * the 16 fp32 Lloyd-Max centroids of the density (1 - x^2)^((head_dim-3)/2)
+ * on [-1, 1], from a 32,768-point grid over [-1 + 1e-6, 1 - 1e-6], quantile
+ * start (the first grid point whose cumulative weight reaches (k + 1/2)/16),
+ * at most 100 updates (cells by midpoints with strict >, centroid = weighted
+ * cell mean, empty cells kept), stopping after the update whose largest
+ * change is below 1e-6; computed in fp64 and rounded to fp32.
+ *   centroids  host float[16], written in ascending order
+ * Returns JF_ERR_INVALID_ARG for head_dim outside [3, 65536] or a NULL pointer.
+ */
+int jf_tq4_codebook(int32_t head_dim, float* centroids);
 
 /*
  * Workspace bytes jf_paged_decode_attn needs for at most `num_splits`
@@ -109,6 +153,8 @@ size_t jf_prefill_workspace_bytes(void);
  *               rows that were skipped.
  * Rows must not target the same slot twice in one call (the result of such
  * a call is one of the rows, unspecified which).  n_rows == 0 is a no-op.
+ * TQ4 pools: each vector is encoded as the TQ4 format block above states
+ * (indices and norm), with the codec in pool->tq4.
  */
 int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                           int32_t num_requests, const int32_t* row_req, const int32_t* row_pos,
@@ -147,6 +193,13 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
  * so any finite bf16 q is accepted); the softmax runs in fp32 with the
  * maximum subtracted; probabilities scaled by the V group scale enter fp16
  * products, so V group scales must stay below 65504.  Output rounded RNE.
+ * TQ4 pools (pool->tq4 required): the query is rotated once, q' = H S_K q /
+ * sqrt(D), and scaled by a power of two into the fp16 range; indices meet
+ * fp16 centroids in fp16 tensor-core products with fp32 accumulation, scores
+ * are scaled by the K norms, probabilities times V norm times 2^-8 enter
+ * fp16 products, and the accumulated output is rotated back by S_V H / sqrt(D)
+ * in fp32.  The verifier, the fused append and the no-workspace variant
+ * return JF_ERR_UNSUPPORTED for TQ4 pools.
  */
 int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                          const int32_t* context_lens, int32_t batch, const void* q,
@@ -217,7 +270,7 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
 
 /*
  * Page-gather checkpoint (Sec. 3.4: read the request's page runs in place and
- * emit one packed stream).  dst[k * page_bytes .. (k+1) * page_bytes) =
+ * emit one packed stream).  Either format.  dst[k * page_bytes .. (k+1) * page_bytes) =
  * page record page_table_row[k] for k < num_pages, tail bytes included.
  *   dst        device buffer, >= num_pages * page_bytes bytes, 16-byte aligned
  *   err_flag   device int32 or NULL (JF_DEV_ERR_PAGE_ID for bad ids; the
@@ -229,7 +282,7 @@ int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int3
 /*
  * Restore (Sec. 3.4: restoration writes packed runs into the existing pool):
  * the inverse of jf_kv_checkpoint.  Page record page_table_row[k] of the pool
- * = src[k * page_bytes ..).  Page ids must be distinct.
+ * = src[k * page_bytes ..).  Page ids must be distinct.  Either format.
  */
 int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
                   const void* src, size_t src_bytes, int32_t* err_flag, void* stream);

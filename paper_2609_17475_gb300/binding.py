@@ -32,6 +32,7 @@ EXPORTS = [
     "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
     "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
+    "jf_kv_page_bytes_fmt", "jf_tq4_codebook",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -42,11 +43,16 @@ class JfError(RuntimeError):
         super().__init__(f"{fn} failed: {status} ({status_string(status)})")
 
 
+class _Tq4Codec(ctypes.Structure):
+    _fields_ = [("centroids", ctypes.c_float * 16), ("signs_k", ctypes.c_int8 * 256),
+                ("signs_v", ctypes.c_int8 * 256)]
+
+
 class _Pool(ctypes.Structure):
     _fields_ = [("base", ctypes.c_void_p), ("num_pages", ctypes.c_int64),
                 ("page_size", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("group_size", ctypes.c_int32),
-                ("format", ctypes.c_int32)]
+                ("format", ctypes.c_int32), ("tq4", ctypes.POINTER(_Tq4Codec))]
 
 
 _lib = None
@@ -79,6 +85,8 @@ def lib() -> ctypes.CDLL:
                                                            P, P, SZ, I32, P]),
             "jf_paged_verify_attn": (ctypes.c_int, [PP, P, I32, P, I32, P, I32, I32, F32, P, P,
                                                     SZ, I32, P]),
+            "jf_kv_page_bytes_fmt": (SZ, [I32, I32, I32, I32]),
+            "jf_tq4_codebook": (ctypes.c_int, [I32, ctypes.POINTER(ctypes.c_float)]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -118,27 +126,65 @@ def _need(t: torch.Tensor, dtype, name: str) -> None:
         raise TypeError(f"{name} must be a contiguous CUDA tensor of dtype {dtype}")
 
 
+def jf_tq4_codebook(head_dim: int):
+    """The 16 ascending fp32 TQ4 centroids for head_dim (computed by the library)."""
+    import numpy as np
+    buf = (ctypes.c_float * 16)()
+    _check("jf_tq4_codebook", lib().jf_tq4_codebook(int(head_dim), buf))
+    return np.frombuffer(bytes(buf), dtype=np.float32).copy()
+
+
+class Tq4Codec:
+    """TQ4 codec (Sec. 3.1 Eq. 4): the library's centroids for head_dim and the
+    K and V random-sign vectors (+1 / -1, length head_dim), which the caller
+    draws (synth.tq4_signs gives the paper's NumPy draw)."""
+
+    def __init__(self, head_dim: int, signs_k, signs_v):
+        import numpy as np
+        sk = np.asarray(signs_k).astype(np.int64)
+        sv = np.asarray(signs_v).astype(np.int64)
+        if sk.shape != (head_dim,) or sv.shape != (head_dim,):
+            raise ValueError("sign vectors must have head_dim entries")
+        if not (np.isin(sk, (-1, 1)).all() and np.isin(sv, (-1, 1)).all()):
+            raise ValueError("signs must be +1 or -1")
+        self.head_dim = int(head_dim)
+        self.centroids = jf_tq4_codebook(head_dim)
+        self.signs_k, self.signs_v = sk, sv
+        c = _Tq4Codec()
+        for i in range(16):
+            c.centroids[i] = float(self.centroids[i])
+        for j in range(head_dim):
+            c.signs_k[j] = int(sk[j])
+            c.signs_v[j] = int(sv[j])
+        self._c = c
+
+
 @dataclasses.dataclass
 class KVPool:
-    """A paged 4-bit KV pool: ``data`` is a CUDA uint8 tensor [num_pages, page_bytes]."""
+    """A paged 4-bit KV pool: ``data`` is a CUDA uint8 tensor [num_pages, page_bytes].
+    ``codec`` is required for the TQ4 format."""
     data: torch.Tensor
     page_size: int
     num_kv_heads: int
     head_dim: int
     group_size: int = 64
     format: int = JF_FMT_AFFINE4_G64
+    codec: Optional[Tq4Codec] = None
 
     @staticmethod
     def allocate(num_pages: int, page_size: int, num_kv_heads: int, head_dim: int,
-                 device="cuda", fill: Optional[int] = 0) -> "KVPool":
-        pb = jf_kv_page_bytes(num_kv_heads, page_size, head_dim)
+                 device="cuda", fill: Optional[int] = 0, format: int = JF_FMT_AFFINE4_G64,
+                 codec: Optional[Tq4Codec] = None) -> "KVPool":
+        pb = jf_kv_page_bytes_fmt(format, num_kv_heads, page_size, head_dim)
         if pb == 0:
             raise ValueError("unsupported pool geometry")
+        if format == JF_FMT_TQ4 and (codec is None or codec.head_dim != head_dim):
+            raise ValueError("a TQ4 pool needs a codec for its head_dim")
         if fill is None:
             data = torch.empty(num_pages, pb, dtype=torch.uint8, device=device)
         else:
             data = torch.full((num_pages, pb), fill, dtype=torch.uint8, device=device)
-        return KVPool(data, page_size, num_kv_heads, head_dim)
+        return KVPool(data, page_size, num_kv_heads, head_dim, format=format, codec=codec)
 
     @property
     def num_pages(self) -> int:
@@ -149,12 +195,19 @@ class KVPool:
         return self.data.shape[1]
 
     def c_struct(self) -> _Pool:
-        return _Pool(self.data.data_ptr(), self.num_pages, self.page_size, self.num_kv_heads,
-                     self.head_dim, self.group_size, self.format)
+        p = _Pool(self.data.data_ptr(), self.num_pages, self.page_size, self.num_kv_heads,
+                  self.head_dim, self.group_size, self.format)
+        if self.codec is not None:
+            p.tq4 = ctypes.pointer(self.codec._c)
+        return p
 
 
 def jf_kv_page_bytes(num_kv_heads: int, page_size: int, head_dim: int) -> int:
     return int(lib().jf_kv_page_bytes(num_kv_heads, page_size, head_dim))
+
+
+def jf_kv_page_bytes_fmt(format: int, num_kv_heads: int, page_size: int, head_dim: int) -> int:
+    return int(lib().jf_kv_page_bytes_fmt(format, num_kv_heads, page_size, head_dim))
 
 
 def jf_attn_workspace_bytes(batch: int, num_q_heads: int, num_kv_heads: int, head_dim: int,
@@ -347,12 +400,15 @@ def jf_kv_restore(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
     _check("jf_kv_restore", st)
 
 
-def default_num_splits(batch: int, num_kv_heads: int, device=None) -> int:
-    """Split cap per (request, KV head) so the split grid fills the GPU twice
-    over.  A batch plans its splits over all requests together, and its
-    workspace then needs room for about two more splits per request than an
-    even share (rounding up per request)."""
+def default_num_splits(batch: int, num_kv_heads: int, device=None,
+                       format: int = JF_FMT_AFFINE4_G64) -> int:
+    """Split cap per (request, KV head) so the split grid fills every SM slot
+    once (two split CTAs per SM for the affine format, one for TQ4, whose
+    centroid table takes a CTA's spare shared memory).  A batch plans its
+    splits over all requests together, and its workspace then needs room for
+    about two more splits per request than an even share (rounding up per
+    request)."""
     props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    target = 2 * props.multi_processor_count
+    target = (1 if format == JF_FMT_TQ4 else 2) * props.multi_processor_count
     per = -(-target // (batch * num_kv_heads))
     return max(1, per if batch == 1 else per + 2)

@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "tq4.cuh"
 
 namespace jfkv {
 int launch_append(const Geom&, const jf_kv_pool&, const int32_t*, int32_t, int32_t,
@@ -17,6 +18,14 @@ int launch_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int3
                   cudaStream_t, const void* k_new = nullptr, const void* v_new = nullptr,
                   int32_t q_len = 1);
 size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S);
+int tq4_codebook_host(int d, float* out);
+int tq4_make_params(const jf_tq4_codec* codec, int d, Tq4Params* p);
+int launch_tq4_append(const Geom&, const jf_kv_pool&, const Tq4Params&, const int32_t*, int32_t,
+                      int32_t, const int32_t*, const int32_t*, const void*, const void*, int32_t,
+                      int32_t*, cudaStream_t);
+int launch_tq4_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const Tq4Params&,
+                      const int32_t*, int32_t, const int32_t*, int32_t, const void*, int32_t,
+                      float, void*, void*, int32_t, cudaStream_t);
 int decode_box_rows();
 int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
                    const void*, int32_t, int32_t, int32_t, float, int32_t, void*, void*,
@@ -35,6 +44,21 @@ int check_pool(const jf_kv_pool* pool) {
   if (pool->num_pages < 1 || pool->num_kv_heads < 1) return JF_ERR_INVALID_ARG;
   if (pool->format != JF_FMT_AFFINE4_G64) return JF_ERR_UNSUPPORTED;
   if (pool->group_size != 64) return JF_ERR_UNSUPPORTED;
+  if (pool->head_dim != 128 && pool->head_dim != 256) return JF_ERR_UNSUPPORTED;
+  if (pool->page_size != 64 && pool->page_size != 128 && pool->page_size != 256)
+    return JF_ERR_UNSUPPORTED;
+  if (pool->num_kv_heads > 65535) return JF_ERR_UNSUPPORTED;
+  if (pool->num_pages > 0x7FFFFFFFLL) return JF_ERR_UNSUPPORTED;
+  return JF_OK;
+}
+
+// Pools of either format, for the entry points that take both (append,
+// single-query decode, checkpoint, restore).  TQ4 pools need their codec.
+int check_pool_any(const jf_kv_pool* pool) {
+  if (!pool || pool->format != JF_FMT_TQ4) return check_pool(pool);
+  if (!pool->base || !aligned(pool->base, 16)) return JF_ERR_INVALID_ARG;
+  if (pool->num_pages < 1 || pool->num_kv_heads < 1) return JF_ERR_INVALID_ARG;
+  if (!pool->tq4) return JF_ERR_INVALID_ARG;
   if (pool->head_dim != 128 && pool->head_dim != 256) return JF_ERR_UNSUPPORTED;
   if (pool->page_size != 64 && pool->page_size != 128 && pool->page_size != 256)
     return JF_ERR_UNSUPPORTED;
@@ -93,6 +117,24 @@ size_t jf_kv_page_bytes(int32_t num_kv_heads, int32_t page_size, int32_t head_di
   return (size_t)make_geom(p).page_bytes;
 }
 
+size_t jf_kv_page_bytes_fmt(int32_t format, int32_t num_kv_heads, int32_t page_size,
+                            int32_t head_dim) {
+  if (format != JF_FMT_AFFINE4_G64 && format != JF_FMT_TQ4) return 0;
+  if (num_kv_heads < 1 || page_size < 1 || (head_dim != 128 && head_dim != 256)) return 0;
+  jf_kv_pool p{};
+  p.num_pages = 1;
+  p.page_size = page_size;
+  p.num_kv_heads = num_kv_heads;
+  p.head_dim = head_dim;
+  p.format = format;
+  return (size_t)make_geom(p).page_bytes;
+}
+
+int jf_tq4_codebook(int32_t head_dim, float* centroids) {
+  if (!centroids || head_dim < 3 || head_dim > 65536) return JF_ERR_INVALID_ARG;
+  return tq4_codebook_host(head_dim, centroids);
+}
+
 size_t jf_attn_workspace_bytes(int32_t batch, int32_t num_q_heads, int32_t num_kv_heads,
                                int32_t head_dim, int32_t num_splits) {
   if (batch < 1 || num_q_heads < 1 || num_kv_heads < 1 || num_splits < 1) return 0;
@@ -107,13 +149,20 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
                           int32_t num_requests, const int32_t* row_req, const int32_t* row_pos,
                           const void* k, const void* v, int32_t n_rows, int32_t* err_flag,
                           void* stream) {
-  int st = check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (n_rows < 0 || pt_stride < 1 || num_requests < 1) return JF_ERR_INVALID_ARG;
   if (n_rows == 0) return JF_OK;
   if (!page_table || !row_req || !row_pos || !k || !v) return JF_ERR_INVALID_ARG;
   if (!aligned(k, 16) || !aligned(v, 16)) return JF_ERR_INVALID_ARG;
   const Geom g = make_geom(*pool);
+  if (pool->format == JF_FMT_TQ4) {
+    Tq4Params prm;
+    st = tq4_make_params(pool->tq4, g.D, &prm);
+    if (st) return st;
+    return launch_tq4_append(g, *pool, prm, page_table, pt_stride, num_requests, row_req,
+                             row_pos, k, v, n_rows, err_flag, static_cast<cudaStream_t>(stream));
+  }
   return launch_append(g, *pool, page_table, pt_stride, num_requests, row_req, row_pos, k, v,
                        n_rows, err_flag, static_cast<cudaStream_t>(stream));
 }
@@ -123,7 +172,8 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
                          const void* v_new, const void* q, int32_t num_q_heads,
                          float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
                          int32_t num_splits, void* stream, int32_t q_len = 1) {
-  int st = check_pool(pool);
+  // TQ4 pools: single-query decode without the fused append
+  int st = (q_len == 1 && !k_new) ? check_pool_any(pool) : check_pool(pool);
   if (st) return st;
   if (!page_table || !context_lens || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
   if (batch < 1 || batch > 65535 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
@@ -138,9 +188,19 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
                                               pool->head_dim, num_splits);
   if (workspace_bytes < need) return JF_ERR_WORKSPACE_TOO_SMALL;
   const Geom g = make_geom(*pool);
+  Tq4Params prm;
+  if (pool->format == JF_FMT_TQ4) {
+    st = tq4_make_params(pool->tq4, g.D, &prm);
+    if (st) return st;
+  }
   CUtensorMap tmap;
   st = make_codes_map(g, pool->base, decode_box_rows(), &tmap);
   if (st) return st;
+  if (pool->format == JF_FMT_TQ4) {
+    return launch_tq4_decode(g, *pool, tmap, prm, page_table, pt_stride, context_lens, batch, q,
+                             num_q_heads, softmax_scale, out, workspace, num_splits,
+                             static_cast<cudaStream_t>(stream));
+  }
   return launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q,
                        num_q_heads, softmax_scale, out, workspace, num_splits,
                        static_cast<cudaStream_t>(stream), k_new, v_new, q_len);
@@ -201,7 +261,7 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
 
 int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
                      void* dst, size_t dst_bytes, int32_t* err_flag, void* stream) {
-  int st = check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (num_pages < 0) return JF_ERR_INVALID_ARG;
   if (num_pages == 0) return JF_OK;
@@ -214,7 +274,7 @@ int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int3
 
 int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
                   const void* src, size_t src_bytes, int32_t* err_flag, void* stream) {
-  int st = check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (num_pages < 0) return JF_ERR_INVALID_ARG;
   if (num_pages == 0) return JF_OK;

@@ -22,9 +22,9 @@ struct Geom {
   // derived
   int32_t CB;     // code bytes per vector  = D/2
   int32_t NG;     // groups per vector      = D/64
-  int32_t SBB;    // scale/bias bytes per vector = 4*NG
+  int32_t SBB;    // side bytes per vector: 4*NG scale/bias (affine), 2 norm (TQ4)
   int64_t codes_region;  // Hkv*P*CB
-  int64_t sb_region;     // Hkv*P*SBB
+  int64_t sb_region;     // Hkv*P*SBB (scale/bias or norm region)
   int64_t page_bytes;
 };
 
@@ -36,7 +36,8 @@ inline Geom make_geom(const jf_kv_pool& p) {
   g.D = p.head_dim;
   g.CB = g.D / 2;
   g.NG = g.D / 64;
-  g.SBB = 4 * g.NG;
+  // side data per vector: affine scale/bias words, or the TQ4 fp16 norm
+  g.SBB = (p.format == JF_FMT_TQ4) ? 2 : 4 * g.NG;
   g.codes_region = (int64_t)g.Hkv * g.P * g.CB;
   g.sb_region = (int64_t)g.Hkv * g.P * g.SBB;
   g.page_bytes = 2 * g.codes_region + 2 * g.sb_region;

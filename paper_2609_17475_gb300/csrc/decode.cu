@@ -36,127 +36,13 @@
 #include <cmath>
 #include <cfloat>
 
+#include "decode.cuh"
 #include "quant.cuh"
 
 namespace jfkv {
 
-constexpr int DTOK = 32;      // positions per pipeline stage (one chunk)
 constexpr int DWARPS = 6;     // warps per split CTA (2 CTAs per SM)
 constexpr int DSTAGES = 2;    // stages per warp
-constexpr int MIN_CPS = 16;   // minimum chunks per split (512 positions)
-constexpr float DTAU = 4.f;   // log2 headroom before the reference maximum moves
-
-struct DecodeArgs {
-  const uint8_t* pool;
-  int64_t num_pages;
-  int64_t page_bytes;
-  int64_t codes_region;   // bytes of one code region (K or V) in a page record
-  int64_t sb_base;     // offset of the K scale/bias region in a page record
-  int64_t sb_region;   // bytes of one scale/bias region (K or V)
-  int32_t P, Hkv, Hq, G;
-  int32_t log2P;        // P is a power of two
-  const int32_t* page_table;
-  int32_t pt_stride;
-  const int32_t* ctx;
-  const uint16_t* q;
-  const uint16_t* knew;   // fused append: new K/V rows [B, Hkv, D], or null
-  const uint16_t* vnew;
-  uint16_t* out;
-  float* part_ml;      // [B, Hq, S, 2]
-  float* part_o;       // [B, Hq, S, D]
-  int32_t* status;
-  int32_t num_splits;
-  float scale_log2;    // softmax_scale * log2(e)
-  int32_t B;           // requests
-  int32_t L;           // query tokens per request (1: decode; 2-4: packed verifier)
-  int32_t NT;          // CTAs per KV head, each for 8 of its G * L (token, head) rows
-  int32_t HqL;         // L * Hq: rows of q, out and the partials per request
-  int32_t balanced;    // 1: batch split plan (balanced_plan), partial rows by global split
-  int32_t budget;      // balanced: target splits per KV head over the whole batch
-};
-
-__host__ __device__ inline void split_plan(int ctx, int num_splits, int& nch, int& cps,
-                                           int& nsplit) {
-  nch = (ctx + DTOK - 1) / DTOK;
-  if (nch <= 0) { nch = 0; cps = MIN_CPS; nsplit = 0; return; }
-  cps = (nch + num_splits - 1) / num_splits;
-  if (cps < MIN_CPS) cps = MIN_CPS;
-  nsplit = (nch + cps - 1) / cps;
-}
-
-// Batch split plan (B > 1).  Splits are sized for the whole batch, not per
-// request: with T the chunks of all requests, every request is cut into
-// pieces of cps = max(MIN_CPS, ceil(T / budget)) chunks, so each split CTA
-// streams about the same bytes however unequal the contexts are.  Request b
-// gets n_b = ceil(nch_b / cps) splits, numbered g0_b .. g0_b + n_b - 1 after
-// those of requests 0 .. b-1; the global number g names the split's partial
-// rows (g * Hq + hq).  Called by one whole warp; for a split CTA (x >= 0) it
-// finds the request and split of global split x (b = -1 when x is past the
-// last), for a merge CTA (want_b >= 0) the first global split and count of
-// request want_b.
-struct BalPlan {
-  int b, split, nsplit, g0, cps;
-};
-
-__device__ BalPlan balanced_plan(const DecodeArgs& a, int x, int want_b, int lane) {
-  const int64_t cap = (int64_t)a.pt_stride * a.P;
-  auto nch_of = [&](int bb) -> int {
-    int64_t c = a.ctx[bb];
-    c = c < 0 ? 0 : (c > cap ? cap : c);
-    return (int)((c + DTOK - 1) / DTOK);
-  };
-  long long T = 0;
-  for (int bb = lane; bb < a.B; bb += 32) T += nch_of(bb);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) T += __shfl_xor_sync(0xffffffffu, T, o);
-  int cps = (int)((T + a.budget - 1) / a.budget);
-  if (cps < MIN_CPS) cps = MIN_CPS;
-  BalPlan p{-1, 0, 0, 0, cps};
-  int base = 0;
-  for (int b0 = 0; b0 < a.B; b0 += 32) {
-    const int bb = b0 + lane;
-    const int n = (bb < a.B) ? (nch_of(bb) + cps - 1) / cps : 0;
-    int incl = n;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    const int excl = base + incl - n;
-    const bool hit = (x >= 0) ? (bb < a.B && x >= excl && x < excl + n) : (bb == want_b);
-    const unsigned m = __ballot_sync(0xffffffffu, hit);
-    if (m) {
-      const int src = __ffs(m) - 1;
-      p.b = __shfl_sync(0xffffffffu, bb, src);
-      p.g0 = __shfl_sync(0xffffffffu, excl, src);
-      p.nsplit = __shfl_sync(0xffffffffu, n, src);
-      p.split = (x >= 0) ? x - p.g0 : 0;
-      return p;
-    }
-    base += __shfl_sync(0xffffffffu, incl, 31);
-  }
-  return p;
-}
-
-__device__ __forceinline__ int checked_ctx(const DecodeArgs& a, int b) {
-  int ctx = a.ctx[b];
-  const int64_t cap = (int64_t)a.pt_stride * a.P;
-  if (ctx < 0 || ctx > cap) {
-    if (threadIdx.x == 0 && blockIdx.x == 0) flag_error(a.status, JF_DEV_ERR_POSITION);
-    ctx = ctx < 0 ? 0 : (int)cap;
-  }
-  return ctx;
-}
-
-// Byte offset of 16-byte chunk `ch` of code row `t` inside a TMA-swizzled
-// stage buffer (128B swizzle for 128-byte rows, 64B swizzle for 64-byte rows).
-template <int CB>
-__device__ __forceinline__ uint32_t swz(int t, int ch) {
-  if constexpr (CB == 128)
-    return t * 128 + ((ch ^ (t & 7)) << 4);
-  else
-    return t * 64 + ((ch ^ ((t >> 1) & 3)) << 4);
-}
 
 // (w >> 8) as an integer multiply-high, which runs on the FMA pipe and spares
 // the ALU pipe that the nibble masks already load.
@@ -1002,7 +888,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 constexpr int BAL_MAX_B = 1024;   // batch plan limit (each plan reads every context length)
 
 // SMs of the current device (cached per device)
-static int sm_count() {
+int sm_count() {
   static int cache[256] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return 152;
@@ -1022,6 +908,24 @@ size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S) {
   const int64_t rows = B * Hq * S;
   const int64_t ml = (rows * 8 + 255) / 256 * 256;
   return (size_t)(256 + ml + rows * D * 4);
+}
+
+// Merge phase: one CTA per (32-wide slice of head_dim, row, request), launched
+// with programmatic dependent launch after the split kernel.
+int launch_decode_merge(const DecodeArgs& a, int D, int B, cudaStream_t stream) {
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t mc = {};
+  mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.HqL, (unsigned)B);
+  mc.blockDim = dim3(MERGE_THREADS);
+  mc.dynamicSmemBytes = 0;
+  mc.stream = stream;
+  mc.attrs = pdl;
+  mc.numAttrs = 1;
+  const cudaError_t e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256>, a)
+                                   : cudaLaunchKernelEx(&mc, decode_merge_kernel<128>, a);
+  return e == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }
 
 template <int D>
@@ -1056,16 +960,7 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   const cudaError_t e = (a.L > 1) ? cudaLaunchKernelEx(&cfg, decode_split_kernel<D, true>, tmap, a)
                                   : cudaLaunchKernelEx(&cfg, decode_split_kernel<D, false>, tmap, a);
   if (e != cudaSuccess) return JF_ERR_CUDA;
-  if (a.num_splits > 1) {
-    cudaLaunchConfig_t mc = {};
-    mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.HqL, (unsigned)B);
-    mc.blockDim = dim3(MERGE_THREADS);
-    mc.dynamicSmemBytes = 0;
-    mc.stream = stream;
-    mc.attrs = pdl;
-    mc.numAttrs = 1;
-    if (cudaLaunchKernelEx(&mc, decode_merge_kernel<D>, a) != cudaSuccess) return JF_ERR_CUDA;
-  }
+  if (a.num_splits > 1) return launch_decode_merge(a, D, B, stream);
   return JF_OK;
 }
 

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from paper_2609_17475_gb300 import binding as B
@@ -61,7 +62,8 @@ FAKE = ctypes.c_void_p(0x20000)   # aligned, never dereferenced: validation fail
     (dict(head_dim=96), B.JF_ERR_UNSUPPORTED),
     (dict(page_size=100), B.JF_ERR_UNSUPPORTED),
     (dict(group_size=32), B.JF_ERR_UNSUPPORTED),
-    (dict(format=1), B.JF_ERR_UNSUPPORTED),
+    (dict(format=1), B.JF_ERR_INVALID_ARG),        # TQ4 without its codec
+    (dict(format=2), B.JF_ERR_UNSUPPORTED),
     (dict(num_pages=0), B.JF_ERR_INVALID_ARG),
 ])
 def test_decode_rejects_bad_pool(kw, expect):
@@ -110,3 +112,57 @@ def test_append_checkpoint_prefill_reject_bad_arguments():
                                    256, None) == B.JF_ERR_INVALID_ARG
     assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 0, 8, 0.1, 1, FAKE, FAKE,
                                    256, None) == B.JF_OK           # empty chunk: no-op
+
+
+# -- TQ4 (Sec. 3.1 Eq. 4; App. A.1 Table 3): host-side logic --------------------
+def _tq4_pool(codec, **kw):
+    p = _pool(format=B.JF_FMT_TQ4, **kw)
+    p.tq4 = ctypes.pointer(codec._c)
+    return p
+
+
+def _codec(d=128):
+    from paper_2609_17475_gb300 import synth
+    return B.Tq4Codec(d, synth.tq4_signs(0, d), synth.tq4_signs(1, d))
+
+
+@pytest.mark.parametrize("d", [3, 64, 128, 256])
+def test_tq4_codebook_equals_the_oracle_bit_for_bit(d):
+    from oracle import tq4
+    assert np.array_equal(B.jf_tq4_codebook(d), tq4.codebook(d))
+
+
+def test_tq4_page_bytes_follow_eq2():
+    assert B.jf_kv_page_bytes_fmt(B.JF_FMT_TQ4, 4, 256, 256) == 256 * 1040
+    assert B.jf_kv_page_bytes_fmt(B.JF_FMT_AFFINE4_G64, 4, 256, 256) == B.jf_kv_page_bytes(4, 256, 256)
+    assert B.jf_kv_page_bytes_fmt(7, 4, 256, 256) == 0
+    assert B.lib().jf_tq4_codebook(2, (ctypes.c_float * 16)()) == B.JF_ERR_INVALID_ARG
+
+
+def test_tq4_bad_codecs_and_unsupported_entry_points():
+    L = B.lib()
+    c = _codec()
+    p = _tq4_pool(c)
+    dec = lambda pool: L.jf_paged_decode_attn(ctypes.byref(pool), FAKE, 4, FAKE, 1, FAKE, 8, 0.1,
+                                               FAKE, FAKE, 1 << 20, 4, None)
+    bad = _codec()
+    bad._c.centroids[3] = bad._c.centroids[2]          # not strictly ascending
+    assert dec(_tq4_pool(bad)) == B.JF_ERR_INVALID_ARG
+    bad = _codec()
+    bad._c.signs_v[5] = 0                              # not +-1
+    assert dec(_tq4_pool(bad)) == B.JF_ERR_INVALID_ARG
+    assert L.jf_kv_quantize_append(ctypes.byref(_tq4_pool(bad)), FAKE, 4, 1, FAKE, FAKE, FAKE,
+                                   FAKE, 5, None, None) == B.JF_ERR_INVALID_ARG
+    # entry points without TQ4 support
+    assert L.jf_paged_verify_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 2, 8, 0.1, FAKE, FAKE,
+                                  1 << 20, 4, None) == B.JF_ERR_UNSUPPORTED
+    assert L.jf_paged_decode_append_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, FAKE, FAKE, 8,
+                                         0.1, FAKE, FAKE, 1 << 20, 4, None) == B.JF_ERR_UNSUPPORTED
+    assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 16, 8, 0.1, 1, FAKE, FAKE, 256,
+                                   None) == B.JF_ERR_UNSUPPORTED
+    assert L.jf_paged_decode_attn_noalloc(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 8, 0.1, FAKE, 4,
+                                          None, None) == B.JF_ERR_UNSUPPORTED
+    # checkpoint sizes use the TQ4 page record
+    pb = B.jf_kv_page_bytes_fmt(B.JF_FMT_TQ4, 2, 256, 128)
+    assert L.jf_kv_checkpoint(ctypes.byref(p), FAKE, 3, FAKE, 3 * pb - 1, None,
+                              None) == B.JF_ERR_INVALID_ARG

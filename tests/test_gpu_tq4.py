@@ -1,0 +1,292 @@
+"""GPU parity for the TQ4 format (Sec. 3.1 Eq. 4; App. A.1 Table 3): encode on
+append bit-exact against the oracle (indices and fp16 norms), page-native
+decode attention within tolerance of the fp64 oracle, checkpoint/restore byte
+identity.  Every call goes through the C ABI (libjfkv.so)."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_17475_gb300 as jf
+from oracle import attention as OT
+from oracle import checkpoint as OC
+from oracle import tq4 as OQ
+from paper_2609_17475_gb300 import synth
+from tests.cases import assert_attention_close, bits, make_case
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def signs(D):
+    return synth.tq4_signs(synth.TQ4_SEED_K, D), synth.tq4_signs(synth.TQ4_SEED_V, D)
+
+
+def oracle_layout(case):
+    sk, sv = signs(case.D)
+    return OQ.Tq4Layout(case.Hkv, case.P, case.D, OQ.make_codec(case.D, sk, sv))
+
+
+def oracle_pool(case, fill=0):
+    lay = oracle_layout(case)
+    pool = OQ.new_pool(lay, case.num_pages, fill=fill)
+    OQ.append(pool, lay, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
+              bits(case.k), bits(case.v))
+    return lay, pool
+
+
+def gpu_pool(case, fill=0):
+    sk, sv = signs(case.D)
+    return jf.KVPool.allocate(case.num_pages, case.P, case.Hkv, case.D, device=DEV, fill=fill,
+                              format=jf.JF_FMT_TQ4, codec=jf.Tq4Codec(case.D, sk, sv))
+
+
+def gpu_append(case, fill=0, k=None, v=None):
+    pool = gpu_pool(case, fill)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, case.page_table.to(DEV), case.req.to(DEV), case.pos.to(DEV),
+                             (case.k if k is None else k).to(DEV),
+                             (case.v if v is None else v).to(DEV), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    return pool
+
+
+def pool_from_numpy(case, arr):
+    pool = gpu_pool(case, fill=None)
+    pool.data.copy_(torch.from_numpy(arr))
+    return pool
+
+
+def gpu_decode(case, pool, splits, ctx=None):
+    ctx = case.ctx if ctx is None else ctx
+    B = len(ctx)
+    out = torch.full((B, case.Hq, case.D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(B, case.Hq, case.Hkv, case.D, splits, device=DEV)
+    ws[256:] = 0xFF    # NaN partials: rows past the split plan must never be used
+    jf.jf_paged_decode_attn(pool, case.page_table.to(DEV),
+                            torch.tensor(ctx, dtype=torch.int32, device=DEV), case.q.to(DEV),
+                            1 / math.sqrt(case.D), out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    return out
+
+
+# --------------------------------------------------------------------------
+# codebook: the library's construction equals the oracle's, bit for bit
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("D", [128, 256])
+def test_tq4_codebook_bit_exact(D):
+    assert np.array_equal(jf.jf_tq4_codebook(D), OQ.codebook(D))
+
+
+# --------------------------------------------------------------------------
+# encode on append: bit-exact against the oracle
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hkv,D,P,ctx,outliers", [
+    (2, 128, 256, [256], False),
+    (2, 128, 64, [1, 63, 130], False),
+    (4, 256, 256, [1000, 517], True),
+    (3, 256, 128, [300], True),
+    (1, 256, 64, [2048], False),
+])
+def test_tq4_append_bit_exact(Hkv, D, P, ctx, outliers):
+    case = make_case(300 + sum(ctx), 2 * Hkv, Hkv, D, P, ctx, outliers=outliers,
+                     num_pages=sum(-(-c // P) for c in ctx) + 2)
+    _, ref = oracle_pool(case, fill=0x5A)
+    pool = gpu_append(case, fill=0x5A)
+    assert np.array_equal(pool.data.cpu().numpy(), ref)
+
+
+def test_tq4_append_special_vectors_bit_exact():
+    """Zero vectors, one-hot vectors, norms past the fp16 range (saturated),
+    tiny magnitudes, a 2^30 magnitude spread, signed zeros."""
+    D, Hkv, P = 256, 2, 64
+    n = 64
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal((2, n, Hkv, D)).astype(np.float32)
+    x[:, 0] = 0.0
+    x[:, 1] = 0.0
+    x[:, 1, :, 7] = -2.5                                   # one-hot
+    x[:, 2] *= 5000.0                                      # norm ~80000 > 65504
+    x[:, 3] *= 1e-20                                       # tiny
+    x[:, 4, :, ::2] *= 2.0 ** -30                          # wide spread
+    x[:, 5, :, ::3] = -0.0
+    x[:, 6] = 1.0                                          # all equal
+    kb = torch.from_numpy(x[0]).to(torch.bfloat16)
+    vb = torch.from_numpy(x[1]).to(torch.bfloat16)
+    case = make_case(9, 2 * Hkv, Hkv, D, P, [n], num_pages=2)
+    case.k, case.v = kb, vb
+    _, ref = oracle_pool(case, fill=0x11)
+    pool = gpu_append(case, fill=0x11)
+    assert np.array_equal(pool.data.cpu().numpy(), ref)
+
+
+def test_tq4_append_many_rows_exercises_both_decision_paths():
+    """8,192 vectors: some lie within 2^-15 rho of a threshold and take the
+    exact fp64 path; all must match the oracle."""
+    case = make_case(77, 8, 4, 256, 256, [1024], outliers=True)
+    _, ref = oracle_pool(case)
+    pool = gpu_append(case)
+    assert np.array_equal(pool.data.cpu().numpy(), ref)
+
+
+def test_tq4_append_flags_bad_rows_and_skips_them():
+    case = make_case(13, 8, 2, 128, 64, [100], num_pages=3)
+    pool = gpu_pool(case, fill=0x77)
+    before = pool.data.clone()
+    pos = case.pos.clone()
+    pos[5] = 10 ** 6                     # beyond the page-table row
+    pt = case.page_table.clone()
+    pt[0, 1] = 999                       # page id outside the pool
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, pt.to(DEV), case.req.to(DEV), pos.to(DEV), case.k.to(DEV),
+                             case.v.to(DEV), err)
+    torch.cuda.synchronize()
+    e = int(err.item())
+    assert e & jf.binding.JF_DEV_ERR_POSITION and e & jf.binding.JF_DEV_ERR_PAGE_ID
+    # rows 64..99 went to the bad page id and were skipped: the page they
+    # would have used under the original table is untouched
+    orig = int(case.page_table[0, 1])
+    assert torch.equal(before[orig], pool.data[orig])
+
+
+# --------------------------------------------------------------------------
+# checkpoint / restore
+# --------------------------------------------------------------------------
+def test_tq4_checkpoint_and_restore_bit_exact():
+    case = make_case(17, 8, 4, 256, 128, [1500], num_pages=15)
+    _, ref = oracle_pool(case, fill=0x33)
+    pool = pool_from_numpy(case, ref)
+    n = -(-1500 // 128)
+    blob = torch.empty(n * pool.page_bytes, dtype=torch.uint8, device=DEV)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_checkpoint(pool, case.page_table[0].to(DEV), n, blob, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    want = OC.checkpoint(ref, case.page_table[0].numpy(), n)
+    assert np.array_equal(blob.cpu().numpy(), want)
+    fresh = gpu_pool(case, fill=0)
+    jf.jf_kv_restore(fresh, case.page_table[0].to(DEV), n, blob, err)
+    torch.cuda.synchronize()
+    exp = np.zeros_like(ref)
+    OC.restore(exp, case.page_table[0].numpy(), n, want)
+    assert np.array_equal(fresh.data.cpu().numpy(), exp)
+
+
+# --------------------------------------------------------------------------
+# decode attention
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,splits,outliers", [
+    (8, 2, 128, 256, [4096], 1, False),            # tiny geometry, one split
+    (8, 2, 128, 256, [4096], 8, False),            # split-K + merge
+    (8, 2, 128, 64, [1, 33, 517, 2000], 4, False),  # ragged batch, partial pages
+    (24, 4, 256, 256, [5000], 3, True),            # paper geometry, outliers
+    (24, 4, 256, 128, [777, 1], 16, True),
+    (4, 4, 256, 64, [1500], 2, False),             # G = 1
+    (16, 2, 256, 256, [2500], 5, False),           # G = 8
+    (8, 2, 128, 256, [70000, 3000], 150, False),   # > 128 live splits
+    (24, 4, 256, 128, [9000, 0, 40], 3, True),     # batch plan with an empty request
+])
+def test_tq4_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
+    case = make_case(400 + Hq + sum(ctx), Hq, Hkv, D, P, ctx, outliers=outliers)
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    out = gpu_decode(case, pool, splits)
+    ref = OT.paged_decode(ref_pool, lay, case.page_table.numpy(), ctx, bits(case.q),
+                          1 / math.sqrt(D))
+    assert_attention_close(out, ref)
+
+
+def test_tq4_decode_edge_contexts():
+    case = make_case(6, 8, 2, 128, 64, [0, 1, 64, 65])
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    for splits in (1, 4):
+        out = gpu_decode(case, pool, splits)
+        assert (out[0].float() == 0).all()
+        ref = OT.paged_decode(ref_pool, lay, case.page_table.numpy(), case.ctx, bits(case.q),
+                              1 / math.sqrt(128))
+        assert_attention_close(out, ref)
+        v0 = OT.gather_head(ref_pool, lay, case.page_table.numpy()[1], 1, 0, OQ.KIND_V)[0]
+        assert np.abs(out[1, 0].float().cpu().numpy() - v0).max() <= 2 ** -7 * np.abs(v0).max()
+
+
+def test_tq4_decode_poison_pages_and_tail_never_leak():
+    """0xFF bytes (fp16 norm NaN) in unwritten pages and tail slots stay out."""
+    case = make_case(62, 8, 2, 128, 64, [200], num_pages=10)
+    lay, ref_pool = oracle_pool(case, fill=0xFF)
+    pool = pool_from_numpy(case, ref_pool)
+    out = gpu_decode(case, pool, 2)
+    ref = OT.paged_decode(ref_pool, lay, case.page_table.numpy(), case.ctx, bits(case.q),
+                          1 / math.sqrt(128))
+    assert_attention_close(out, ref)
+
+
+def test_tq4_decode_after_gpu_append_and_split_invariance():
+    case = make_case(81, 24, 4, 256, 256, [12000], outliers=True)
+    lay, ref_pool = oracle_pool(case)
+    pool = gpu_append(case)
+    assert np.array_equal(pool.data.cpu().numpy(), ref_pool)
+    ref = OT.paged_decode(ref_pool, lay, case.page_table.numpy(), case.ctx, bits(case.q), 1 / 16)
+    outs = [gpu_decode(case, pool, s) for s in (1, 2, 7, 38)]
+    for o in outs:
+        assert_attention_close(o, ref)
+
+
+def test_tq4_rejected_by_entry_points_without_tq4_support():
+    case = make_case(3, 8, 2, 128, 64, [100])
+    pool = gpu_pool(case)
+    ws = jf.verify_workspace(1, 2, 8, 2, 128, 2, device=DEV)
+    q2 = torch.zeros(1, 2, 8, 128, dtype=torch.bfloat16, device=DEV)
+    with pytest.raises(jf.JfError) as e:
+        jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
+                                torch.tensor([100], dtype=torch.int32, device=DEV), q2, 0.1,
+                                torch.empty_like(q2), ws, 2)
+    assert e.value.status == jf.binding.JF_ERR_UNSUPPORTED
+
+
+def test_tq4_decode_full_window_256k_one_head():
+    """The 256K full-window workload (24/4/256, 1,024 pages in a random physical
+    order, K outlier channels) in TQ4 at full size and in the benchmark's launch
+    shape; KV head 2 checked against the oracle, bytes of sampled pages too."""
+    w = synth.WORKLOADS["full_window_256k"]
+    geo = w["geometry"]
+    ctx = w["context_lens"][0]
+    gen = synth.generator(w["seed"])
+    channels = synth.outlier_channels(gen, geo.num_kv_heads, geo.head_dim)
+    k, v = synth.kv_rows(gen, ctx, geo.num_kv_heads, geo.head_dim, channels)
+    pt, npages = synth.page_tables(gen, [ctx], geo.page_size)
+    q = synth.normal_bf16(gen, (1, geo.num_q_heads, geo.head_dim))
+    req, pos = synth.append_rows_for([ctx])
+    sk, sv = signs(geo.head_dim)
+    pool = jf.KVPool.allocate(npages, geo.page_size, geo.num_kv_heads, geo.head_dim, device=DEV,
+                              format=jf.JF_FMT_TQ4, codec=jf.Tq4Codec(geo.head_dim, sk, sv))
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, pt.to(DEV), req.to(DEV), pos.to(DEV), k.to(DEV), v.to(DEV), err)
+    splits = jf.default_num_splits(1, geo.num_kv_heads, format=jf.JF_FMT_TQ4)
+    out = torch.empty(1, geo.num_q_heads, geo.head_dim, dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(1, geo.num_q_heads, geo.num_kv_heads, geo.head_dim, splits, device=DEV)
+    scale = 1 / math.sqrt(geo.head_dim)
+    jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor([ctx], dtype=torch.int32, device=DEV),
+                            q.to(DEV), scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws) == 0
+    G, kvh = geo.group, 2
+    L1 = OQ.Tq4Layout(1, geo.page_size, geo.head_dim, OQ.make_codec(geo.head_dim, sk, sv))
+    opool = OQ.new_pool(L1, npages)
+    OQ.append(opool, L1, pt.numpy(), req.numpy(), pos.numpy(),
+              bits(k[:, kvh:kvh + 1]), bits(v[:, kvh:kvh + 1]))
+    ref = OT.paged_decode(opool, L1, pt.numpy(), [ctx], bits(q[:, kvh * G:(kvh + 1) * G]), scale)
+    assert_attention_close(out[:, kvh * G:(kvh + 1) * G], ref)
+    gp = pool.data.cpu().numpy()
+    L4 = OQ.Tq4Layout(geo.num_kv_heads, geo.page_size, geo.head_dim, L1.codec)
+    for page in pt[0, [0, 511, 1023]].tolist():
+        for kind in (OQ.KIND_K, OQ.KIND_V):
+            o4, o1 = L4.codes_offset(kind, kvh, 0), L1.codes_offset(kind, 0, 0)
+            n = geo.page_size * L4.code_bytes
+            assert np.array_equal(gp[page, o4:o4 + n], opool[page, o1:o1 + n])
+            o4, o1 = L4.norm_offset(kind, kvh, 0), L1.norm_offset(kind, 0, 0)
+            assert np.array_equal(gp[page, o4:o4 + 2 * geo.page_size],
+                                  opool[page, o1:o1 + 2 * geo.page_size])
