@@ -38,7 +38,7 @@ UNIT = "positions/s"
 
 def measured_traffic(kernel):
     """DRAM bytes per launch of `kernel` from the committed ncu record, or None
-    when the kernel source changed since the capture."""
+    when any of the kernel's source files changed since the capture."""
     import hashlib
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
@@ -46,9 +46,10 @@ def measured_traffic(kernel):
     rec = json.load(open(p)).get(kernel)
     if not rec:
         return None
-    src = os.path.join(ROOT, rec["source"])
-    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != rec["sha256"]:
-        return None
+    for name, sha in rec["sources"].items():
+        src = os.path.join(ROOT, name)
+        if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != sha:
+            return None
     return rec["dram_read"] + rec["dram_write"]
 
 
@@ -346,7 +347,7 @@ def _event_time(fn, reps, stream):
 ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify", "tq4")
 
 
-def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
+def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None, tq4_copies=8):
     """Tiny decode, append, prefill chunk, decode loop, checkpoint, two-request and
     mixed-batch decode (`only` selects one group of ROW_GROUPS).  Every tensor is
     allocated on `stream`, the stream the kernels run on, so the caching allocator
@@ -356,7 +357,7 @@ def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
         if only is None or only == "verify":
             out["verify_256k"] = _bench_verify(jf, dev, stream)
         if only is None or only == "tq4":
-            out["tq4_256k"] = _bench_tq4(jf, synth, dev, stream, peaks_gbs)
+            out["tq4_256k"] = _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=tq4_copies)
         return out
 
 
@@ -413,7 +414,8 @@ def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
     gbs = alg / (t / 1e3) / 1e9
     res = {"decode_us": t * 1e3, "positions_per_s": ctx / (t / 1e3), "GBps": gbs,
            "frac_of_measured": gbs / peaks_gbs, "splits": splits, "bytes_per_position": bpp,
-           "alg_bytes_per_call": alg, "append_2048_rows_us": ta * 1e3,
+           "alg_bytes_per_call": alg, "traffic": measured_traffic("tq4_split_kernel<256>"),
+           "append_2048_rows_us": ta * 1e3,
            "append_GBps": (2048 * Hkv * D * 2 * 2 + 2048 * bpp) / (ta / 1e3) / 1e9}
     del pools
     return res
@@ -730,6 +732,8 @@ def main():
     ap.add_argument("--row", choices=ROW_GROUPS, default=None,
                     help="run only this group of the row measurements (for profiling) and "
                          "print it; no bench line")
+    ap.add_argument("--copies", type=int, default=8,
+                    help="independent 256K caches the tq4 row cycles through (1 for profiling)")
     args = ap.parse_args()
     if args.row:
         import paper_2609_17475_gb300 as jf
@@ -740,7 +744,8 @@ def main():
         pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
         peak_tf = float(json.load(open(pk))["bf16_tflops"]) if os.path.exists(pk) else 1900.0
         stream = torch.cuda.Stream(device=dev)
-        print(json.dumps(bench_rows(jf, synth, dev, stream, hbm, peak_tf, only=args.row)))
+        print(json.dumps(bench_rows(jf, synth, dev, stream, hbm, peak_tf, only=args.row,
+                                    tq4_copies=args.copies)))
         return
     args.warmup = max(3, args.warmup)
     world, rank, local = dist_env()

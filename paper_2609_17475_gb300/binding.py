@@ -139,7 +139,9 @@ class Tq4Codec:
     K and V random-sign vectors (+1 / -1, length head_dim), which the caller
     draws (synth.tq4_signs gives the paper's NumPy draw)."""
 
-    def __init__(self, head_dim: int, signs_k, signs_v):
+    def __init__(self, head_dim: int, signs_k, signs_v, centroids=None):
+        """``centroids`` (16 ascending fp32 values, |c| < 1) replaces the
+        library's Lloyd-Max codebook when given."""
         import numpy as np
         sk = np.asarray(signs_k).astype(np.int64)
         sv = np.asarray(signs_v).astype(np.int64)
@@ -148,7 +150,12 @@ class Tq4Codec:
         if not (np.isin(sk, (-1, 1)).all() and np.isin(sv, (-1, 1)).all()):
             raise ValueError("signs must be +1 or -1")
         self.head_dim = int(head_dim)
-        self.centroids = jf_tq4_codebook(head_dim)
+        if centroids is None:
+            self.centroids = jf_tq4_codebook(head_dim)
+        else:
+            self.centroids = np.asarray(centroids, dtype=np.float32).copy()
+            if self.centroids.shape != (16,):
+                raise ValueError("a TQ4 codebook has 16 centroids")
         self.signs_k, self.signs_v = sk, sv
         c = _Tq4Codec()
         for i in range(16):

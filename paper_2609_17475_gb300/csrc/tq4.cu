@@ -15,8 +15,10 @@
 // within 2^-17 rho of the exact value: 8 levels of rounding, each at most
 // 2^-24 of a partial sum bounded by sum|x| <= sqrt(d) rho), and a warp with
 // any closer element redoes its vector with the fp64 butterfly, which is
-// exact for bf16 inputs whose magnitudes span less than 2^37.  rho is the fp32
-// rounding of the square root of the fp64 sum of squares.
+// exact for bf16 inputs whose magnitudes span less than 2^37, and compares
+// those elements with the thresholds their fast-path bracket leaves open.
+// rho is the fp32 rounding of the square root of the fp64 sum of squares,
+// obtained from a certified double-float sum (fp64 only near a tie).
 //
 // Decode.  The query is rotated once per CTA, q' = H_d S_K q / sqrt(d), so
 //   <q, K_t> = rho_hat_t <q', c[z_t]>,  sum_t p_t V_t = S_V H_d (sum_t p_t
@@ -108,6 +110,12 @@ int tq4_make_params(const jf_tq4_codec* codec, int d, Tq4Params* p) {
     p->t[k] = s * 0.5f;
     p->tq[k] = sd * p->t[k];
   }
+  // the append's fast path needs neighbouring thresholds more than 4 margins
+  // (2^-15 rho each) apart; a codebook with closer ones decides every index
+  // in fp64
+  p->exact_all = 0;
+  for (int k = 0; k < 14; ++k)
+    if (!((double)p->tq[k + 1] - (double)p->tq[k] > 0x1p-12)) p->exact_all = 1;
   for (int j = 0; j < 8; ++j) p->sk[j] = p->sv[j] = 0u;
   for (int j = 0; j < d; ++j) {
     const int a = codec->signs_k[j], b = codec->signs_v[j];
@@ -171,13 +179,47 @@ __device__ __forceinline__ void warp_fwht(T (&u)[E], int lane) {
   }
 #pragma unroll
   for (int m = 1; m < 32; m <<= 1) {
-    const bool upper = (lane & m) != 0;
+    // lower lane: u + o; upper lane: o - u (one rounding either way)
+    const T sg = (lane & m) ? T(-1) : T(1);
 #pragma unroll
     for (int i = 0; i < E; ++i) {
       const T o = __shfl_xor_sync(0xffffffffu, u[i], m);
-      u[i] = upper ? (o - u[i]) : (u[i] + o);
+      u[i] = fma(u[i], sg, o);
     }
   }
+}
+
+// Count of the 15 ascending thresholds T_k with u > T_k, by a branch-free
+// 4-level search, and the thresholds bracketing u (lo < u <= hi; -inf / +inf
+// past the ends).
+__device__ __forceinline__ int bracket15(float u, const float (&T)[15], float& lo, float& hi) {
+  const bool b3 = u > T[7];
+  lo = b3 ? T[7] : -INFINITY;
+  hi = b3 ? INFINITY : T[7];
+  const float t2 = b3 ? T[11] : T[3];
+  const bool b2 = u > t2;
+  lo = b2 ? t2 : lo;
+  hi = b2 ? hi : t2;
+  const float t1 = b3 ? (b2 ? T[13] : T[9]) : (b2 ? T[5] : T[1]);
+  const bool b1 = u > t1;
+  lo = b1 ? t1 : lo;
+  hi = b1 ? hi : t1;
+  const float t0 = b3 ? (b2 ? (b1 ? T[14] : T[12]) : (b1 ? T[10] : T[8]))
+                      : (b2 ? (b1 ? T[6] : T[4]) : (b1 ? T[2] : T[0]));
+  const bool b0 = u > t0;
+  lo = b0 ? t0 : lo;
+  hi = b0 ? hi : t0;
+  return (b3 ? 8 : 0) + (b2 ? 4 : 0) + (b1 ? 2 : 0) + (b0 ? 1 : 0);
+}
+
+// (s_hi, s_lo) += b for a double-float accumulator (Knuth's TwoSum; the
+// error term of s_hi + b is exact)
+__device__ __forceinline__ void two_sum_acc(float& sh, float& sl, float b) {
+  const float s = __fadd_rn(sh, b);
+  const float bb = __fsub_rn(s, sh);
+  const float err = __fadd_rn(__fsub_rn(sh, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  sh = s;
+  sl = __fadd_rn(sl, err);
 }
 
 template <int D>
@@ -198,13 +240,45 @@ __global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, 
   load_bf16<E>((kind ? a.v : a.k) + (row * a.Hkv + head) * D + lane * E, x);
   const uint32_t sbits = ((kind ? prm.sv : prm.sk)[(lane * E) >> 5]) >> ((lane * E) & 31);
 
-  // rho: fp32 rounding of sqrt of the fp64 sum of squares (each square exact)
-  double s = 0.0;
+  // rho = RN32(sqrt(s)), s the fp64 sum of squares.  Squares of bf16 values
+  // are exact in fp32; their sum is carried as a double-float (TwoSum, error
+  // about 2^-40 s) and its square root rounded from r = RN32(sqrt(s_hi)) and
+  // the exact residual s_hi - r^2 (one fma).  When the result lies within
+  // 2^-10 half-ulp of a rounding boundary, or s is out of the safe range, the
+  // warp recomputes s in fp64 (GB300's fp64 rate is low, so this stays rare).
+  float sh = 0.f, sl = 0.f;
 #pragma unroll
-  for (int e = 0; e < E; ++e) s += (double)x[e] * (double)x[e];
+  for (int e = 0; e < E; ++e) two_sum_acc(sh, sl, __fmul_rn(x[e], x[e]));
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  const float rho = __double2float_rn(sqrt(s));
+  for (int o = 16; o > 0; o >>= 1) {
+    const float bh = __shfl_xor_sync(0xffffffffu, sh, o);
+    const float bl = __shfl_xor_sync(0xffffffffu, sl, o);
+    two_sum_acc(sh, sl, bh);
+    sl = __fadd_rn(sl, bl);
+  }
+  float rho;
+  {
+    const float r = __fsqrt_rn(sh);
+    const float res = __fmaf_rn(-r, r, sh);                // exact: s_hi - r^2
+    // sqrt(s) = r + dl up to ~2^-41 r; rounding boundaries at half an ulp on
+    // either side (the spacing below a power of two is half the one above)
+    const float dl = __fmul_rn(__fadd_rn(res, sl), __fdiv_rn(0.5f, r));
+    const float up = __int_as_float(__float_as_int(r) + 1);
+    const float dn = __int_as_float(__float_as_int(r) - 1);
+    const float half = (dl > 0.f) ? 0.5f * (up - r) : 0.5f * (r - dn);
+    const float ad = fabsf(dl);
+    const bool sure = (sh >= 0x1p-100f) && (sh <= 0x1p+120f) &&
+                      (fabsf(ad - half) > half * 0x1p-10f) && !(ad > 2.f * half);
+    rho = (ad < half) ? r : (dl > 0.f ? up : dn);
+    if (!sure) {   // uniform: every lane holds the same (sh, sl)
+      double s = 0.0;
+#pragma unroll
+      for (int e = 0; e < E; ++e) s += (double)x[e] * (double)x[e];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      rho = __double2float_rn(sqrt(s));
+    }
+  }
 
   // fast path: fp32 butterfly, decided where no threshold is within 2^-15 rho
   float u[E];
@@ -215,34 +289,38 @@ __global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, 
 #pragma unroll
   for (int k = 0; k < 15; ++k) T[k] = rho * prm.tq[k];
   const float M = rho * 0x1p-15f;
-  bool near = !(rho >= 1e-30f && rho <= 1e36f);
-  uint32_t word = 0;
+  bool near = !(rho >= 1e-30f && rho <= 1e36f) || prm.exact_all;
+  // thresholds are farther apart than 2M, so only the two bracketing ones can
+  // lie within M of u
+  uint32_t word = 0, nearmask = 0;
 #pragma unroll
   for (int e = 0; e < E; ++e) {
-    const float lo = u[e] - M, hi = u[e] + M;
-    int zlo = 0, zhi = 0;
-#pragma unroll
-    for (int k = 0; k < 15; ++k) {
-      zlo += (lo > T[k]) ? 1 : 0;
-      zhi += (hi > T[k]) ? 1 : 0;
-    }
-    near = near || (zlo != zhi);
-    word |= (uint32_t)zlo << (4 * e);
+    float lo, hi;
+    const int z = bracket15(u[e], T, lo, hi);
+    if (u[e] - lo <= M || hi - u[e] <= M) nearmask |= 1u << e;
+    word |= (uint32_t)z << (4 * e);
   }
+  near = near || (nearmask != 0);
   if (__any_sync(0xffffffffu, near)) {
-    // exact path: fp64 butterfly and the threshold products T_k of the contract
+    // exact path: fp64 butterfly; an element within M of a threshold compares
+    // against the contract's threshold products T_k = fp64(fp64(sqrt(D) rho)
+    // t_k) for its two bracketing thresholds (all 15 when the norm is outside
+    // the fast path's range)
     double ud[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) ud[e] = ((sbits >> e) & 1u) ? -(double)x[e] : (double)x[e];
     warp_fwht<double, E>(ud, lane);
     const double r = (double)rho * sqrt((double)D);
-    word = 0;
+    const bool all = !(rho >= 1e-30f && rho <= 1e36f) || prm.exact_all;
 #pragma unroll
     for (int e = 0; e < E; ++e) {
-      int z = 0;
-#pragma unroll
-      for (int k = 0; k < 15; ++k) z += (ud[e] > r * (double)prm.t[k]) ? 1 : 0;
-      word |= (uint32_t)z << (4 * e);
+      if (all || ((nearmask >> e) & 1u)) {
+        const int zf = (word >> (4 * e)) & 0xF;
+        const int k0 = all ? 0 : max(zf - 1, 0), k1 = all ? 15 : min(zf + 1, 15);
+        int z = k0;
+        for (int k = k0; k < k1; ++k) z += (ud[e] > r * (double)prm.t[k]) ? 1 : 0;
+        word = (word & ~(0xFu << (4 * e))) | ((uint32_t)z << (4 * e));
+      }
     }
   }
 
@@ -312,7 +390,7 @@ int launch_tq4_append(const Geom& g, const jf_kv_pool& pool, const Tq4Params& pr
 // ---------------------------------------------------------------------------
 // Decode: split kernel
 // ---------------------------------------------------------------------------
-constexpr int TQ_WARPS = 10;    // one CTA per SM (the centroid table takes 32 KB)
+constexpr int TQ_WARPS = 11;    // one CTA per SM (the centroid table takes 32 KB)
 constexpr int TQ_STAGES = 2;    // stages per warp
 
 template <int D>
@@ -326,15 +404,17 @@ struct Tq4Smem {
   static constexpr int LUT_BYTES = 256 * 32 * 4;
   static constexpr int NORM_OFF = LUT_OFF + LUT_BYTES;
   static constexpr int NORM_BYTES = NBUF * 2 * NORM_BUF;
-  static constexpr int Q_OFF = NORM_OFF + NORM_BYTES;
-  static constexpr int Q_BYTES = 8 * D * 4;      // rotated queries / combined output, fp32
-  static constexpr int BAR_OFF = Q_OFF + Q_BYTES;
+  // rotated queries (before the first copy is issued) and the combined output
+  // (after the last stage is consumed), fp32 [8][D], inside the stage rings
+  static constexpr int Q_BYTES = 8 * D * 4;
+  static constexpr int Q_OFF = CODES_BYTES - Q_BYTES;
+  static constexpr int BAR_OFF = NORM_OFF + NORM_BYTES;
   static constexpr int BAR_BYTES = NBUF * 8;
-  static constexpr int MISC_OFF = BAR_OFF + BAR_BYTES;   // plan (4 ints) + |q'| max
-  static constexpr int TOTAL = MISC_OFF + 32;
+  static constexpr int MISC_OFF = BAR_OFF + BAR_BYTES;   // plan (4 ints), per-warp |q'| max (8)
+  static constexpr int TOTAL = MISC_OFF + 64;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * NORM_BUF;
-  static_assert(TQ_WARPS * 8 * (D + 4) * 4 + TQ_WARPS * 8 * 3 * 4 + 64 <= CODES_BYTES,
-                "combine buffers must fit the stage rings");
+  static_assert(TQ_WARPS * 8 * (D + 4) * 4 + TQ_WARPS * 8 * 3 * 4 + 64 <= Q_OFF,
+                "combine buffers and the combined output must fit the stage rings");
   static_assert(TOTAL <= 227 * 1024, "shared memory");
 };
 
@@ -369,9 +449,11 @@ __device__ __forceinline__ float h2f(const uint8_t* p) {
   return __half2float(__ushort_as_half(*reinterpret_cast<const uint16_t*>(p)));
 }
 
-// One 32-position chunk.  FULL: every position valid; otherwise positions >=
-// nvalid get -inf logits and zero weights (their bytes are never trusted).
-template <int D, bool FULL>
+// One 32-position chunk; positions >= nvalid get -inf logits and zero weights
+// (their bytes are never trusted).  The masks are plain selects, so full and
+// partial chunks share one body (the body is large: one copy keeps it in the
+// instruction cache).
+template <int D>
 __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[D / 32][2][2],
                                           uint32_t kc, const uint8_t* kn, uint32_t lut_lane,
                                           const uint32_t (&koff)[D / 64], float cS, int r,
@@ -407,14 +489,10 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
     }
     const int ta = 16 * j + r, tb = ta + 8;
     const float na = h2f(kn + 2 * ta) * cS, nb = h2f(kn + 2 * tb) * cS;
-    sc[j][0] = acc[0] * na;
-    sc[j][1] = acc[1] * na;
-    sc[j][2] = acc[2] * nb;
-    sc[j][3] = acc[3] * nb;
-    if constexpr (!FULL) {
-      if (ta >= nvalid) { sc[j][0] = NEG_INF; sc[j][1] = NEG_INF; }
-      if (tb >= nvalid) { sc[j][2] = NEG_INF; sc[j][3] = NEG_INF; }
-    }
+    sc[j][0] = (ta < nvalid) ? acc[0] * na : NEG_INF;
+    sc[j][1] = (ta < nvalid) ? acc[1] * na : NEG_INF;
+    sc[j][2] = (tb < nvalid) ? acc[2] * nb : NEG_INF;
+    sc[j][3] = (tb < nvalid) ? acc[3] * nb : NEG_INF;
   }
 
   // ---- online softmax with a lazily moved reference maximum -------------
@@ -449,17 +527,10 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
   float p[NJ][4];
 #pragma unroll
   for (int j = 0; j < NJ; ++j) {
-    if constexpr (FULL) {
-      p[j][0] = fast_exp2(sc[j][0] - st.m0);
-      p[j][1] = fast_exp2(sc[j][1] - st.m1);
-      p[j][2] = fast_exp2(sc[j][2] - st.m0);
-      p[j][3] = fast_exp2(sc[j][3] - st.m1);
-    } else {
-      p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
-      p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
-      p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
-      p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
-    }
+    p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
+    p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
+    p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
+    p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
     st.l0 += p[j][0] + p[j][2];
     st.l1 += p[j][1] + p[j][3];
   }
@@ -468,11 +539,8 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
 #pragma unroll
   for (int j = 0; j < NJ; ++j) {
     const int ta = 16 * j + r, tb = ta + 8;
-    float wa = h2f(vn + 2 * ta) * 0.00390625f, wb = h2f(vn + 2 * tb) * 0.00390625f;
-    if constexpr (!FULL) {
-      if (ta >= nvalid) wa = 0.f;
-      if (tb >= nvalid) wb = 0.f;
-    }
+    const float wa = (ta < nvalid) ? h2f(vn + 2 * ta) * 0.00390625f : 0.f;
+    const float wb = (tb < nvalid) ? h2f(vn + 2 * tb) * 0.00390625f : 0.f;
     const uint32_t b0 = movm_t(pack_f16x2(wa * p[j][0], wa * p[j][1]));
     const uint32_t b1 = movm_t(pack_f16x2(wb * p[j][2], wb * p[j][3]));
 #pragma unroll
@@ -537,7 +605,6 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     const int b = i >> 5;
     lut_w[i] = pack_f16x2(prm.c[b & 15], prm.c[b >> 4]);
   }
-  if (threadIdx.x == 0) misc[4] = 0;
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
 
   int split, b, ctx, nch, cps, nsplit;
@@ -583,39 +650,37 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   auto chunk_of = [&](int it) { return c_begin + warp + it * TQ_WARPS; };
 
   // ---- rotated queries q' = H S_K q / sqrt(D) (rows >= G stay zero) -------
-  for (int i = threadIdx.x; i < 8 * D; i += blockDim.x) {
-    const int h = i / D, d = i % D;
-    float v = 0.f;
-    if (h < rows) {
-      v = __bfloat162float(__ushort_as_bfloat16(
-          a.q[((int64_t)b * a.HqL + kvh * a.G + h) * D + d]));
-      if ((prm.sk[d >> 5] >> (d & 31)) & 1u) v = -v;
+  // warp h < 8 transforms head row h with shuffles (E elements per lane)
+  constexpr int E = D / 32;
+  if (warp < 8) {
+    float x[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) x[e] = 0.f;
+    if (warp < rows) {
+      load_bf16<E>(a.q + ((int64_t)b * a.HqL + kvh * a.G + warp) * D + lane * E, x);
+      const uint32_t sb = prm.sk[(lane * E) >> 5] >> ((lane * E) & 31);
+#pragma unroll
+      for (int e = 0; e < E; ++e)
+        if ((sb >> e) & 1u) x[e] = -x[e];
     }
-    qbuf[i] = v;
-  }
-  __syncthreads();
-  for (int hs = 1; hs < D; hs <<= 1) {
-    for (int i = threadIdx.x; i < 8 * D / 2; i += blockDim.x) {
-      const int h = i / (D / 2), pr = i % (D / 2);
-      const int lo = (pr / hs) * 2 * hs + (pr % hs);
-      float* row = qbuf + h * D;
-      const float x = row[lo], y = row[lo + hs];
-      row[lo] = x + y;
-      row[lo + hs] = x - y;
-    }
-    __syncthreads();
-  }
-  // fp16 range: scale q' by 2^-qe so that max |q'| lies in [2^13, 2^14)
-  {
+    warp_fwht<float, E>(x, lane);
     float mx = 0.f;
-    for (int i = threadIdx.x; i < 8 * D; i += blockDim.x) mx = fmaxf(mx, fabsf(qbuf[i]));
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      qbuf[warp * D + lane * E + e] = x[e];
+      mx = fmaxf(mx, fabsf(x[e]));
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    if (lane == 0) atomicMax(&misc[4], __float_as_int(mx));
+    if (lane == 0) misc[8 + warp] = __float_as_int(mx);
   }
   __syncthreads();
+  // fp16 range: scale q' by 2^-qe so that max |q'| lies in [2^13, 2^14)
+  float qabs = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) qabs = fmaxf(qabs, __int_as_float(misc[8 + w]));
   const float qs0 = a.scale_log2 * rsqrtf((float)D);
-  const float qmax = __int_as_float(misc[4]) * fabsf(qs0);
+  const float qmax = qabs * fabsf(qs0);
   const int qe = (qmax > 0.f && qmax < INFINITY) ? ilogbf(qmax) - 13 : 0;
   const float qmul = qs0 * ldexpf(1.f, -qe);
   const float cS = ldexpf(1.f, qe);
@@ -629,6 +694,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
       bq[ch][s][0] = pack_f16x2(v.x * qmul, v.y * qmul);
       bq[ch][s][1] = pack_f16x2(v.z * qmul, v.w * qmul);
     }
+  __syncthreads();   // the query buffer lies in the stage rings the copies fill
 
   // ---- page ids and TMA producer (as in the affine decode) ---------------
   auto load_pages = [&](int blk) -> int {
@@ -684,7 +750,6 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   const uint32_t lut_lane = smem_u32(lut_w) + 4u * lane;
 
   int done = 0;
-#pragma unroll TQ_STAGES
   for (int it = 0; it < my_n; ++it) {
     const int s = it % TQ_STAGES;
     const uint32_t par = (it / TQ_STAGES) & 1;
@@ -697,10 +762,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     const int tokbase = chunk_of(it) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * TQ_STAGES + s) * 2 * L::CODE_BUF);
     const uint8_t* kn = norms + (warp * TQ_STAGES + s) * 2 * L::NORM_BUF;
-    if (ok && tokbase + DTOK <= ctx)
-      tq4_chunk<D, true>(st, bq, kc, kn, lut_lane, koff, cS, r, DTOK);
-    else
-      tq4_chunk<D, false>(st, bq, kc, kn, lut_lane, koff, cS, r, ok ? ctx - tokbase : 0);
+    tq4_chunk<D>(st, bq, kc, kn, lut_lane, koff, cS, r, ok ? min(ctx - tokbase, DTOK) : 0);
     __syncwarp();
     if (it + TQ_STAGES < my_n) {
       fence_proxy_async_smem();
@@ -780,40 +842,38 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     *reinterpret_cast<float4*>(qbuf + h * D + d) = acc;
   }
   __syncthreads();
-  // inverse rotation: o = S_V H (2^8 acc) / sqrt(D)
-  for (int hs = 1; hs < D; hs <<= 1) {
-    for (int i = threadIdx.x; i < rows * (D / 2); i += blockDim.x) {
-      const int h = i / (D / 2), pr = i % (D / 2);
-      const int lo = (pr / hs) * 2 * hs + (pr % hs);
-      float* row = qbuf + h * D;
-      const float x = row[lo], y = row[lo + hs];
-      row[lo] = x + y;
-      row[lo + hs] = x - y;
-    }
-    __syncthreads();
-  }
-  const float osc = 256.f * rsqrtf((float)D);
-  for (int idx = threadIdx.x; idx < rows * (D / 4); idx += blockDim.x) {
-    const int h = idx / (D / 4), d = 4 * (idx % (D / 4));
-    float4 v = *reinterpret_cast<const float4*>(qbuf + h * D + d);
-    const uint32_t sb = prm.sv[d >> 5] >> (d & 31);
-    v.x *= (sb & 1u) ? -osc : osc;
-    v.y *= (sb & 2u) ? -osc : osc;
-    v.z *= (sb & 4u) ? -osc : osc;
-    v.w *= (sb & 8u) ? -osc : osc;
+  // inverse rotation o = S_V H (2^8 acc) / sqrt(D): warp h < rows takes head h
+  if (warp < rows) {
+    const int h = warp;
+    float x[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) x[e] = qbuf[h * D + lane * E + e];
+    warp_fwht<float, E>(x, lane);
+    const float osc = 256.f * rsqrtf((float)D);
+    const uint32_t sb = prm.sv[(lane * E) >> 5] >> ((lane * E) & 31);
+#pragma unroll
+    for (int e = 0; e < E; ++e) x[e] *= ((sb >> e) & 1u) ? -osc : osc;
     const int fr = kvh * a.G + h;
+    const int d0 = lane * E;
     if (direct) {
-      uint2 o;
-      o.x = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
-            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.y)) << 16);
-      o.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
-            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(v.w)) << 16);
-      *reinterpret_cast<uint2*>(a.out + ((int64_t)b * a.HqL + fr) * D + d) = o;
+      uint32_t w[E / 2];
+#pragma unroll
+      for (int e = 0; e < E / 2; ++e)
+        w[e] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(x[2 * e])) |
+               ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(x[2 * e + 1])) << 16);
+      uint16_t* dst = a.out + ((int64_t)b * a.HqL + fr) * D + d0;
+      if constexpr (E == 8)
+        *reinterpret_cast<uint4*>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+      else
+        *reinterpret_cast<uint2*>(dst) = make_uint2(w[0], w[1]);
     } else {
       const int64_t row = a.balanced ? (int64_t)blockIdx.x * a.HqL + fr
                                      : ((int64_t)b * a.HqL + fr) * a.num_splits + blockIdx.x;
-      *reinterpret_cast<float4*>(a.part_o + row * D + d) = v;
-      if (d == 0) {
+      float* dst = a.part_o + row * D + d0;
+#pragma unroll
+      for (int e = 0; e < E; e += 4)
+        *reinterpret_cast<float4*>(dst + e) = make_float4(x[e], x[e + 1], x[e + 2], x[e + 3]);
+      if (lane == 0) {
         a.part_ml[row * 2 + 0] = shl[h * 2 + 0];
         a.part_ml[row * 2 + 1] = shl[h * 2 + 1];
       }

@@ -12,6 +12,7 @@ struct Tq4Params {
   float tq[15];     // fp32(sqrt(d) t_k): thresholds in units of rho (fast path)
   uint32_t sk[8];   // sign bits of S for K: bit j set <=> S_jj = -1
   uint32_t sv[8];   // ... for V
+  int32_t exact_all;   // thresholds closer than 2^-12 rho apart: every index takes the fp64 path
 };
 
 }  // namespace jfkv

@@ -132,6 +132,31 @@ def test_tq4_append_many_rows_exercises_both_decision_paths():
     assert np.array_equal(pool.data.cpu().numpy(), ref)
 
 
+def test_tq4_append_close_thresholds_take_the_exact_path_everywhere():
+    """A codebook with two thresholds closer than the fast path's margins:
+    every index is decided in fp64, still bit-exact against the oracle."""
+    D, Hkv = 256, 2
+    c = OQ.codebook(D).copy()
+    c[8] = np.float32(c[7] + np.float32(2e-7))            # c_7, c_8, c_9 within 4e-7:
+    c[9] = np.float32(c[8] + np.float32(2e-7))            # t_7 and t_8 nearly equal
+    assert np.all(np.diff(c) > 0)
+    assert np.diff(np.float32(16) * OQ.thresholds(c)).min() < 2 ** -12
+    sk, sv = signs(D)
+    case = make_case(21, 2 * Hkv, Hkv, D, 64, [300], num_pages=6)
+    lay = OQ.Tq4Layout(Hkv, 64, D, OQ.Codec(D, c, sk.astype(np.float64), sv.astype(np.float64)))
+    ref = OQ.new_pool(lay, case.num_pages)
+    OQ.append(ref, lay, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
+              bits(case.k), bits(case.v))
+    pool = jf.KVPool.allocate(case.num_pages, 64, Hkv, D, device=DEV, format=jf.JF_FMT_TQ4,
+                              codec=jf.Tq4Codec(D, sk, sv, centroids=c))
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, case.page_table.to(DEV), case.req.to(DEV), case.pos.to(DEV),
+                             case.k.to(DEV), case.v.to(DEV), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    assert np.array_equal(pool.data.cpu().numpy(), ref)
+
+
 def test_tq4_append_flags_bad_rows_and_skips_them():
     case = make_case(13, 8, 2, 128, 64, [100], num_pages=3)
     pool = gpu_pool(case, fill=0x77)
