@@ -344,7 +344,7 @@ def _event_time(fn, reps, stream):
     return e0.elapsed_time(e1) / reps
 
 
-ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify", "tq4")
+ROW_GROUPS = ("tiny", "prompt", "two_request", "mixed", "verify", "tq4", "prefill_batch")
 
 
 def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None, tq4_copies=8):
@@ -358,7 +358,52 @@ def bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None, tq4_copies
             out["verify_256k"] = _bench_verify(jf, dev, stream)
         if only is None or only == "tq4":
             out["tq4_256k"] = _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=tq4_copies)
+        if only is None or only == "prefill_batch":
+            out["prefill_batch"] = _bench_prefill_batch(jf, dev, stream, peak_tf)
         return out
+
+
+def _bench_prefill_batch(jf, dev, stream, peak_tf):
+    """Prefill chunks of 8 requests (24/4/256, P 256, prefixes 4K..32K of
+    32,768-position caches) in one jf_prefill_batch_attn launch against one
+    jf_prefill_chunk_attn launch per request: 64-query chunks (the cadence the
+    scheduler uses beside active decoders, Sec. 3.3) and 512-query chunks."""
+    Hq, Hkv, D, P, B, ctx = 24, 4, 256, 256, 8, 32768
+    g = torch.Generator(device=dev)
+    g.manual_seed(31)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    npg = B * ctx // P
+    pool = jf.KVPool.allocate(npg, P, Hkv, D, device=dev, fill=None)
+    pt = torch.randperm(npg, device=dev, generator=g).to(torch.int32).view(B, ctx // P)
+    for b in range(B):
+        kk = torch.randn(ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        vv = torch.randn(ctx, Hkv, D, generator=g, device=dev).to(torch.bfloat16)
+        jf.jf_kv_quantize_append(pool, pt, torch.full((ctx,), b, dtype=torch.int32, device=dev),
+                                 torch.arange(ctx, dtype=torch.int32, device=dev), kk, vv, err,
+                                 stream=stream)
+    ws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=dev)
+    scale = 1 / math.sqrt(D)
+    res = {}
+    for C in (64, 512):
+        starts = [4096 * (b + 1) - C for b in range(B)]
+        q = torch.randn(B * C, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        o = torch.empty_like(q)
+        tb = _event_time(lambda: jf.jf_prefill_batch_attn(pool, pt, starts, [C] * B, q, scale,
+                                                          True, o, ws, stream=stream), 20, stream)
+
+        def singles():
+            for b in range(B):
+                jf.jf_prefill_chunk_attn(pool, pt[b], q[b * C:(b + 1) * C], starts[b], scale,
+                                         True, o[b * C:(b + 1) * C], ws, stream=stream)
+        ts = _event_time(singles, 20, stream)
+        stream.synchronize()
+        assert jf.workspace_status(ws) == 0 and int(err.item()) == 0
+        flops = sum(4 * Hq * D * (C * s0 + C * (C + 1) // 2) for s0 in starts)
+        res[f"chunk_{C}"] = {"batched_us": tb * 1e3, "separate_us": ts * 1e3,
+                             "speedup": ts / tb, "TFLOPs_batched": flops / (tb / 1e3) / 1e12,
+                             "frac_tensor": flops / (tb / 1e3) / 1e12 / peak_tf}
+    del pool
+    return res
 
 
 def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):

@@ -269,6 +269,41 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
                           size_t workspace_bytes, void* stream);
 
 /*
+ * Prefill chunks of several requests in one launch (Sec. 3.3: the scheduler
+ * advances admitted prompts in bounded chunks between decode opportunities;
+ * Sec. 3.1 / Eq. 5 for the attention).  Request b's chunk_len[b] queries at
+ * absolute positions q_start[b] + i attend positions [0, q_start[b] + i]
+ * (causal != 0) or [0, q_start[b] + chunk_len[b]) of its own cache, whose
+ * pages are page_table[b * pt_stride ..]; every chunk's rows must already be
+ * appended.  Each output equals jf_prefill_chunk_attn on that request alone.
+ *   page_table   int32 [batch, pt_stride] (device)
+ *   q_start, chunk_len  int32 [batch] on the HOST (scheduling metadata the
+ *                caller already holds); q_start[b] + chunk_len[b] <=
+ *                pt_stride * P; a zero chunk_len is skipped
+ *   q, out       bf16 [sum_b chunk_len[b], Hq, D]; request b's rows start at
+ *                row sum_{b' < b} chunk_len[b']
+ *   batch        1 .. JF_PREFILL_MAX_BATCH (JF_ERR_UNSUPPORTED above)
+ *   workspace    >= jf_prefill_workspace_bytes(); int32 status word.
+ * The longest request's query tiles are scheduled first.
+ */
+#define JF_PREFILL_MAX_BATCH 64
+
+int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                          int32_t batch, const int32_t* q_start, const int32_t* chunk_len,
+                          const void* q, int32_t num_q_heads, float softmax_scale, int32_t causal,
+                          void* out, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Page reservation of one unshared request (Eq. 7):
+ *   R = ceil((prompt_len + min(output_len, g_out)) / page_size)
+ * page equivalents, g_out the guaranteed output (8,192 in the paper, page
+ * size 256).  Host only.  Returns -1 for a negative length or guarantee, a
+ * page size below 1, or a sum that overflows int64.
+ */
+int64_t jf_reservation_pages(int64_t prompt_len, int64_t output_len, int64_t g_out,
+                             int32_t page_size);
+
+/*
  * Page-gather checkpoint (Sec. 3.4: read the request's page runs in place and
  * emit one packed stream).  Either format.  dst[k * page_bytes .. (k+1) * page_bytes) =
  * page record page_table_row[k] for k < num_pages, tail bytes included.

@@ -18,6 +18,7 @@ tq4         TQ4 format (Sec. 3.1 Eq. 4; App. A.1 Table 3): Lloyd-Max
             codebook, Hadamard rotation with random signs, exact index
             decision, FP16 norms, page layout, append and reconstruction.
 checkpoint  page-gather checkpoint and its inverse (restore scatter).
+reservation the page reservation rule of Eq. 7.
 
 Parity status: every function here is pinned by the ``-m "not gpu"`` tests in
 ``tests/test_oracle_*.py`` (closed forms, invariants, brute force on tiny
@@ -25,4 +26,4 @@ inputs, library routines on special cases, hand-derived fixtures in
 ``tests/golden/``).  The TQ4 codebook is pinned to the continuous-density
 Lloyd iteration to within the grid's resolution (about 1e-4), not bit for bit.
 """
-from . import affine4, attention, checkpoint, tq4  # noqa: F401
+from . import affine4, attention, checkpoint, reservation, tq4  # noqa: F401

@@ -32,7 +32,7 @@ EXPORTS = [
     "jf_kv_quantize_append", "jf_paged_decode_attn", "jf_prefill_chunk_attn",
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
     "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
-    "jf_kv_page_bytes_fmt", "jf_tq4_codebook",
+    "jf_kv_page_bytes_fmt", "jf_tq4_codebook", "jf_prefill_batch_attn", "jf_reservation_pages",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -87,6 +87,9 @@ def lib() -> ctypes.CDLL:
                                                     SZ, I32, P]),
             "jf_kv_page_bytes_fmt": (SZ, [I32, I32, I32, I32]),
             "jf_tq4_codebook": (ctypes.c_int, [I32, ctypes.POINTER(ctypes.c_float)]),
+            "jf_prefill_batch_attn": (ctypes.c_int, [PP, P, I32, I32, P, P, P, I32, F32, I32, P,
+                                                     P, SZ, P]),
+            "jf_reservation_pages": (I64, [I64, I64, I64, I32]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -380,6 +383,44 @@ def jf_prefill_chunk_attn(pool: KVPool, page_table_row: torch.Tensor, q: torch.T
                                       _ptr(out), _ptr(workspace), workspace.numel(),
                                       _stream(stream))
     _check("jf_prefill_chunk_attn", st)
+
+
+JF_PREFILL_MAX_BATCH = 64
+
+
+def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk_len,
+                          q: torch.Tensor, softmax_scale: float, causal: bool, out: torch.Tensor,
+                          workspace: torch.Tensor, stream=None) -> None:
+    """Prefill chunks of several requests in one launch.  ``q`` / ``out`` are
+    the requests' chunks concatenated, [sum(chunk_len), Hq, D]; ``q_start`` and
+    ``chunk_len`` are host sequences (one entry per page-table row)."""
+    _need(page_table, torch.int32, "page_table")
+    _need(q, torch.bfloat16, "q")
+    _need(out, torch.bfloat16, "out")
+    _need(workspace, torch.uint8, "workspace")
+    B = page_table.shape[0]
+    if len(q_start) != B or len(chunk_len) != B:
+        raise ValueError("one q_start and chunk_len per page-table row")
+    N, Hq, D = q.shape
+    if out.shape != q.shape or D != pool.head_dim or N != sum(int(c) for c in chunk_len):
+        raise ValueError("shape mismatch")
+    qs = (ctypes.c_int32 * B)(*[int(x) for x in q_start])
+    cl = (ctypes.c_int32 * B)(*[int(x) for x in chunk_len])
+    st = lib().jf_prefill_batch_attn(ctypes.byref(pool.c_struct()), _ptr(page_table),
+                                      page_table.shape[1], B, qs, cl, _ptr(q), Hq,
+                                      float(softmax_scale), int(bool(causal)), _ptr(out),
+                                      _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("jf_prefill_batch_attn", st)
+
+
+def jf_reservation_pages(prompt_len: int, output_len: int, g_out: int = 8192,
+                         page_size: int = 256) -> int:
+    """Eq. 7: ceil((prompt_len + min(output_len, g_out)) / page_size)."""
+    r = int(lib().jf_reservation_pages(int(prompt_len), int(output_len), int(g_out),
+                                       int(page_size)))
+    if r < 0:
+        raise ValueError("invalid reservation arguments")
+    return r
 
 
 def jf_kv_checkpoint(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,

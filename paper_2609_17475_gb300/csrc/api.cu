@@ -30,6 +30,9 @@ int decode_box_rows();
 int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
                    const void*, int32_t, int32_t, int32_t, float, int32_t, void*, void*,
                    cudaStream_t);
+int launch_prefill_batch(const Geom&, const jf_kv_pool&, const int32_t* const*, const int32_t*,
+                         const int32_t*, const void*, const int64_t*, int32_t, int32_t, float,
+                         int32_t, void*, void*, cudaStream_t);
 }  // namespace jfkv
 
 using namespace jfkv;
@@ -257,6 +260,47 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
   CUtensorMap tmap{};
   return launch_prefill(g, *pool, tmap, page_table_row, q, q_start, chunk_len, num_q_heads,
                         softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
+}
+
+int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
+                          int32_t batch, const int32_t* q_start, const int32_t* chunk_len,
+                          const void* q, int32_t num_q_heads, float softmax_scale, int32_t causal,
+                          void* out, void* workspace, size_t workspace_bytes, void* stream) {
+  int st = check_pool(pool);
+  if (st) return st;
+  if (batch < 1 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
+  if (batch > JF_PREFILL_MAX_BATCH) return JF_ERR_UNSUPPORTED;
+  if (!page_table || !q_start || !chunk_len || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
+  if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
+  if (num_q_heads / pool->num_kv_heads > 128) return JF_ERR_UNSUPPORTED;
+  if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
+  if (workspace_bytes < jf_prefill_workspace_bytes()) return JF_ERR_WORKSPACE_TOO_SMALL;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 16)) return JF_ERR_INVALID_ARG;
+  const int32_t* rows[JF_PREFILL_MAX_BATCH];
+  int64_t row0[JF_PREFILL_MAX_BATCH];
+  int64_t acc = 0;
+  for (int b = 0; b < batch; ++b) {
+    if (q_start[b] < 0 || chunk_len[b] < 0) return JF_ERR_INVALID_ARG;
+    if ((int64_t)q_start[b] + chunk_len[b] > (int64_t)pt_stride * pool->page_size)
+      return JF_ERR_INVALID_ARG;   // the chunk must fit the request's page-table row
+    rows[b] = page_table + (int64_t)b * pt_stride;
+    row0[b] = acc;
+    acc += chunk_len[b];
+  }
+  if (acc == 0) return JF_OK;
+  if (acc > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
+  const Geom g = make_geom(*pool);
+  return launch_prefill_batch(g, *pool, rows, q_start, chunk_len, q, row0, batch, num_q_heads,
+                              softmax_scale, causal, out, workspace,
+                              static_cast<cudaStream_t>(stream));
+}
+
+int64_t jf_reservation_pages(int64_t prompt_len, int64_t output_len, int64_t g_out,
+                             int32_t page_size) {
+  if (prompt_len < 0 || output_len < 0 || g_out < 0 || page_size < 1) return -1;
+  const int64_t out = output_len < g_out ? output_len : g_out;
+  if (prompt_len > INT64_MAX - out - page_size) return -1;
+  return (prompt_len + out + page_size - 1) / page_size;
 }
 
 int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,

@@ -7,7 +7,9 @@
 // fused into the attention kernel as fp16 shared-memory tiles that feed
 // tcgen05.mma directly.
 //
-// CTA = (tile of QPC = 128 / G queries, KV head); its 128 MMA rows are the
+// CTA = (tile of QPC = 128 / G queries of one request, KV head); one launch
+// may cover the chunks of several requests (each with its own page-table row,
+// prefix length and queries).  Its 128 MMA rows are the
 // (query, head) pairs r = i * G + j of the G query heads that share the KV
 // head, so every dequantized K/V tile is reused by all of them.  Two CTAs on
 // two SMs form a pair (a cluster of 2, tcgen05 cta_group::2): the pair runs
@@ -54,6 +56,17 @@ constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
 constexpr int PF_KVBUF = 4;     // K/V half-tile buffers in shared memory
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
 
+// One request's chunk in a launch: its query tiles are CTAs tile0 ..
+// tile0 + n_tiles2 - 1 (n_tiles2 even, so a CTA pair never spans requests).
+struct PfReq {
+  const int32_t* pt;    // its page-table row
+  const uint16_t* q;    // its chunk's queries [C, Hq, D]
+  uint16_t* out;        // [C, Hq, D]
+  int32_t q_start, C, tile0, n_tiles2;
+};
+
+constexpr int PF_MAX_REQ = 64;   // requests per launch
+
 struct PrefillArgs {
   const uint8_t* pool;
   int64_t num_pages;
@@ -62,13 +75,11 @@ struct PrefillArgs {
   int64_t sb_base;
   int64_t sb_region;
   int32_t P, Hkv, Hq, G, QPC;
-  const int32_t* pt;
-  const uint16_t* q;
-  uint16_t* out;
-  int32_t q_start, C, causal;
+  int32_t causal;
   float scale_log2;
   int32_t* status;
-  int32_t n_tiles2;   // query tiles, rounded up to pairs
+  int32_t nreq;
+  PfReq req[PF_MAX_REQ];
 };
 
 // Each CTA of a pair holds half of every K/V tile: K rows 32 r .. 32 r + 31
@@ -124,7 +135,7 @@ __device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2)
 
 template <int D>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PF_THREADS, 1)
-prefill_kernel(const PrefillArgs a) {
+prefill_kernel(const __grid_constant__ PrefillArgs a) {
   using L = PfSmem<D>;
   constexpr int NKB = D / 64;           // 64-wide d blocks
   constexpr int UPI = (D == 256) ? 2 : 1;   // 16-byte code units per dequant item
@@ -151,19 +162,27 @@ prefill_kernel(const PrefillArgs a) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = tc::cluster_rank();
+  // this CTA's request (tile ranges ascend with the request index)
+  int ri = 0;
+  for (int i = 1; i < a.nreq; ++i)
+    if ((int)blockIdx.x >= a.req[i].tile0) ri = i;
+  const PfReq& rq = a.req[ri];
+  const int32_t* const pt = rq.pt;
+  const int q_start = rq.q_start, C = rq.C;
+  const int bx = (int)blockIdx.x - rq.tile0;
   // query tile of this CTA and of its partner: latest (longest) tiles first
-  const int qt = a.n_tiles2 - 1 - (int)blockIdx.x;
-  const int qt_partner = a.n_tiles2 - 1 - (int)(blockIdx.x ^ 1u);
+  const int qt = rq.n_tiles2 - 1 - bx;
+  const int qt_partner = rq.n_tiles2 - 1 - (bx ^ 1);
   const int kvh = blockIdx.y;
   const int q0 = qt * a.QPC;
-  const int nq = max(0, min(a.QPC, a.C - q0));
+  const int nq = max(0, min(a.QPC, C - q0));
   const int rows = nq * a.G;
-  const int total = a.q_start + a.C;
+  const int total = q_start + C;
   // positions a query tile attends (0 for the padding tile of an odd count)
   auto kmax_of = [&](int t) {
     const int first = t * a.QPC;
-    const int n = max(0, min(a.QPC, a.C - first));
-    return n == 0 ? 0 : (a.causal ? a.q_start + first + n : total);
+    const int n = max(0, min(a.QPC, C - first));
+    return n == 0 ? 0 : (a.causal ? q_start + first + n : total);
   };
   const int kmax = kmax_of(qt);
   const int kmax_pair = max(kmax, kmax_of(qt_partner));
@@ -199,7 +218,7 @@ prefill_kernel(const PrefillArgs a) {
   const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
   int qe = 0;                                  // per-row power of two kept out of fp16
   if (warp > PF_DQ_WARPS) {
-    const uint16_t* qrow = a.q + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
+    const uint16_t* qrow = rq.q + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
     float qmax = 0.f;
     if (row_ok) {
       for (int c8 = 0; c8 < D / 8; ++c8) {
@@ -296,7 +315,7 @@ prefill_kernel(const PrefillArgs a) {
     };
     // page id of tile j (P >= 64, so a tile lies in one page); it is loaded a
     // step before its tile's code loads need it
-    auto page_of = [&](int j) -> int { return j < ntiles ? __ldg(a.pt + (j * PF_BN) / a.P) : -1; };
+    auto page_of = [&](int j) -> int { return j < ntiles ? __ldg(pt + (j * PF_BN) / a.P) : -1; };
     auto load_tile = [&](int j, int page, Tile& x) {
       const int key0 = j * PF_BN;
       const bool pok = page >= 0 && page < a.num_pages;
@@ -359,7 +378,7 @@ prefill_kernel(const PrefillArgs a) {
     // Rows past the chunk (padding) see every position: their Q rows are zero
     // and their outputs are never stored, and keeping them unmasked keeps the
     // warp on the same (mask-free) path as its real rows.
-    const int limit = (row_ok && a.causal) ? a.q_start + q0 + qi : kmax_pair - 1;
+    const int limit = (row_ok && a.causal) ? q_start + q0 + qi : kmax_pair - 1;
     const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
@@ -442,7 +461,7 @@ prefill_kernel(const PrefillArgs a) {
                                 ((ntiles - 1) / PF_KVBUF) & 1)) {
       tc::fence_after();
       const float inv = l > 0.f ? 1.f / l : 0.f;
-      uint16_t* orow = a.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
+      uint16_t* orow = rq.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
 #pragma unroll 1
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t o[32];
@@ -481,10 +500,14 @@ prefill_kernel(const PrefillArgs a) {
   }
 }
 
-int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
-                   const int32_t* page_table_row, const void* q, int32_t q_start,
-                   int32_t chunk_len, int32_t Hq, float softmax_scale, int32_t causal, void* out,
-                   void* workspace, cudaStream_t stream) {
+// One launch over the chunks of `nreq` requests (nreq <= PF_MAX_REQ); requests
+// with an empty chunk get no CTAs.  The request with the most attended
+// positions goes first, so the longest CTA pairs start earliest.
+int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* const* pt_rows,
+                         const int32_t* q_start, const int32_t* chunk_len, const void* q,
+                         const int64_t* q_row0, int32_t nreq, int32_t Hq, float softmax_scale,
+                         int32_t causal, void* out, void* workspace, cudaStream_t stream) {
+  if (nreq < 1 || nreq > PF_MAX_REQ) return JF_ERR_UNSUPPORTED;
   PrefillArgs a;
   a.pool = static_cast<const uint8_t*>(pool.base);
   a.num_pages = g.num_pages;
@@ -498,18 +521,39 @@ int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
   a.G = Hq / g.Hkv;
   if (a.G > PF_BM) return JF_ERR_UNSUPPORTED;
   a.QPC = PF_BM / a.G;
-  a.pt = page_table_row;
-  a.q = static_cast<const uint16_t*>(q);
-  a.out = static_cast<uint16_t*>(out);
-  a.q_start = q_start;
-  a.C = chunk_len;
   a.causal = causal ? 1 : 0;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.status = static_cast<int32_t*>(workspace);
-  const int n_qtiles = (chunk_len + a.QPC - 1) / a.QPC;
-  a.n_tiles2 = (n_qtiles + 1) & ~1;   // CTA pairs
-  if (g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
-  dim3 grid((unsigned)a.n_tiles2, (unsigned)g.Hkv);
+  int order[PF_MAX_REQ];
+  int n = 0;
+  for (int b = 0; b < nreq; ++b)
+    if (chunk_len[b] > 0) order[n++] = b;
+  if (n == 0) return JF_OK;
+  auto span = [&](int b) { return (int64_t)q_start[b] + chunk_len[b]; };
+  for (int i = 1; i < n; ++i)   // longest first (insertion sort, n <= 64)
+    for (int j = i; j > 0 && span(order[j]) > span(order[j - 1]); --j) {
+      const int t = order[j];
+      order[j] = order[j - 1];
+      order[j - 1] = t;
+    }
+  const size_t row_elems = (size_t)Hq * g.D;
+  int64_t tiles = 0;
+  for (int i = 0; i < n; ++i) {
+    const int b = order[i];
+    PfReq& r = a.req[i];
+    r.pt = pt_rows[b];
+    r.q = static_cast<const uint16_t*>(q) + (size_t)q_row0[b] * row_elems;
+    r.out = static_cast<uint16_t*>(out) + (size_t)q_row0[b] * row_elems;
+    r.q_start = q_start[b];
+    r.C = chunk_len[b];
+    r.tile0 = (int32_t)tiles;
+    const int n_qtiles = (chunk_len[b] + a.QPC - 1) / a.QPC;
+    r.n_tiles2 = (n_qtiles + 1) & ~1;   // CTA pairs
+    tiles += r.n_tiles2;
+  }
+  a.nreq = n;
+  if (tiles > 0x7FFFFFFF || g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
+  dim3 grid((unsigned)tiles, (unsigned)g.Hkv);
   if (g.D == 256) {
     static bool attr = false;
     if (!attr) {
@@ -530,6 +574,15 @@ int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
     prefill_kernel<128><<<grid, PF_THREADS, PfSmem<128>::TOTAL, stream>>>(a);
   }
   return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
+}
+
+int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
+                   const int32_t* page_table_row, const void* q, int32_t q_start,
+                   int32_t chunk_len, int32_t Hq, float softmax_scale, int32_t causal, void* out,
+                   void* workspace, cudaStream_t stream) {
+  const int64_t row0 = 0;
+  return launch_prefill_batch(g, pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1, Hq,
+                              softmax_scale, causal, out, workspace, stream);
 }
 
 }  // namespace jfkv

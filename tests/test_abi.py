@@ -166,3 +166,19 @@ def test_tq4_bad_codecs_and_unsupported_entry_points():
     pb = B.jf_kv_page_bytes_fmt(B.JF_FMT_TQ4, 2, 256, 128)
     assert L.jf_kv_checkpoint(ctypes.byref(p), FAKE, 3, FAKE, 3 * pb - 1, None,
                               None) == B.JF_ERR_INVALID_ARG
+
+
+def test_prefill_batch_rejects_bad_arguments():
+    L = B.lib()
+    p = _pool()
+    I = ctypes.c_int32
+    qs = (I * 2)(0, 100)
+    cl = (I * 2)(16, 16)
+    call = lambda batch=2, stride=4, q_start=qs, clen=cl, wsb=256: L.jf_prefill_batch_attn(
+        ctypes.byref(p), FAKE, stride, batch, q_start, clen, FAKE, 8, 0.1, 1, FAKE, FAKE, wsb, None)
+    assert call(batch=0) == B.JF_ERR_INVALID_ARG
+    assert call(batch=65, q_start=(I * 65)(), clen=(I * 65)()) == B.JF_ERR_UNSUPPORTED
+    assert call(wsb=0) == B.JF_ERR_WORKSPACE_TOO_SMALL
+    assert call(stride=1, q_start=(I * 2)(0, 250), clen=(I * 2)(4, 16)) == B.JF_ERR_INVALID_ARG
+    assert call(q_start=(I * 2)(-1, 0)) == B.JF_ERR_INVALID_ARG
+    assert call(clen=(I * 2)(0, 0)) == B.JF_OK                     # nothing to do

@@ -471,3 +471,42 @@ def test_prefill_poison_pages_never_leak():
     out = gpu_prefill(case, pool, q, 200, True, 0.1)
     ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q), 200, 0.1)
     assert_attention_close(out, ref)
+
+
+# --------------------------------------------------------------------------
+# prefill chunks of several requests in one launch
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hq,Hkv,D,P,spans,causal", [
+    # (q_start, chunk_len) per request
+    (24, 4, 256, 256, [(1000, 64), (0, 256), (4000, 130), (300, 0), (17, 1)], True),
+    (8, 2, 128, 64, [(70, 200), (0, 21), (500, 77)], True),
+    (24, 4, 256, 128, [(200, 64), (900, 33)], False),
+])
+def test_prefill_batch_matches_oracle_and_single_calls(Hq, Hkv, D, P, spans, causal):
+    from paper_2609_17475_gb300 import synth
+    totals = [qs + c for qs, c in spans]
+    case = make_case(600 + sum(totals), Hq, Hkv, D, P, totals, outliers=True)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    C = [c for _, c in spans]
+    qs = [q for q, _ in spans]
+    q = synth.normal_bf16(synth.generator(601), (sum(C), Hq, D))
+    scale = 1 / math.sqrt(D)
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=DEV)
+    jf.jf_prefill_batch_attn(pool, case.page_table.to(DEV), qs, C, q.to(DEV), scale, causal,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    row = 0
+    for b, (q0, c) in enumerate(spans):
+        if c:
+            ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[b].numpy(),
+                                   bits(q[row:row + c]), q0, scale, causal=causal)
+            assert_attention_close(out[row:row + c], ref)
+            one = torch.empty(c, Hq, D, dtype=torch.bfloat16, device=DEV)
+            jf.jf_prefill_chunk_attn(pool, case.page_table[b].to(DEV), q[row:row + c].to(DEV),
+                                     q0, scale, causal, one, ws)
+            torch.cuda.synchronize()
+            assert torch.equal(one, out[row:row + c])   # same tiles, same arithmetic
+        row += c
