@@ -384,12 +384,32 @@ def _bench_prefill_batch(jf, dev, stream, peak_tf):
     ws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=dev)
     scale = 1 / math.sqrt(D)
     res = {}
+    # one request: a 64-query chunk after a 32,704-position prefix, whole history
+    # per CTA pair vs the history split across CTA pairs and merged
+    q1 = torch.randn(64, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o1 = torch.empty_like(q1)
+    s1 = jf.default_prefill_splits([ctx - 64], [64], Hq, Hkv)
+    w1 = jf.prefill_batch_workspace(64, Hq, D, s1, device=dev)
+    t_one = _event_time(lambda: jf.jf_prefill_chunk_attn(pool, pt[0], q1, ctx - 64, scale, True,
+                                                         o1, ws, stream=stream), 20, stream)
+    t_one_s = _event_time(lambda: jf.jf_prefill_batch_attn(pool, pt[:1], [ctx - 64], [64], q1,
+                                                           scale, True, o1, w1, num_splits=s1,
+                                                           stream=stream), 20, stream)
+    fl1 = 4 * Hq * D * (64 * (ctx - 64) + 64 * 65 // 2)
+    res["one_chunk_64_at_32704"] = {"whole_history_us": t_one * 1e3, "splits": s1,
+                                    "split_us": t_one_s * 1e3, "speedup": t_one / t_one_s,
+                                    "TFLOPs_split": fl1 / (t_one_s / 1e3) / 1e12}
     for C in (64, 512):
         starts = [4096 * (b + 1) - C for b in range(B)]
         q = torch.randn(B * C, Hq, D, generator=g, device=dev).to(torch.bfloat16)
         o = torch.empty_like(q)
         tb = _event_time(lambda: jf.jf_prefill_batch_attn(pool, pt, starts, [C] * B, q, scale,
                                                           True, o, ws, stream=stream), 20, stream)
+        sp = jf.default_prefill_splits(starts, [C] * B, Hq, Hkv)
+        wsp = jf.prefill_batch_workspace(B * C, Hq, D, sp, device=dev)
+        tbs = _event_time(lambda: jf.jf_prefill_batch_attn(pool, pt, starts, [C] * B, q, scale,
+                                                           True, o, wsp, num_splits=sp,
+                                                           stream=stream), 20, stream)
 
         def singles():
             for b in range(B):
@@ -397,11 +417,14 @@ def _bench_prefill_batch(jf, dev, stream, peak_tf):
                                          True, o[b * C:(b + 1) * C], ws, stream=stream)
         ts = _event_time(singles, 20, stream)
         stream.synchronize()
-        assert jf.workspace_status(ws) == 0 and int(err.item()) == 0
+        assert jf.workspace_status(ws) == 0 and jf.workspace_status(wsp) == 0
+        assert int(err.item()) == 0
         flops = sum(4 * Hq * D * (C * s0 + C * (C + 1) // 2) for s0 in starts)
         res[f"chunk_{C}"] = {"batched_us": tb * 1e3, "separate_us": ts * 1e3,
                              "speedup": ts / tb, "TFLOPs_batched": flops / (tb / 1e3) / 1e12,
-                             "frac_tensor": flops / (tb / 1e3) / 1e12 / peak_tf}
+                             "frac_tensor": flops / (tb / 1e3) / 1e12 / peak_tf,
+                             "splits": sp, "batched_split_us": tbs * 1e3,
+                             "TFLOPs_batched_split": flops / (tbs / 1e3) / 1e12}
     del pool
     return res
 

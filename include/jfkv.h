@@ -283,15 +283,29 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
  *   q, out       bf16 [sum_b chunk_len[b], Hq, D]; request b's rows start at
  *                row sum_{b' < b} chunk_len[b']
  *   batch        1 .. JF_PREFILL_MAX_BATCH (JF_ERR_UNSUPPORTED above)
- *   workspace    >= jf_prefill_workspace_bytes(); int32 status word.
+ *   num_splits   >= 1: each query tile's history (its attended positions, in
+ *                whole 64-position tiles) is cut into num_splits contiguous
+ *                ranges, each its own pair of CTAs writing an unnormalized
+ *                partial (max, sum, output); a second kernel merges them.
+ *                Short chunks over long prefixes need it to fill the GPU;
+ *                1 is a single pass (no partials, no merge).
+ *   workspace    >= jf_prefill_batch_workspace_bytes(sum_b chunk_len[b], Hq,
+ *                D, num_splits) bytes, 256-byte aligned; its first int32 is
+ *                the device status word.
  * The longest request's query tiles are scheduled first.
  */
 #define JF_PREFILL_MAX_BATCH 64
 
+/* 256 bytes for num_splits == 1, else 256 + roundup(8 R S, 256) + 4 R S D
+ * with R = total_rows * Hq (0 for invalid arguments). */
+size_t jf_prefill_batch_workspace_bytes(int64_t total_rows, int32_t num_q_heads, int32_t head_dim,
+                                        int32_t num_splits);
+
 int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                           int32_t batch, const int32_t* q_start, const int32_t* chunk_len,
                           const void* q, int32_t num_q_heads, float softmax_scale, int32_t causal,
-                          void* out, void* workspace, size_t workspace_bytes, void* stream);
+                          int32_t num_splits, void* out, void* workspace, size_t workspace_bytes,
+                          void* stream);
 
 /*
  * Page reservation of one unshared request (Eq. 7):

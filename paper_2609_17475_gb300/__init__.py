@@ -10,5 +10,5 @@ from .binding import (  # noqa: F401
     jf_paged_verify_attn, jf_prefill_chunk_attn, jf_prefill_workspace_bytes, lib,
     status_string, version, verify_workspace, default_verify_splits, workspace_status,
     JF_FMT_AFFINE4_G64, JF_FMT_TQ4, Tq4Codec, jf_kv_page_bytes_fmt, jf_tq4_codebook,
-    jf_prefill_batch_attn, jf_reservation_pages,
+    jf_prefill_batch_attn, jf_reservation_pages, prefill_batch_workspace, default_prefill_splits,
 )

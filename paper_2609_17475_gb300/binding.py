@@ -33,6 +33,7 @@ EXPORTS = [
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
     "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
     "jf_kv_page_bytes_fmt", "jf_tq4_codebook", "jf_prefill_batch_attn", "jf_reservation_pages",
+    "jf_prefill_batch_workspace_bytes",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -87,8 +88,9 @@ def lib() -> ctypes.CDLL:
                                                     SZ, I32, P]),
             "jf_kv_page_bytes_fmt": (SZ, [I32, I32, I32, I32]),
             "jf_tq4_codebook": (ctypes.c_int, [I32, ctypes.POINTER(ctypes.c_float)]),
-            "jf_prefill_batch_attn": (ctypes.c_int, [PP, P, I32, I32, P, P, P, I32, F32, I32, P,
-                                                     P, SZ, P]),
+            "jf_prefill_batch_attn": (ctypes.c_int, [PP, P, I32, I32, P, P, P, I32, F32, I32, I32,
+                                                     P, P, SZ, P]),
+            "jf_prefill_batch_workspace_bytes": (SZ, [I64, I32, I32, I32]),
             "jf_reservation_pages": (I64, [I64, I64, I64, I32]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
@@ -388,12 +390,50 @@ def jf_prefill_chunk_attn(pool: KVPool, page_table_row: torch.Tensor, q: torch.T
 JF_PREFILL_MAX_BATCH = 64
 
 
+def prefill_batch_workspace(total_rows: int, num_q_heads: int, head_dim: int, num_splits: int,
+                            device="cuda") -> torch.Tensor:
+    n = int(lib().jf_prefill_batch_workspace_bytes(int(total_rows), num_q_heads, head_dim,
+                                                   num_splits))
+    if n == 0:
+        raise ValueError("invalid workspace geometry")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: int,
+                           device=None) -> int:
+    """History splits for a launch: the kernel runs one CTA per SM, two per
+    pair, so about SMs / 2 pairs run at once; split so that the longest pair's
+    share of history tiles (64 positions each) is no more than the average
+    work per pair slot, without cutting any split below 8 tiles."""
+    G = num_q_heads // num_kv_heads
+    qpc = max(1, 128 // G)
+    total, longest = 0, 0
+    for s0, c in zip(q_start, chunk_len):
+        c = int(c)
+        if c:
+            pairs = (-(-c // qpc) + 1) // 2
+            for k in range(pairs):   # pair k holds query tiles 2k, 2k+1 (the later is longer)
+                last = min(c, (2 * k + 2) * qpc)
+                tiles = -(-(int(s0) + last) // 64)
+                total += tiles * num_kv_heads
+                longest = max(longest, tiles)
+    if total == 0:
+        return 1
+    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
+    slots = props.multi_processor_count // 2
+    per_slot = max(1.0, total / slots)
+    want = -(-longest // int(per_slot)) if per_slot >= 1 else 1
+    return int(max(1, min(want, longest // 8, 64)))
+
+
 def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk_len,
                           q: torch.Tensor, softmax_scale: float, causal: bool, out: torch.Tensor,
-                          workspace: torch.Tensor, stream=None) -> None:
+                          workspace: torch.Tensor, num_splits: int = 1, stream=None) -> None:
     """Prefill chunks of several requests in one launch.  ``q`` / ``out`` are
     the requests' chunks concatenated, [sum(chunk_len), Hq, D]; ``q_start`` and
-    ``chunk_len`` are host sequences (one entry per page-table row)."""
+    ``chunk_len`` are host sequences (one entry per page-table row).  With
+    ``num_splits`` > 1 each query tile's history is split across CTA pairs and
+    merged (workspace from prefill_batch_workspace)."""
     _need(page_table, torch.int32, "page_table")
     _need(q, torch.bfloat16, "q")
     _need(out, torch.bfloat16, "out")
@@ -408,8 +448,9 @@ def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk
     cl = (ctypes.c_int32 * B)(*[int(x) for x in chunk_len])
     st = lib().jf_prefill_batch_attn(ctypes.byref(pool.c_struct()), _ptr(page_table),
                                       page_table.shape[1], B, qs, cl, _ptr(q), Hq,
-                                      float(softmax_scale), int(bool(causal)), _ptr(out),
-                                      _ptr(workspace), workspace.numel(), _stream(stream))
+                                      float(softmax_scale), int(bool(causal)), int(num_splits),
+                                      _ptr(out), _ptr(workspace), workspace.numel(),
+                                      _stream(stream))
     _check("jf_prefill_batch_attn", st)
 
 

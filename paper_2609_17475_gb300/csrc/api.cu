@@ -32,7 +32,8 @@ int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int
                    cudaStream_t);
 int launch_prefill_batch(const Geom&, const jf_kv_pool&, const int32_t* const*, const int32_t*,
                          const int32_t*, const void*, const int64_t*, int32_t, int32_t, float,
-                         int32_t, void*, void*, cudaStream_t);
+                         int32_t, void*, void*, cudaStream_t, int32_t, int64_t);
+size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S);
 }  // namespace jfkv
 
 using namespace jfkv;
@@ -262,10 +263,18 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
                         softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
 }
 
+size_t jf_prefill_batch_workspace_bytes(int64_t total_rows, int32_t num_q_heads, int32_t head_dim,
+                                        int32_t num_splits) {
+  if (total_rows < 0 || num_q_heads < 1 || num_splits < 1 || num_splits > 65535) return 0;
+  if (head_dim != 128 && head_dim != 256) return 0;
+  return prefill_workspace_bytes(total_rows, num_q_heads, head_dim, num_splits);
+}
+
 int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                           int32_t batch, const int32_t* q_start, const int32_t* chunk_len,
                           const void* q, int32_t num_q_heads, float softmax_scale, int32_t causal,
-                          void* out, void* workspace, size_t workspace_bytes, void* stream) {
+                          int32_t num_splits, void* out, void* workspace, size_t workspace_bytes,
+                          void* stream) {
   int st = check_pool(pool);
   if (st) return st;
   if (batch < 1 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
@@ -274,8 +283,8 @@ int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int
   if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
   if (num_q_heads / pool->num_kv_heads > 128) return JF_ERR_UNSUPPORTED;
   if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
-  if (workspace_bytes < jf_prefill_workspace_bytes()) return JF_ERR_WORKSPACE_TOO_SMALL;
-  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 16)) return JF_ERR_INVALID_ARG;
+  if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 256)) return JF_ERR_INVALID_ARG;
   const int32_t* rows[JF_PREFILL_MAX_BATCH];
   int64_t row0[JF_PREFILL_MAX_BATCH];
   int64_t acc = 0;
@@ -287,12 +296,14 @@ int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int
     row0[b] = acc;
     acc += chunk_len[b];
   }
-  if (acc == 0) return JF_OK;
   if (acc > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
+  if (workspace_bytes < prefill_workspace_bytes(acc, num_q_heads, pool->head_dim, num_splits))
+    return JF_ERR_WORKSPACE_TOO_SMALL;
+  if (acc == 0) return JF_OK;
   const Geom g = make_geom(*pool);
   return launch_prefill_batch(g, *pool, rows, q_start, chunk_len, q, row0, batch, num_q_heads,
                               softmax_scale, causal, out, workspace,
-                              static_cast<cudaStream_t>(stream));
+                              static_cast<cudaStream_t>(stream), num_splits, acc);
 }
 
 int64_t jf_reservation_pages(int64_t prompt_len, int64_t output_len, int64_t g_out,

@@ -63,6 +63,7 @@ struct PfReq {
   const uint16_t* q;    // its chunk's queries [C, Hq, D]
   uint16_t* out;        // [C, Hq, D]
   int32_t q_start, C, tile0, n_tiles2;
+  int32_t row0;         // its first query's row in the launch (split partials)
 };
 
 constexpr int PF_MAX_REQ = 64;   // requests per launch
@@ -78,6 +79,9 @@ struct PrefillArgs {
   int32_t causal;
   float scale_log2;
   int32_t* status;
+  int32_t num_splits;   // > 1: history ranges per query tile, partials + merge
+  float* part_ml;       // [rows * Hq][num_splits][2] (m, l)
+  float* part_o;        // [rows * Hq][num_splits][D], unnormalized
   int32_t nreq;
   PfReq req[PF_MAX_REQ];
 };
@@ -186,7 +190,12 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   };
   const int kmax = kmax_of(qt);
   const int kmax_pair = max(kmax, kmax_of(qt_partner));
-  const int ntiles = (kmax_pair + PF_BN - 1) / PF_BN;   // the pair walks the same tiles
+  const int ntiles_all = (kmax_pair + PF_BN - 1) / PF_BN;
+  // this CTA pair's contiguous range of history tiles (the whole history when
+  // there is one split); both CTAs of the pair walk the same tiles
+  const int jb = (int)(((int64_t)ntiles_all * blockIdx.z) / a.num_splits);
+  const int je = (int)(((int64_t)ntiles_all * (blockIdx.z + 1)) / a.num_splits);
+  const int ntiles = je - jb;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < PF_KVBUF; ++i) {
@@ -262,7 +271,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     if (rank == 0 && lane == 0) {
       const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV);
       bool ok = true;
-      auto pv = [&](int j) {
+      auto pv = [&](int j) {   // j: local tile index within this split
         const int sb = j & 1, kb = j % PF_KVBUF;
         if (!tc::wait_cluster(&p_full[sb], (j >> 1) & 1)) { ok = false; return; }
         tc::fence_after();
@@ -286,7 +295,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         tc::commit2_both(&s_full[sb]);
         if (j >= 1) pv(j - 1);
       }
-      if (ok) pv(ntiles - 1);
+      if (ok && ntiles > 0) pv(ntiles - 1);
       if (!ok) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
     }
     __syncwarp();
@@ -315,9 +324,12 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     };
     // page id of tile j (P >= 64, so a tile lies in one page); it is loaded a
     // step before its tile's code loads need it
-    auto page_of = [&](int j) -> int { return j < ntiles ? __ldg(pt + (j * PF_BN) / a.P) : -1; };
+    // j: local tile index; the history tile is jb + j
+    auto page_of = [&](int j) -> int {
+      return j < ntiles ? __ldg(pt + ((jb + j) * PF_BN) / a.P) : -1;
+    };
     auto load_tile = [&](int j, int page, Tile& x) {
-      const int key0 = j * PF_BN;
+      const int key0 = (jb + j) * PF_BN;
       const bool pok = page >= 0 && page < a.num_pages;
       if (!pok && dt == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
       x.valid = pok && (key0 + tpos < kmax_pair);
@@ -365,7 +377,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       __syncwarp();
       if (lane == 0) tc::arrive_cluster(&kv_full[kbuf], 0);
     };
-    load_tile(0, page_of(0), ta);
+    if (ntiles > 0) load_tile(0, page_of(0), ta);
     if (ntiles > 1) load_tile(1, page_of(1), tb);
     for (int j = 0; j < ntiles && ok; j += 3) {
       step(j, ta, tcur);
@@ -390,7 +402,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       tc::ld32(tS + b * PF_BN + lane_off, s0);
       tc::ld32(tS + b * PF_BN + 32 + lane_off, s1);
       tc::wait_ld();
-      const int key0 = j * PF_BN;
+      const int key0 = (jb + j) * PF_BN;
       float x[PF_BN];
       float mt = -INFINITY;
       {
@@ -456,18 +468,42 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       __syncwarp();
       if (lane == 0) tc::arrive_cluster(&p_full[b], 0);
     }
-    // epilogue: O / l -> bf16, undoing the d order 0,4,1,5,2,6,3,7
-    if (ok && tc::wait_cluster(&pv_done[(ntiles - 1) % PF_KVBUF],
-                                ((ntiles - 1) / PF_KVBUF) & 1)) {
+    // epilogue: O / l -> bf16 (one split) or the unnormalized partial
+    // (m, l, O) in fp32 (several), undoing the d order 0,4,1,5,2,6,3,7
+    const bool split = a.num_splits > 1;
+    const int64_t prow = ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) *
+                         a.num_splits + blockIdx.z;
+    if (ntiles == 0) {   // an empty history range: a neutral partial
+      if (split && row_ok) {
+        a.part_ml[prow * 2 + 0] = -INFINITY;
+        a.part_ml[prow * 2 + 1] = 0.f;
+        float4* po = reinterpret_cast<float4*>(a.part_o + prow * D);
+        for (int c = 0; c < D / 4; ++c) po[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    } else if (ok && tc::wait_cluster(&pv_done[(ntiles - 1) % PF_KVBUF],
+                                       ((ntiles - 1) / PF_KVBUF) & 1)) {
       tc::fence_after();
-      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const float inv = split ? 1.f : (l > 0.f ? 1.f / l : 0.f);
       uint16_t* orow = rq.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
+      float* prow_o = split ? a.part_o + prow * D : nullptr;
+      if (split && row_ok) {
+        a.part_ml[prow * 2 + 0] = m_ref;
+        a.part_ml[prow * 2 + 1] = l;
+      }
 #pragma unroll 1
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t o[32];
         tc::ld32(tO + c0 + lane_off, o);
         tc::wait_ld();
-        if (row_ok) {
+        if (row_ok && split) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float* v = reinterpret_cast<const float*>(o + 8 * k);
+            float4* dst = reinterpret_cast<float4*>(prow_o + c0 + 8 * k);
+            dst[0] = make_float4(v[0], v[2], v[4], v[6]);
+            dst[1] = make_float4(v[1], v[3], v[5], v[7]);
+          }
+        } else if (row_ok) {
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const float* v = reinterpret_cast<const float*>(o + 8 * k);
@@ -500,14 +536,72 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   }
 }
 
+// Merge of a launch's history splits: one warp per (query, head) row combines
+// its S partials, o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+template <int D>
+__global__ void __launch_bounds__(256)
+prefill_merge_kernel(const float* part_ml, const float* part_o, uint16_t* out, int64_t rows,
+                     int S) {
+  constexpr int E = D / 32;
+  const int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;   // whole warps
+  const float2* ml = reinterpret_cast<const float2*>(part_ml) + row * S;
+  float M = -INFINITY;
+  for (int s2 = lane; s2 < S; s2 += 32) M = fmaxf(M, ml[s2].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+  float acc[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) acc[e] = 0.f;
+  float L = 0.f;
+  if (M != -INFINITY) {
+    for (int s2 = 0; s2 < S; ++s2) {
+      const float2 v = ml[s2];
+      if (v.x == -INFINITY) continue;   // an empty history range
+      const float w = fast_exp2(v.x - M);
+      L = fmaf(w, v.y, L);
+      const float4* po = reinterpret_cast<const float4*>(part_o + (row * S + s2) * D + lane * E);
+#pragma unroll
+      for (int e = 0; e < E / 4; ++e) {
+        const float4 x = po[e];
+        acc[4 * e + 0] = fmaf(w, x.x, acc[4 * e + 0]);
+        acc[4 * e + 1] = fmaf(w, x.y, acc[4 * e + 1]);
+        acc[4 * e + 2] = fmaf(w, x.z, acc[4 * e + 2]);
+        acc[4 * e + 3] = fmaf(w, x.w, acc[4 * e + 3]);
+      }
+    }
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  uint32_t wv[E / 2];
+#pragma unroll
+  for (int e = 0; e < E / 2; ++e)
+    wv[e] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e] * inv)) |
+            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e + 1] * inv)) << 16);
+  uint16_t* dst = out + row * D + lane * E;
+  if constexpr (E == 8)
+    *reinterpret_cast<uint4*>(dst) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+  else
+    *reinterpret_cast<uint2*>(dst) = make_uint2(wv[0], wv[1]);
+}
+
+// Workspace of a split prefill launch: status word, (m, l) and O partials.
+size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S) {
+  if (S <= 1) return 256;
+  const int64_t n = rows * Hq * S;
+  return (size_t)(256 + (n * 8 + 255) / 256 * 256 + n * D * 4);
+}
+
 // One launch over the chunks of `nreq` requests (nreq <= PF_MAX_REQ); requests
 // with an empty chunk get no CTAs.  The request with the most attended
 // positions goes first, so the longest CTA pairs start earliest.
 int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* const* pt_rows,
                          const int32_t* q_start, const int32_t* chunk_len, const void* q,
                          const int64_t* q_row0, int32_t nreq, int32_t Hq, float softmax_scale,
-                         int32_t causal, void* out, void* workspace, cudaStream_t stream) {
+                         int32_t causal, void* out, void* workspace, cudaStream_t stream,
+                         int32_t num_splits, int64_t total_rows) {
   if (nreq < 1 || nreq > PF_MAX_REQ) return JF_ERR_UNSUPPORTED;
+  if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
   PrefillArgs a;
   a.pool = static_cast<const uint8_t*>(pool.base);
   a.num_pages = g.num_pages;
@@ -524,6 +618,13 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
   a.causal = causal ? 1 : 0;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.status = static_cast<int32_t*>(workspace);
+  a.num_splits = num_splits;
+  {
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    const int64_t n = total_rows * Hq * num_splits;
+    a.part_ml = reinterpret_cast<float*>(ws + 256);
+    a.part_o = reinterpret_cast<float*>(ws + 256 + (n * 8 + 255) / 256 * 256);
+  }
   int order[PF_MAX_REQ];
   int n = 0;
   for (int b = 0; b < nreq; ++b)
@@ -546,6 +647,7 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
     r.out = static_cast<uint16_t*>(out) + (size_t)q_row0[b] * row_elems;
     r.q_start = q_start[b];
     r.C = chunk_len[b];
+    r.row0 = (int32_t)q_row0[b];
     r.tile0 = (int32_t)tiles;
     const int n_qtiles = (chunk_len[b] + a.QPC - 1) / a.QPC;
     r.n_tiles2 = (n_qtiles + 1) & ~1;   // CTA pairs
@@ -553,7 +655,7 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
   }
   a.nreq = n;
   if (tiles > 0x7FFFFFFF || g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
-  dim3 grid((unsigned)tiles, (unsigned)g.Hkv);
+  dim3 grid((unsigned)tiles, (unsigned)g.Hkv, (unsigned)num_splits);
   if (g.D == 256) {
     static bool attr = false;
     if (!attr) {
@@ -573,7 +675,20 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
     }
     prefill_kernel<128><<<grid, PF_THREADS, PfSmem<128>::TOTAL, stream>>>(a);
   }
-  return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
+  if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  if (num_splits > 1) {
+    const int64_t rows = total_rows * Hq;
+    const int64_t blocks = (rows + 7) / 8;
+    if (blocks > 0x7FFFFFFF) return JF_ERR_UNSUPPORTED;
+    if (g.D == 256)
+      prefill_merge_kernel<256><<<(unsigned)blocks, 256, 0, stream>>>(
+          a.part_ml, a.part_o, static_cast<uint16_t*>(out), rows, num_splits);
+    else
+      prefill_merge_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(
+          a.part_ml, a.part_o, static_cast<uint16_t*>(out), rows, num_splits);
+    if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  }
+  return JF_OK;
 }
 
 int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
@@ -582,7 +697,7 @@ int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
                    void* workspace, cudaStream_t stream) {
   const int64_t row0 = 0;
   return launch_prefill_batch(g, pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1, Hq,
-                              softmax_scale, causal, out, workspace, stream);
+                              softmax_scale, causal, out, workspace, stream, 1, chunk_len);
 }
 
 }  // namespace jfkv

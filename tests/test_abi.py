@@ -174,11 +174,18 @@ def test_prefill_batch_rejects_bad_arguments():
     I = ctypes.c_int32
     qs = (I * 2)(0, 100)
     cl = (I * 2)(16, 16)
-    call = lambda batch=2, stride=4, q_start=qs, clen=cl, wsb=256: L.jf_prefill_batch_attn(
-        ctypes.byref(p), FAKE, stride, batch, q_start, clen, FAKE, 8, 0.1, 1, FAKE, FAKE, wsb, None)
+    call = lambda batch=2, stride=4, q_start=qs, clen=cl, wsb=256, splits=1: L.jf_prefill_batch_attn(
+        ctypes.byref(p), FAKE, stride, batch, q_start, clen, FAKE, 8, 0.1, 1, splits, FAKE, FAKE,
+        wsb, None)
     assert call(batch=0) == B.JF_ERR_INVALID_ARG
     assert call(batch=65, q_start=(I * 65)(), clen=(I * 65)()) == B.JF_ERR_UNSUPPORTED
     assert call(wsb=0) == B.JF_ERR_WORKSPACE_TOO_SMALL
     assert call(stride=1, q_start=(I * 2)(0, 250), clen=(I * 2)(4, 16)) == B.JF_ERR_INVALID_ARG
     assert call(q_start=(I * 2)(-1, 0)) == B.JF_ERR_INVALID_ARG
     assert call(clen=(I * 2)(0, 0)) == B.JF_OK                     # nothing to do
+    assert call(splits=0) == B.JF_ERR_INVALID_ARG
+    need = L.jf_prefill_batch_workspace_bytes
+    n = need(32, 8, 128, 4)
+    assert n == 256 + (32 * 8 * 4 * 8 + 255) // 256 * 256 + 32 * 8 * 4 * 128 * 4
+    assert need(32, 8, 128, 1) == 256 and need(32, 8, 96, 4) == 0
+    assert call(splits=4, wsb=n - 1) == B.JF_ERR_WORKSPACE_TOO_SMALL
