@@ -399,6 +399,21 @@ def _bench_prefill_batch(jf, dev, stream, peak_tf):
     res["one_chunk_64_at_32704"] = {"whole_history_us": t_one * 1e3, "splits": s1,
                                     "split_us": t_one_s * 1e3, "speedup": t_one / t_one_s,
                                     "TFLOPs_split": fl1 / (t_one_s / 1e3) / 1e12}
+    # a large chunk: 2,048 queries after 30,720 positions, unsplit vs the default split
+    q2 = torch.randn(2048, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    o2 = torch.empty_like(q2)
+    s2 = jf.default_prefill_splits([ctx - 2048], [2048], Hq, Hkv)
+    w2 = jf.prefill_batch_workspace(2048, Hq, D, s2, device=dev)
+    t2 = _event_time(lambda: jf.jf_prefill_chunk_attn(pool, pt[0], q2, ctx - 2048, scale, True,
+                                                      o2, ws, stream=stream), 5, stream)
+    t2s = _event_time(lambda: jf.jf_prefill_batch_attn(pool, pt[:1], [ctx - 2048], [2048], q2,
+                                                       scale, True, o2, w2, num_splits=s2,
+                                                       stream=stream), 5, stream)
+    fl2 = 4 * Hq * D * (2048 * (ctx - 2048) + 2048 * 2049 // 2)
+    res["one_chunk_2048_at_30720"] = {"unsplit_ms": t2, "splits": s2, "split_ms": t2s,
+                                      "TFLOPs_unsplit": fl2 / (t2 / 1e3) / 1e12,
+                                      "TFLOPs_split": fl2 / (t2s / 1e3) / 1e12}
+    del w2
     for C in (64, 512):
         starts = [4096 * (b + 1) - C for b in range(B)]
         q = torch.randn(B * C, Hq, D, generator=g, device=dev).to(torch.bfloat16)

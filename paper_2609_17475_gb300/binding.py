@@ -401,29 +401,43 @@ def prefill_batch_workspace(total_rows: int, num_q_heads: int, head_dim: int, nu
 
 def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: int,
                            device=None) -> int:
-    """History splits for a launch: the kernel runs one CTA per SM, two per
-    pair, so about SMs / 2 pairs run at once; split so that the longest pair's
-    share of history tiles (64 positions each) is no more than the average
-    work per pair slot, without cutting any split below 8 tiles."""
+    """History splits for a launch.  The kernel runs one CTA per SM, two per
+    pair, so SMs / 2 pairs run at once; each candidate split count is scored
+    by its makespan when the pairs' history tiles (64 positions each, plus a
+    fixed cost per pair) are list-scheduled longest first onto those slots,
+    and the smallest count within 10 % of the best is returned (splits cost
+    partial writes and a merge the estimate leaves out; no split below 8
+    tiles)."""
+    import heapq
     G = num_q_heads // num_kv_heads
     qpc = max(1, 128 // G)
-    total, longest = 0, 0
+    work = []   # history tiles of every CTA pair (per KV head)
     for s0, c in zip(q_start, chunk_len):
         c = int(c)
-        if c:
-            pairs = (-(-c // qpc) + 1) // 2
-            for k in range(pairs):   # pair k holds query tiles 2k, 2k+1 (the later is longer)
-                last = min(c, (2 * k + 2) * qpc)
-                tiles = -(-(int(s0) + last) // 64)
-                total += tiles * num_kv_heads
-                longest = max(longest, tiles)
-    if total == 0:
+        for k in range((-(-c // qpc) + 1) // 2 if c else 0):
+            last = min(c, (2 * k + 2) * qpc)
+            work += [-(-(int(s0) + last) // 64)] * num_kv_heads
+    if not work:
         return 1
     props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    slots = props.multi_processor_count // 2
-    per_slot = max(1.0, total / slots)
-    want = -(-longest // int(per_slot)) if per_slot >= 1 else 1
-    return int(max(1, min(want, longest // 8, 64)))
+    slots = max(1, props.multi_processor_count // 2)
+    longest = max(work)
+    scores = []
+    for S in [1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 12, 14, 16, 20, 24, 32, 48, 64]:
+        if S > 1 and longest // S < 8:
+            break
+        items = sorted((-(-w // S) + 2 for w in work for _ in range(S)), reverse=True)
+        if len(items) <= slots:
+            t = items[0]
+        else:
+            heap = [0] * slots
+            for it in items:
+                heapq.heapreplace(heap, heap[0] + it)
+            t = max(heap)
+        t += 2 if S > 1 else 0   # the merge pass
+        scores.append((S, t))
+    best_t = min(t for _, t in scores)
+    return next(S for S, t in scores if t <= 1.1 * best_t)
 
 
 def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk_len,
