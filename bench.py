@@ -490,8 +490,18 @@ def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
     pp = torch.arange(0, 2048, dtype=torch.int32, device=dev)
     ta = _event_time(lambda: jf.jf_kv_quantize_append(pools[0], tables[0], rr, pp, kk, vv, err,
                                                       stream=stream), 20, stream)
+    # prefill over TQ4 pages: 2,048 causal queries after a 30,720-position
+    # prefix of the first cache (rotated queries, centroid tiles, merge with
+    # the inverse rotation)
+    Cq, q0 = 2048, 30720
+    qp = torch.randn(Cq, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+    op = torch.empty_like(qp)
+    wp = jf.prefill_batch_workspace(Cq, Hq, D, 1, device=dev, format=jf.JF_FMT_TQ4)
+    tp = _event_time(lambda: jf.jf_prefill_chunk_attn(pools[0], tables[0][0], qp, q0, 1 / 16, True,
+                                                      op, wp, stream=stream), 5, stream)
+    fl = 4 * Hq * D * (Cq * q0 + Cq * (Cq + 1) // 2)
     stream.synchronize()
-    assert jf.workspace_status(ws) == 0 and int(err.item()) == 0
+    assert jf.workspace_status(ws) == 0 and int(err.item()) == 0 and jf.workspace_status(wp) == 0
     bpp = 2 * Hkv * (D // 2 + 2)
     alg = ctx * bpp + 2 * Hq * D * 2 + (ctx // P) * 4
     gbs = alg / (t / 1e3) / 1e9
@@ -499,7 +509,8 @@ def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
            "frac_of_measured": gbs / peaks_gbs, "splits": splits, "bytes_per_position": bpp,
            "alg_bytes_per_call": alg, "traffic": measured_traffic("tq4_split_kernel<256>"),
            "append_2048_rows_us": ta * 1e3,
-           "append_GBps": (2048 * Hkv * D * 2 * 2 + 2048 * bpp) / (ta / 1e3) / 1e9}
+           "append_GBps": (2048 * Hkv * D * 2 * 2 + 2048 * bpp) / (ta / 1e3) / 1e9,
+           "prefill_2048_at_30720_ms": tp, "prefill_TFLOPs": fl / (tp / 1e3) / 1e12}
     del pools
     return res
 

@@ -261,7 +261,15 @@ int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_tabl
  * already hold the chunk's own rows (append, then attend).
  *   page_table_row  int32 [>= ceil((q_start + chunk_len) / P)]
  *   q, out          bf16 [chunk_len, Hq, D]
- *   workspace       >= jf_prefill_workspace_bytes(); int32 status word.
+ *   workspace       affine pool: >= jf_prefill_workspace_bytes() (an int32
+ *                   status word); TQ4 pool: >= jf_prefill_batch_workspace_bytes(
+ *                   JF_FMT_TQ4, chunk_len, Hq, D, 1), 256-byte aligned.
+ * TQ4 pools (Sec. 3.1: page lookup, unpacking, centroid lookup, inverse
+ * rotation and norm restoration fused into the attention's operand path):
+ * the queries are rotated once (q' = H S_K q / sqrt(D), fp32 in the
+ * workspace), K and V tiles are built in shared memory as norm * centroid
+ * (fp16) in the rotated basis, and each output row is rotated back
+ * (S_V H / sqrt(D)) as the partials are merged.
  */
 int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
                           const void* q, int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
@@ -289,17 +297,19 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
  *                partial (max, sum, output); a second kernel merges them.
  *                Short chunks over long prefixes need it to fill the GPU;
  *                1 is a single pass (no partials, no merge).
- *   workspace    >= jf_prefill_batch_workspace_bytes(sum_b chunk_len[b], Hq,
- *                D, num_splits) bytes, 256-byte aligned; its first int32 is
- *                the device status word.
- * The longest request's query tiles are scheduled first.
+ *   workspace    >= jf_prefill_batch_workspace_bytes(pool->format,
+ *                sum_b chunk_len[b], Hq, D, num_splits) bytes, 256-byte
+ *                aligned; its first int32 is the device status word.
+ * The longest request's query tiles are scheduled first.  Either format.
  */
 #define JF_PREFILL_MAX_BATCH 64
 
-/* 256 bytes for num_splits == 1, else 256 + roundup(8 R S, 256) + 4 R S D
- * with R = total_rows * Hq (0 for invalid arguments). */
-size_t jf_prefill_batch_workspace_bytes(int64_t total_rows, int32_t num_q_heads, int32_t head_dim,
-                                        int32_t num_splits);
+/* Workspace of a prefill launch over a pool of `format`: 256 bytes for an
+ * affine pool with num_splits == 1; else 256 + roundup(8 R S, 256) + 4 R S D,
+ * R = total_rows * Hq (the split partials), plus 4 R D for a TQ4 pool (its
+ * rotated queries).  0 for invalid arguments. */
+size_t jf_prefill_batch_workspace_bytes(int32_t format, int64_t total_rows, int32_t num_q_heads,
+                                        int32_t head_dim, int32_t num_splits);
 
 int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                           int32_t batch, const int32_t* q_start, const int32_t* chunk_len,

@@ -90,7 +90,7 @@ def lib() -> ctypes.CDLL:
             "jf_tq4_codebook": (ctypes.c_int, [I32, ctypes.POINTER(ctypes.c_float)]),
             "jf_prefill_batch_attn": (ctypes.c_int, [PP, P, I32, I32, P, P, P, I32, F32, I32, I32,
                                                      P, P, SZ, P]),
-            "jf_prefill_batch_workspace_bytes": (SZ, [I64, I32, I32, I32]),
+            "jf_prefill_batch_workspace_bytes": (SZ, [I32, I64, I32, I32, I32]),
             "jf_reservation_pages": (I64, [I64, I64, I64, I32]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
@@ -391,9 +391,9 @@ JF_PREFILL_MAX_BATCH = 64
 
 
 def prefill_batch_workspace(total_rows: int, num_q_heads: int, head_dim: int, num_splits: int,
-                            device="cuda") -> torch.Tensor:
-    n = int(lib().jf_prefill_batch_workspace_bytes(int(total_rows), num_q_heads, head_dim,
-                                                   num_splits))
+                            device="cuda", format: int = JF_FMT_AFFINE4_G64) -> torch.Tensor:
+    n = int(lib().jf_prefill_batch_workspace_bytes(int(format), int(total_rows), num_q_heads,
+                                                   head_dim, num_splits))
     if n == 0:
         raise ValueError("invalid workspace geometry")
     return torch.zeros(n, dtype=torch.uint8, device=device)
@@ -405,9 +405,8 @@ def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: i
     pair, so SMs / 2 pairs run at once; each candidate split count is scored
     by its makespan when the pairs' history tiles (64 positions each, plus a
     fixed cost per pair) are list-scheduled longest first onto those slots,
-    and the smallest count within 10 % of the best is returned (splits cost
-    partial writes and a merge the estimate leaves out; no split below 8
-    tiles)."""
+    and the best is returned (no split below 8 tiles; a 2 % margin keeps the
+    smaller count on a near tie, splits costing partial writes and a merge)."""
     import heapq
     G = num_q_heads // num_kv_heads
     qpc = max(1, 128 // G)
@@ -437,7 +436,7 @@ def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: i
         t += 2 if S > 1 else 0   # the merge pass
         scores.append((S, t))
     best_t = min(t for _, t in scores)
-    return next(S for S, t in scores if t <= 1.1 * best_t)
+    return next(S for S, t in scores if t <= 1.02 * best_t)
 
 
 def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk_len,

@@ -32,8 +32,9 @@ int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int
                    cudaStream_t);
 int launch_prefill_batch(const Geom&, const jf_kv_pool&, const int32_t* const*, const int32_t*,
                          const int32_t*, const void*, const int64_t*, int32_t, int32_t, float,
-                         int32_t, void*, void*, cudaStream_t, int32_t, int64_t);
-size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S);
+                         int32_t, void*, void*, cudaStream_t, int32_t, int64_t,
+                         const Tq4Params*);
+size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S, int fmt);
 }  // namespace jfkv
 
 using namespace jfkv;
@@ -246,28 +247,43 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
                           int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
                           float softmax_scale, int32_t causal, void* out, void* workspace,
                           size_t workspace_bytes, void* stream) {
-  int st = check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (!page_table_row || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
   if (q_start < 0 || chunk_len < 0 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
   if (num_q_heads % pool->num_kv_heads) return JF_ERR_INVALID_ARG;
   if (!(softmax_scale == softmax_scale)) return JF_ERR_INVALID_ARG;
-  if (workspace_bytes < jf_prefill_workspace_bytes()) return JF_ERR_WORKSPACE_TOO_SMALL;
-  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, 16)) return JF_ERR_INVALID_ARG;
+  const bool tq = pool->format == JF_FMT_TQ4;
+  const size_t need = tq ? prefill_workspace_bytes(chunk_len, num_q_heads, pool->head_dim, 1,
+                                                   JF_FMT_TQ4)
+                         : jf_prefill_workspace_bytes();
+  if (workspace_bytes < need) return JF_ERR_WORKSPACE_TOO_SMALL;
+  if (!aligned(q, 16) || !aligned(out, 16) || !aligned(workspace, tq ? 256 : 16))
+    return JF_ERR_INVALID_ARG;
   if ((int64_t)q_start + chunk_len > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
   if (chunk_len == 0) return JF_OK;
   const Geom g = make_geom(*pool);
   if (num_q_heads / pool->num_kv_heads > 128) return JF_ERR_UNSUPPORTED;
+  if (tq) {
+    Tq4Params prm;
+    st = tq4_make_params(pool->tq4, g.D, &prm);
+    if (st) return st;
+    const int64_t row0 = 0;
+    return launch_prefill_batch(g, *pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1,
+                                num_q_heads, softmax_scale, causal, out, workspace,
+                                static_cast<cudaStream_t>(stream), 1, chunk_len, &prm);
+  }
   CUtensorMap tmap{};
   return launch_prefill(g, *pool, tmap, page_table_row, q, q_start, chunk_len, num_q_heads,
                         softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
 }
 
-size_t jf_prefill_batch_workspace_bytes(int64_t total_rows, int32_t num_q_heads, int32_t head_dim,
-                                        int32_t num_splits) {
+size_t jf_prefill_batch_workspace_bytes(int32_t format, int64_t total_rows, int32_t num_q_heads,
+                                        int32_t head_dim, int32_t num_splits) {
+  if (format != JF_FMT_AFFINE4_G64 && format != JF_FMT_TQ4) return 0;
   if (total_rows < 0 || num_q_heads < 1 || num_splits < 1 || num_splits > 65535) return 0;
   if (head_dim != 128 && head_dim != 256) return 0;
-  return prefill_workspace_bytes(total_rows, num_q_heads, head_dim, num_splits);
+  return prefill_workspace_bytes(total_rows, num_q_heads, head_dim, num_splits, format);
 }
 
 int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
@@ -275,7 +291,7 @@ int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int
                           const void* q, int32_t num_q_heads, float softmax_scale, int32_t causal,
                           int32_t num_splits, void* out, void* workspace, size_t workspace_bytes,
                           void* stream) {
-  int st = check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (batch < 1 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
   if (batch > JF_PREFILL_MAX_BATCH) return JF_ERR_UNSUPPORTED;
@@ -297,13 +313,20 @@ int jf_prefill_batch_attn(const jf_kv_pool* pool, const int32_t* page_table, int
     acc += chunk_len[b];
   }
   if (acc > 0x7FFFFFFF) return JF_ERR_INVALID_ARG;
-  if (workspace_bytes < prefill_workspace_bytes(acc, num_q_heads, pool->head_dim, num_splits))
+  if (workspace_bytes <
+      prefill_workspace_bytes(acc, num_q_heads, pool->head_dim, num_splits, pool->format))
     return JF_ERR_WORKSPACE_TOO_SMALL;
   if (acc == 0) return JF_OK;
   const Geom g = make_geom(*pool);
+  Tq4Params prm;
+  if (pool->format == JF_FMT_TQ4) {
+    st = tq4_make_params(pool->tq4, g.D, &prm);
+    if (st) return st;
+  }
   return launch_prefill_batch(g, *pool, rows, q_start, chunk_len, q, row0, batch, num_q_heads,
                               softmax_scale, causal, out, workspace,
-                              static_cast<cudaStream_t>(stream), num_splits, acc);
+                              static_cast<cudaStream_t>(stream), num_splits, acc,
+                              pool->format == JF_FMT_TQ4 ? &prm : nullptr);
 }
 
 int64_t jf_reservation_pages(int64_t prompt_len, int64_t output_len, int64_t g_out,

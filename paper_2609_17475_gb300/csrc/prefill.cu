@@ -45,6 +45,7 @@
 #include <cmath>
 
 #include "tc.cuh"
+#include "tq4.cuh"
 
 namespace jfkv {
 
@@ -82,6 +83,8 @@ struct PrefillArgs {
   int32_t num_splits;   // > 1: history ranges per query tile, partials + merge
   float* part_ml;       // [rows * Hq][num_splits][2] (m, l)
   float* part_o;        // [rows * Hq][num_splits][D], unnormalized
+  const float* qrot;     // TQ4: rotated queries H S_K q / sqrt(D), fp32 [rows * Hq][D]
+  float cent[16];        // TQ4: centroids
   int32_t nreq;
   PfReq req[PF_MAX_REQ];
 };
@@ -89,15 +92,22 @@ struct PrefillArgs {
 // Each CTA of a pair holds half of every K/V tile: K rows 32 r .. 32 r + 31
 // (all of head_dim, K-major) and V columns D/2 r .. D/2 (r + 1) (all 64
 // positions, MN-major), r = its rank in the pair.
-template <int D>
+template <int D, int FMT>
 struct PfSmem {
   static constexpr int KT_BYTES = (PF_BN / 2) * D * 2;   // [D/64][32 rows][128 B]
   static constexpr int VT_BYTES = PF_BN * (D / 2) * 2;   // [D/128][64 rows][128 B]
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = PF_KVBUF * KT_BYTES;
   static constexpr int OFF_BAR = OFF_V + PF_KVBUF * VT_BYTES;
-  static constexpr int TOTAL = 1024 + OFF_BAR + 256;
+  static constexpr int OFF_LUT = OFF_BAR + 256;   // TQ4 centroid table (lane-replicated)
+  static constexpr int TOTAL = 1024 + OFF_LUT + (FMT == JF_FMT_TQ4 ? 256 * 32 * 4 : 0);
 };
+
+__device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("mul.rn.f16x2 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
 
 __device__ __forceinline__ uint32_t hadd2(uint32_t a, uint32_t b) {
   uint32_t r;
@@ -137,10 +147,13 @@ __device__ __forceinline__ void sb_to_h2(uint32_t w, uint32_t& s2, uint32_t& b2)
   b2 = pack_f16x2(b, b);
 }
 
-template <int D>
+// FMT: JF_FMT_AFFINE4_G64, or JF_FMT_TQ4 (centroid table, rotated queries,
+// natural d order, partial outputs rotated back by the merge kernel)
+template <int D, int FMT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PF_THREADS, 1)
 prefill_kernel(const __grid_constant__ PrefillArgs a) {
-  using L = PfSmem<D>;
+  using L = PfSmem<D, FMT>;
+  constexpr bool TQ = FMT == JF_FMT_TQ4;
   constexpr int NKB = D / 64;           // 64-wide d blocks
   constexpr int UPI = (D == 256) ? 2 : 1;   // 16-byte code units per dequant item
   constexpr int SBB = D / 16;
@@ -208,6 +221,11 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     }
     fence_barrier_init();
   }
+  if constexpr (TQ) {   // centroid pair of code byte b for lane l: word b * 32 + l
+    uint32_t* lut = reinterpret_cast<uint32_t*>(sm + L::OFF_LUT);
+    for (int i = threadIdx.x; i < 256 * 32; i += blockDim.x)
+      lut[i] = pack_f16x2(a.cent[(i >> 5) & 15], a.cent[i >> 9]);
+  }
   if (warp == 0) tc::alloc2(tmem_slot, 512);
   tc::fence_before();
   __syncthreads();
@@ -226,7 +244,33 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   const int qi = row_ok ? r / a.G : 0;
   const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
   int qe = 0;                                  // per-row power of two kept out of fp16
-  if (warp > PF_DQ_WARPS) {
+  if (TQ && warp > PF_DQ_WARPS) {
+    // rotated fp32 query row, natural d order (the centroid pairs are too)
+    const float* qrow = a.qrot + ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
+    float qmax = 0.f;
+    if (row_ok) {
+      for (int c4 = 0; c4 < D / 4; ++c4) {
+        const float4 w = *reinterpret_cast<const float4*>(qrow + 4 * c4);
+        qmax = fmaxf(qmax, fmaxf(fmaxf(fabsf(w.x), fabsf(w.y)), fmaxf(fabsf(w.z), fabsf(w.w))));
+      }
+    }
+    qmax *= fabsf(a.scale_log2);
+    qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
+    const float qs = ldexpf(a.scale_log2, -qe);
+#pragma unroll 1
+    for (int c0 = 0; c0 < D / 2; c0 += 32) {   // 32 TMEM columns = 64 values
+      uint32_t v[32];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        float4 w = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (row_ok) w = *reinterpret_cast<const float4*>(qrow + 2 * c0 + 4 * k);
+        v[2 * k + 0] = pack_f16x2(w.x * qs, w.y * qs);
+        v[2 * k + 1] = pack_f16x2(w.z * qs, w.w * qs);
+      }
+      tc::st32(tQ + c0 + lane_off, v);
+    }
+    tc::wait_st();
+  } else if (warp > PF_DQ_WARPS) {
     const uint16_t* qrow = rq.q + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
     float qmax = 0.f;
     if (row_ok) {
@@ -316,7 +360,9 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
                              : sK + kbl * ((PF_BN / 2) * 128) + t * 128;
     const int tile_bytes = is_v ? L::VT_BYTES : L::KT_BYTES;
     const int64_t code_off = (is_v ? a.codes_region : 0) + kb * 32 + u0 * 16;
-    const int64_t sb_off = a.sb_base + (is_v ? a.sb_region : 0) + kb * 4;
+    // affine: the block's scale/bias word; TQ4: the vector's fp16 norm
+    const int64_t sb_off = a.sb_base + (is_v ? a.sb_region : 0) + (TQ ? 0 : kb * 4);
+    const uint32_t lut_lane = smem_u32(sm + L::OFF_LUT) + 4u * (uint32_t)lane;
     struct Tile {
       uint4 c[UPI];
       uint32_t sbw;
@@ -339,18 +385,43 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         const uint8_t* cp = base + code_off + row * CB;
 #pragma unroll
         for (int u = 0; u < UPI; ++u) x.c[u] = __ldg(reinterpret_cast<const uint4*>(cp + 16 * u));
-        x.sbw = __ldg(reinterpret_cast<const uint32_t*>(base + sb_off + row * SBB));
+        if constexpr (TQ)
+          x.sbw = __ldg(reinterpret_cast<const uint16_t*>(base + sb_off + row * 2));
+        else
+          x.sbw = __ldg(reinterpret_cast<const uint32_t*>(base + sb_off + row * SBB));
       }
     };
     auto store = [&](uint8_t* tile, const Tile& x) {
-      uint32_t s2, b2;
-      sb_to_h2(x.sbw, s2, b2);
       uint4 o[UPI][4];
+      if constexpr (TQ) {
+        // TQ4: norm * centroid of each index, natural d order (byte i gives
+        // d 2i, 2i+1); |c| < 1/4 and norm <= 65504 keep it in fp16 range
+        const uint32_t n2 = (x.sbw & 0xFFFFu) | (x.sbw << 16);
 #pragma unroll
-      for (int u = 0; u < UPI; ++u) {
-        const uint32_t cw[4] = {x.c[u].x, x.c[u].y, x.c[u].z, x.c[u].w};
+        for (int u = 0; u < UPI; ++u) {
+          const uint32_t cw[4] = {x.c[u].x, x.c[u].y, x.c[u].z, x.c[u].w};
 #pragma unroll
-        for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
+          for (int w = 0; w < 4; ++w) {
+            uint32_t q4[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              uint32_t v;
+              asm("ld.shared.b32 %0, [%1];\n"
+                  : "=r"(v) : "r"(lut_lane + __byte_perm(cw[w], 0u, 0x4440u + k) * 128u));
+              q4[k] = hmul2(v, n2);
+            }
+            o[u][w] = make_uint4(q4[0], q4[1], q4[2], q4[3]);
+          }
+        }
+      } else {
+        uint32_t s2, b2;
+        sb_to_h2(x.sbw, s2, b2);
+#pragma unroll
+        for (int u = 0; u < UPI; ++u) {
+          const uint32_t cw[4] = {x.c[u].x, x.c[u].y, x.c[u].z, x.c[u].w};
+#pragma unroll
+          for (int w = 0; w < 4; ++w) o[u][w] = dequant8(cw[w], s2, b2);
+        }
       }
 #pragma unroll
       for (int u = 0; u < UPI; ++u)
@@ -470,7 +541,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     }
     // epilogue: O / l -> bf16 (one split) or the unnormalized partial
     // (m, l, O) in fp32 (several), undoing the d order 0,4,1,5,2,6,3,7
-    const bool split = a.num_splits > 1;
+    const bool split = TQ || a.num_splits > 1;   // TQ4: the merge rotates O back
     const int64_t prow = ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) *
                          a.num_splits + blockIdx.z;
     if (ntiles == 0) {   // an empty history range: a neutral partial
@@ -500,8 +571,13 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
           for (int k = 0; k < 4; ++k) {
             const float* v = reinterpret_cast<const float*>(o + 8 * k);
             float4* dst = reinterpret_cast<float4*>(prow_o + c0 + 8 * k);
-            dst[0] = make_float4(v[0], v[2], v[4], v[6]);
-            dst[1] = make_float4(v[1], v[3], v[5], v[7]);
+            if constexpr (TQ) {
+              dst[0] = make_float4(v[0], v[1], v[2], v[3]);
+              dst[1] = make_float4(v[4], v[5], v[6], v[7]);
+            } else {
+              dst[0] = make_float4(v[0], v[2], v[4], v[6]);
+              dst[1] = make_float4(v[1], v[3], v[5], v[7]);
+            }
           }
         } else if (row_ok) {
 #pragma unroll
@@ -536,12 +612,47 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   }
 }
 
-// Merge of a launch's history splits: one warp per (query, head) row combines
-// its S partials, o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s.
+struct SignBits {
+  uint32_t w[8];   // bit j set: S_jj = -1
+};
+
+// TQ4 prefill: rotated queries q' = H S_K q / sqrt(D) in fp32, one warp per
+// (query, head) row (Sec. 3.1 Eq. 4: keys stay in the rotated basis).
 template <int D>
 __global__ void __launch_bounds__(256)
+prefill_rotate_q_kernel(const uint16_t* q, float* qrot, int64_t rows, SignBits sk) {
+  constexpr int E = D / 32;
+  const int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;   // whole warps
+  const uint16_t* src = q + row * D + lane * E;
+  float x[E];
+#pragma unroll
+  for (int e = 0; e < E; e += 2) {
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(src + e);
+    x[e] = bf16lo_to_f32(w);
+    x[e + 1] = bf16hi_to_f32(w);
+  }
+  const uint32_t sb = sk.w[(lane * E) >> 5] >> ((lane * E) & 31);
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if ((sb >> e) & 1u) x[e] = -x[e];
+  warp_fwht<float, E>(x, lane);
+  const float r = rsqrtf((float)D);
+  float* dst = qrot + row * D + lane * E;
+#pragma unroll
+  for (int e = 0; e < E; e += 4)
+    *reinterpret_cast<float4*>(dst + e) = make_float4(x[e] * r, x[e + 1] * r, x[e + 2] * r,
+                                                      x[e + 3] * r);
+}
+
+// Merge of a launch's history splits: one warp per (query, head) row combines
+// its S partials, o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s; for TQ4
+// (ROT) the result is rotated back, o <- S_V H o / sqrt(D).
+template <int D, bool ROT>
+__global__ void __launch_bounds__(256)
 prefill_merge_kernel(const float* part_ml, const float* part_o, uint16_t* out, int64_t rows,
-                     int S) {
+                     int S, SignBits sv) {
   constexpr int E = D / 32;
   const int64_t row = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
@@ -573,11 +684,23 @@ prefill_merge_kernel(const float* part_ml, const float* part_o, uint16_t* out, i
     }
   }
   const float inv = L > 0.f ? 1.f / L : 0.f;
+  if constexpr (ROT) {
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] *= inv;
+    warp_fwht<float, E>(acc, lane);
+    const float r = rsqrtf((float)D);
+    const uint32_t sb = sv.w[(lane * E) >> 5] >> ((lane * E) & 31);
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] *= ((sb >> e) & 1u) ? -r : r;
+  } else {
+#pragma unroll
+    for (int e = 0; e < E; ++e) acc[e] *= inv;
+  }
   uint32_t wv[E / 2];
 #pragma unroll
   for (int e = 0; e < E / 2; ++e)
-    wv[e] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e] * inv)) |
-            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e + 1] * inv)) << 16);
+    wv[e] = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e])) |
+            ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * e + 1])) << 16);
   uint16_t* dst = out + row * D + lane * E;
   if constexpr (E == 8)
     *reinterpret_cast<uint4*>(dst) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
@@ -585,11 +708,29 @@ prefill_merge_kernel(const float* part_ml, const float* part_o, uint16_t* out, i
     *reinterpret_cast<uint2*>(dst) = make_uint2(wv[0], wv[1]);
 }
 
-// Workspace of a split prefill launch: status word, (m, l) and O partials.
-size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S) {
-  if (S <= 1) return 256;
+// Workspace of a prefill launch: status word, then (split launches and every
+// TQ4 launch) (m, l) and O partials, then (TQ4) the rotated queries.
+size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S, int fmt) {
+  const bool tq = fmt == JF_FMT_TQ4;
+  if (S <= 1 && !tq) return 256;
   const int64_t n = rows * Hq * S;
-  return (size_t)(256 + (n * 8 + 255) / 256 * 256 + n * D * 4);
+  const int64_t part = 256 + (n * 8 + 255) / 256 * 256 + n * D * 4;
+  return (size_t)(part + (tq ? rows * Hq * D * 4 : 0));
+}
+
+// One prefill launch of a given instantiation (its shared-memory opt-in is
+// set once per instantiation).
+template <int D, int FMT>
+static int launch_pf(const dim3& grid, const PrefillArgs& a, cudaStream_t stream) {
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(prefill_kernel<D, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             PfSmem<D, FMT>::TOTAL) != cudaSuccess)
+      return JF_ERR_CUDA;
+    attr = true;
+  }
+  prefill_kernel<D, FMT><<<grid, PF_THREADS, PfSmem<D, FMT>::TOTAL, stream>>>(a);
+  return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }
 
 // One launch over the chunks of `nreq` requests (nreq <= PF_MAX_REQ); requests
@@ -599,8 +740,9 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
                          const int32_t* q_start, const int32_t* chunk_len, const void* q,
                          const int64_t* q_row0, int32_t nreq, int32_t Hq, float softmax_scale,
                          int32_t causal, void* out, void* workspace, cudaStream_t stream,
-                         int32_t num_splits, int64_t total_rows) {
+                         int32_t num_splits, int64_t total_rows, const Tq4Params* tq4) {
   if (nreq < 1 || nreq > PF_MAX_REQ) return JF_ERR_UNSUPPORTED;
+  const bool tq = tq4 != nullptr;
   if (num_splits < 1 || num_splits > 65535) return JF_ERR_INVALID_ARG;
   PrefillArgs a;
   a.pool = static_cast<const uint8_t*>(pool.base);
@@ -619,11 +761,20 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.status = static_cast<int32_t*>(workspace);
   a.num_splits = num_splits;
+  SignBits sk{}, sv{};
   {
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     const int64_t n = total_rows * Hq * num_splits;
     a.part_ml = reinterpret_cast<float*>(ws + 256);
     a.part_o = reinterpret_cast<float*>(ws + 256 + (n * 8 + 255) / 256 * 256);
+    a.qrot = tq ? reinterpret_cast<const float*>(ws + 256 + (n * 8 + 255) / 256 * 256 +
+                                                 n * g.D * 4)
+                : nullptr;
+    for (int k = 0; k < 16; ++k) a.cent[k] = tq ? tq4->c[k] : 0.f;
+    for (int k = 0; k < 8; ++k) {
+      sk.w[k] = tq ? tq4->sk[k] : 0u;
+      sv.w[k] = tq ? tq4->sv[k] : 0u;
+    }
   }
   int order[PF_MAX_REQ];
   int n = 0;
@@ -656,36 +807,43 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
   a.nreq = n;
   if (tiles > 0x7FFFFFFF || g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
   dim3 grid((unsigned)tiles, (unsigned)g.Hkv, (unsigned)num_splits);
-  if (g.D == 256) {
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(prefill_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               PfSmem<256>::TOTAL) != cudaSuccess)
-        return JF_ERR_CUDA;
-      attr = true;
-    }
-    prefill_kernel<256><<<grid, PF_THREADS, PfSmem<256>::TOTAL, stream>>>(a);
-  } else {
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(prefill_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               PfSmem<128>::TOTAL) != cudaSuccess)
-        return JF_ERR_CUDA;
-      attr = true;
-    }
-    prefill_kernel<128><<<grid, PF_THREADS, PfSmem<128>::TOTAL, stream>>>(a);
-  }
-  if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
-  if (num_splits > 1) {
-    const int64_t rows = total_rows * Hq;
-    const int64_t blocks = (rows + 7) / 8;
-    if (blocks > 0x7FFFFFFF) return JF_ERR_UNSUPPORTED;
+  const int64_t rows = total_rows * Hq;
+  const int64_t rblocks = (rows + 7) / 8;   // 8 warps per CTA, one row each
+  if (rblocks > 0x7FFFFFFF) return JF_ERR_UNSUPPORTED;
+  if (tq) {   // rotated queries first
     if (g.D == 256)
-      prefill_merge_kernel<256><<<(unsigned)blocks, 256, 0, stream>>>(
-          a.part_ml, a.part_o, static_cast<uint16_t*>(out), rows, num_splits);
+      prefill_rotate_q_kernel<256><<<(unsigned)rblocks, 256, 0, stream>>>(
+          static_cast<const uint16_t*>(q), const_cast<float*>(a.qrot), rows, sk);
     else
-      prefill_merge_kernel<128><<<(unsigned)blocks, 256, 0, stream>>>(
-          a.part_ml, a.part_o, static_cast<uint16_t*>(out), rows, num_splits);
+      prefill_rotate_q_kernel<128><<<(unsigned)rblocks, 256, 0, stream>>>(
+          static_cast<const uint16_t*>(q), const_cast<float*>(a.qrot), rows, sk);
+    if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
+  }
+  int st;
+  if (g.D == 256)
+    st = tq ? launch_pf<256, JF_FMT_TQ4>(grid, a, stream)
+            : launch_pf<256, JF_FMT_AFFINE4_G64>(grid, a, stream);
+  else
+    st = tq ? launch_pf<128, JF_FMT_TQ4>(grid, a, stream)
+            : launch_pf<128, JF_FMT_AFFINE4_G64>(grid, a, stream);
+  if (st) return st;
+  if (num_splits > 1 || tq) {
+    uint16_t* o = static_cast<uint16_t*>(out);
+    if (g.D == 256) {
+      if (tq)
+        prefill_merge_kernel<256, true><<<(unsigned)rblocks, 256, 0, stream>>>(
+            a.part_ml, a.part_o, o, rows, num_splits, sv);
+      else
+        prefill_merge_kernel<256, false><<<(unsigned)rblocks, 256, 0, stream>>>(
+            a.part_ml, a.part_o, o, rows, num_splits, sv);
+    } else {
+      if (tq)
+        prefill_merge_kernel<128, true><<<(unsigned)rblocks, 256, 0, stream>>>(
+            a.part_ml, a.part_o, o, rows, num_splits, sv);
+      else
+        prefill_merge_kernel<128, false><<<(unsigned)rblocks, 256, 0, stream>>>(
+            a.part_ml, a.part_o, o, rows, num_splits, sv);
+    }
     if (cudaGetLastError() != cudaSuccess) return JF_ERR_CUDA;
   }
   return JF_OK;
@@ -697,7 +855,8 @@ int launch_prefill(const Geom& g, const jf_kv_pool& pool, const CUtensorMap&,
                    void* workspace, cudaStream_t stream) {
   const int64_t row0 = 0;
   return launch_prefill_batch(g, pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1, Hq,
-                              softmax_scale, causal, out, workspace, stream, 1, chunk_len);
+                              softmax_scale, causal, out, workspace, stream, 1, chunk_len,
+                              nullptr);
 }
 
 }  // namespace jfkv

@@ -162,33 +162,6 @@ __device__ __forceinline__ void load_bf16(const uint16_t* src, float (&x)[E]) {
   }
 }
 
-// In-place unnormalized Walsh-Hadamard transform (Sylvester order) of a
-// vector spread over a warp, lane l holding elements E l .. E l + E - 1.
-template <typename T, int E>
-__device__ __forceinline__ void warp_fwht(T (&u)[E], int lane) {
-#pragma unroll
-  for (int h = 1; h < E; h <<= 1) {
-#pragma unroll
-    for (int i = 0; i < E; ++i) {
-      if (!(i & h)) {
-        const T a = u[i], b = u[i + h];
-        u[i] = a + b;
-        u[i + h] = a - b;
-      }
-    }
-  }
-#pragma unroll
-  for (int m = 1; m < 32; m <<= 1) {
-    // lower lane: u + o; upper lane: o - u (one rounding either way)
-    const T sg = (lane & m) ? T(-1) : T(1);
-#pragma unroll
-    for (int i = 0; i < E; ++i) {
-      const T o = __shfl_xor_sync(0xffffffffu, u[i], m);
-      u[i] = fma(u[i], sg, o);
-    }
-  }
-}
-
 // Count of the 15 ascending thresholds T_k with u > T_k, by a branch-free
 // 4-level search, and the thresholds bracketing u (lo < u <= hi; -inf / +inf
 // past the ends).

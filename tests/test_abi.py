@@ -159,7 +159,7 @@ def test_tq4_bad_codecs_and_unsupported_entry_points():
     assert L.jf_paged_decode_append_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, FAKE, FAKE, 8,
                                          0.1, FAKE, FAKE, 1 << 20, 4, None) == B.JF_ERR_UNSUPPORTED
     assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 16, 8, 0.1, 1, FAKE, FAKE, 256,
-                                   None) == B.JF_ERR_UNSUPPORTED
+                                   None) == B.JF_ERR_WORKSPACE_TOO_SMALL   # TQ4 needs more
     assert L.jf_paged_decode_attn_noalloc(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 8, 0.1, FAKE, 4,
                                           None, None) == B.JF_ERR_UNSUPPORTED
     # checkpoint sizes use the TQ4 page record
@@ -185,7 +185,10 @@ def test_prefill_batch_rejects_bad_arguments():
     assert call(clen=(I * 2)(0, 0)) == B.JF_OK                     # nothing to do
     assert call(splits=0) == B.JF_ERR_INVALID_ARG
     need = L.jf_prefill_batch_workspace_bytes
-    n = need(32, 8, 128, 4)
+    n = need(0, 32, 8, 128, 4)
     assert n == 256 + (32 * 8 * 4 * 8 + 255) // 256 * 256 + 32 * 8 * 4 * 128 * 4
-    assert need(32, 8, 128, 1) == 256 and need(32, 8, 96, 4) == 0
+    assert need(0, 32, 8, 128, 1) == 256 and need(0, 32, 8, 96, 4) == 0
+    # TQ4: partials even unsplit, plus the rotated queries
+    assert need(1, 32, 8, 128, 1) == 256 + (32 * 8 * 8 + 255) // 256 * 256 + 2 * 32 * 8 * 128 * 4
+    assert need(5, 32, 8, 128, 1) == 0
     assert call(splits=4, wsb=n - 1) == B.JF_ERR_WORKSPACE_TOO_SMALL

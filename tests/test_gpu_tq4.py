@@ -315,3 +315,59 @@ def test_tq4_decode_full_window_256k_one_head():
             o4, o1 = L4.norm_offset(kind, kvh, 0), L1.norm_offset(kind, 0, 0)
             assert np.array_equal(gp[page, o4:o4 + 2 * geo.page_size],
                                   opool[page, o1:o1 + 2 * geo.page_size])
+
+
+# --------------------------------------------------------------------------
+# prefill chunk attention over TQ4 pages
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("Hq,Hkv,D,P,q_start,C,causal", [
+    (8, 2, 128, 256, 0, 256, True),
+    (8, 2, 128, 64, 300, 77, True),
+    (24, 4, 256, 256, 1000, 130, True),
+    (24, 4, 256, 128, 517, 200, False),
+    (4, 4, 256, 64, 100, 129, True),      # G = 1
+])
+def test_tq4_prefill_matches_oracle(Hq, Hkv, D, P, q_start, C, causal):
+    total = q_start + C
+    case = make_case(700 + Hq + total, Hq, Hkv, D, P, [total], outliers=True)
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    q = synth.normal_bf16(synth.generator(8 + C), (C, Hq, D))
+    scale = 1 / math.sqrt(D)
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = jf.prefill_batch_workspace(C, Hq, D, 1, device=DEV, format=jf.JF_FMT_TQ4)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), q_start, scale, causal,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    ref = OT.prefill_chunk(ref_pool, lay, case.page_table[0].numpy(), bits(q), q_start, scale,
+                           causal=causal)
+    assert_attention_close(out, ref)
+
+
+@pytest.mark.parametrize("spans,splits", [
+    ([(3000, 64), (0, 40), (700, 150)], 1),
+    ([(3000, 64), (0, 40), (700, 150)], 5),
+])
+def test_tq4_prefill_batch_with_splits_matches_oracle(spans, splits):
+    Hq, Hkv, D, P = 24, 4, 256, 256
+    totals = [a + c for a, c in spans]
+    case = make_case(800 + splits, Hq, Hkv, D, P, totals)
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    C = [c for _, c in spans]
+    qs = [a for a, _ in spans]
+    q = synth.normal_bf16(synth.generator(801), (sum(C), Hq, D))
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = jf.prefill_batch_workspace(sum(C), Hq, D, splits, device=DEV, format=jf.JF_FMT_TQ4)
+    ws[256:] = 0xFF
+    jf.jf_prefill_batch_attn(pool, case.page_table.to(DEV), qs, C, q.to(DEV), 1 / 16, True, out,
+                             ws, num_splits=splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    row = 0
+    for b, (a0, c) in enumerate(spans):
+        ref = OT.prefill_chunk(ref_pool, lay, case.page_table[b].numpy(), bits(q[row:row + c]), a0,
+                               1 / 16)
+        assert_attention_close(out[row:row + c], ref)
+        row += c
