@@ -500,6 +500,18 @@ def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
     tp = _event_time(lambda: jf.jf_prefill_chunk_attn(pools[0], tables[0][0], qp, q0, 1 / 16, True,
                                                       op, wp, stream=stream), 5, stream)
     fl = 4 * Hq * D * (Cq * q0 + Cq * (Cq + 1) // 2)
+    # packed verifier over the first cache: q_len 2-4 tokens in one call
+    ver = {}
+    for Lq in (2, 3, 4):
+        qv = torch.randn(1, Lq, Hq, D, generator=g, device=dev).to(torch.bfloat16)
+        ov = torch.empty_like(qv)
+        sv = jf.default_verify_splits(1, Lq, Hq, Hkv, format=jf.JF_FMT_TQ4)
+        wv = jf.verify_workspace(1, Lq, Hq, Hkv, D, sv, device=dev)
+        tv = _event_time(lambda: jf.jf_paged_verify_attn(pools[0], tables[0], c, qv, 1 / 16, ov,
+                                                         wv, sv, stream=stream), 10, stream)
+        stream.synchronize()
+        assert jf.workspace_status(wv) == 0
+        ver[f"q_len_{Lq}"] = {"us": tv * 1e3, "splits": sv}
     stream.synchronize()
     assert jf.workspace_status(ws) == 0 and int(err.item()) == 0 and jf.workspace_status(wp) == 0
     bpp = 2 * Hkv * (D // 2 + 2)
@@ -510,7 +522,8 @@ def _bench_tq4(jf, synth, dev, stream, peaks_gbs, copies=8):
            "alg_bytes_per_call": alg, "traffic": measured_traffic("tq4_split_kernel<256>"),
            "append_2048_rows_us": ta * 1e3,
            "append_GBps": (2048 * Hkv * D * 2 * 2 + 2048 * bpp) / (ta / 1e3) / 1e9,
-           "prefill_2048_at_30720_ms": tp, "prefill_TFLOPs": fl / (tp / 1e3) / 1e12}
+           "prefill_2048_at_30720_ms": tp, "prefill_TFLOPs": fl / (tp / 1e3) / 1e12,
+           "verify": ver}
     del pools
     return res
 

@@ -198,8 +198,10 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
  * fp16 centroids in fp16 tensor-core products with fp32 accumulation, scores
  * are scaled by the K norms, probabilities times V norm times 2^-8 enter
  * fp16 products, and the accumulated output is rotated back by S_V H / sqrt(D)
- * in fp32.  The verifier, the fused append and the no-workspace variant
- * return JF_ERR_UNSUPPORTED for TQ4 pools.
+ * in fp32.  jf_paged_verify_attn and jf_paged_decode_append_attn take TQ4
+ * pools the same way (the fused step encodes the new rows exactly as
+ * jf_kv_quantize_append does); the no-workspace variant returns
+ * JF_ERR_UNSUPPORTED for them.
  */
 int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int32_t pt_stride,
                          const int32_t* context_lens, int32_t batch, const void* q,

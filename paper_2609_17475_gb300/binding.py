@@ -336,12 +336,14 @@ def verify_workspace(batch, q_len, num_q_heads, num_kv_heads, head_dim, num_spli
 
 
 def default_verify_splits(batch: int, q_len: int, num_q_heads: int, num_kv_heads: int,
-                          device=None) -> int:
+                          device=None, format: int = JF_FMT_AFFINE4_G64) -> int:
     """Split cap for the verifier: each split of a KV head runs
-    ceil(G * q_len / 8) CTAs, so fewer splits fill the GPU."""
+    ceil(G * q_len / 8) CTAs, so fewer splits fill the GPU (two split CTAs per
+    SM for the affine format, one for TQ4)."""
     nt = -(-(num_q_heads // num_kv_heads) * q_len // 8)
     props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    per = (2 * props.multi_processor_count) // (batch * num_kv_heads * nt)   # one full wave
+    slots = (1 if format == JF_FMT_TQ4 else 2) * props.multi_processor_count
+    per = slots // (batch * num_kv_heads * nt)   # one full wave
     return max(1, per if batch == 1 else per + 2)
 
 

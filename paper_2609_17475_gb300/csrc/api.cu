@@ -25,7 +25,8 @@ int launch_tq4_append(const Geom&, const jf_kv_pool&, const Tq4Params&, const in
                       int32_t*, cudaStream_t);
 int launch_tq4_decode(const Geom&, const jf_kv_pool&, const CUtensorMap&, const Tq4Params&,
                       const int32_t*, int32_t, const int32_t*, int32_t, const void*, int32_t,
-                      float, void*, void*, int32_t, cudaStream_t);
+                      float, void*, void*, int32_t, cudaStream_t, const void*, const void*,
+                      int32_t);
 int decode_box_rows();
 int launch_prefill(const Geom&, const jf_kv_pool&, const CUtensorMap&, const int32_t*,
                    const void*, int32_t, int32_t, int32_t, float, int32_t, void*, void*,
@@ -177,8 +178,7 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
                          const void* v_new, const void* q, int32_t num_q_heads,
                          float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
                          int32_t num_splits, void* stream, int32_t q_len = 1) {
-  // TQ4 pools: single-query decode without the fused append
-  int st = (q_len == 1 && !k_new) ? check_pool_any(pool) : check_pool(pool);
+  int st = check_pool_any(pool);
   if (st) return st;
   if (!page_table || !context_lens || !q || !out || !workspace) return JF_ERR_INVALID_ARG;
   if (batch < 1 || batch > 65535 || pt_stride < 1 || num_q_heads < 1) return JF_ERR_INVALID_ARG;
@@ -204,7 +204,7 @@ static int decode_common(const jf_kv_pool* pool, const int32_t* page_table, int3
   if (pool->format == JF_FMT_TQ4) {
     return launch_tq4_decode(g, *pool, tmap, prm, page_table, pt_stride, context_lens, batch, q,
                              num_q_heads, softmax_scale, out, workspace, num_splits,
-                             static_cast<cudaStream_t>(stream));
+                             static_cast<cudaStream_t>(stream), k_new, v_new, q_len);
   }
   return launch_decode(g, *pool, tmap, page_table, pt_stride, context_lens, batch, q,
                        num_q_heads, softmax_scale, out, workspace, num_splits,

@@ -195,22 +195,15 @@ __device__ __forceinline__ void two_sum_acc(float& sh, float& sl, float b) {
   sl = __fadd_rn(sl, err);
 }
 
+// Encode one vector of D bf16 elements (src) with a whole warp: returns this
+// lane's E = D/32 indices (element E lane + e in bits 4e .. 4e+3) and sets
+// rho (the fp32 norm; every lane gets the same value).  kind 0: K, 1: V.
 template <int D>
-__global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, const Tq4Params prm) {
-  constexpr int E = D / 32;   // elements per lane
-  const int lane = threadIdx.x & 31;
-  const int64_t vec = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t total = (int64_t)a.n_rows * a.Hkv * 2;
-  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  if (vec >= total) return;   // whole warps
-  const int64_t row = vec / (2 * a.Hkv);
-  const int rem = (int)(vec % (2 * a.Hkv));
-  const int kind = rem / a.Hkv;
-  const int head = rem % a.Hkv;
-
+__device__ __forceinline__ uint32_t tq4_encode(const uint16_t* src, int kind, const Tq4Params& prm,
+                                               int lane, float& rho_out) {
+  constexpr int E = D / 32;
   float x[E];
-  load_bf16<E>((kind ? a.v : a.k) + (row * a.Hkv + head) * D + lane * E, x);
+  load_bf16<E>(src + lane * E, x);
   const uint32_t sbits = ((kind ? prm.sv : prm.sk)[(lane * E) >> 5]) >> ((lane * E) & 31);
 
   // rho = RN32(sqrt(s)), s the fp64 sum of squares.  Squares of bf16 values
@@ -297,6 +290,47 @@ __global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, 
     }
   }
 
+  rho_out = rho;
+  return word;
+}
+
+// Store a lane's indices and (lane 0) the fp16 norm into slot `vrow` (head *
+// P + slot) of a page record.
+template <int D>
+__device__ __forceinline__ void tq4_store(uint8_t* pg, int64_t codes_region, int64_t norm_region,
+                                          int kind, int64_t vrow, int lane, uint32_t word,
+                                          float rho) {
+  constexpr int E = D / 32;
+  uint8_t* dst = pg + kind * codes_region + vrow * (D / 2);
+  if constexpr (E == 8)
+    reinterpret_cast<uint32_t*>(dst)[lane] = word;
+  else
+    reinterpret_cast<uint16_t*>(dst)[lane] = (uint16_t)word;
+  if (lane == 0) {
+    const __half h = __float2half_rn(fminf(rho, 65504.f));
+    *reinterpret_cast<uint16_t*>(pg + 2 * codes_region + kind * norm_region + vrow * 2) =
+        __half_as_ushort(h);
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, const Tq4Params prm) {
+  constexpr int E = D / 32;   // elements per lane
+  const int lane = threadIdx.x & 31;
+  const int64_t vec = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t total = (int64_t)a.n_rows * a.Hkv * 2;
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  if (vec >= total) return;   // whole warps
+  const int64_t row = vec / (2 * a.Hkv);
+  const int rem = (int)(vec % (2 * a.Hkv));
+  const int kind = rem / a.Hkv;
+  const int head = rem % a.Hkv;
+
+  float rho;
+  const uint32_t word = tq4_encode<D>((kind ? a.v : a.k) + (row * a.Hkv + head) * D, kind, prm,
+                                       lane, rho);
+
   const int32_t req = a.row_req[row];
   const int32_t pos = a.row_pos[row];
   if (req < 0 || req >= a.num_requests || pos < 0 || pos / a.P >= a.pt_stride) {
@@ -308,18 +342,8 @@ __global__ void __launch_bounds__(256) tq4_append_kernel(const Tq4AppendArgs a, 
     if (lane == 0) flag_error(a.err, JF_DEV_ERR_PAGE_ID);
     return;
   }
-  uint8_t* pg = a.pool + (int64_t)page * a.page_bytes;
-  const int64_t vrow = (int64_t)head * a.P + pos % a.P;
-  uint8_t* dst = pg + kind * a.codes_region + vrow * (D / 2);
-  if constexpr (E == 8)
-    reinterpret_cast<uint32_t*>(dst)[lane] = word;
-  else
-    reinterpret_cast<uint16_t*>(dst)[lane] = (uint16_t)word;
-  if (lane == 0) {
-    const __half h = __float2half_rn(fminf(rho, 65504.f));
-    *reinterpret_cast<uint16_t*>(pg + 2 * a.codes_region + kind * a.norm_region + vrow * 2) =
-        __half_as_ushort(h);
-  }
+  tq4_store<D>(a.pool + (int64_t)page * a.page_bytes, a.codes_region, a.norm_region, kind,
+               (int64_t)head * a.P + pos % a.P, lane, word, rho);
 }
 
 int launch_tq4_append(const Geom& g, const jf_kv_pool& pool, const Tq4Params& prm,
@@ -423,14 +447,16 @@ __device__ __forceinline__ float h2f(const uint8_t* p) {
 }
 
 // One 32-position chunk; positions >= nvalid get -inf logits and zero weights
-// (their bytes are never trusted).  The masks are plain selects, so full and
+// (their bytes are never trusted), and the rows of this thread's columns 2c
+// and 2c+1 see only positions < nv0 and < nv1 (the verifier's causal limits;
+// both are nvalid for a single query).  The masks are plain selects, so full and
 // partial chunks share one body (the body is large: one copy keeps it in the
 // instruction cache).
-template <int D>
+template <int D, bool VER>
 __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[D / 32][2][2],
                                           uint32_t kc, const uint8_t* kn, uint32_t lut_lane,
                                           const uint32_t (&koff)[D / 64], float cS, int r,
-                                          int nvalid) {
+                                          int nvalid, int nv0, int nv1) {
   constexpr int CB = D / 2;
   constexpr int NJ = DTOK / 16;
   constexpr int NCH = D / 64;
@@ -462,10 +488,17 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
     }
     const int ta = 16 * j + r, tb = ta + 8;
     const float na = h2f(kn + 2 * ta) * cS, nb = h2f(kn + 2 * tb) * cS;
-    sc[j][0] = (ta < nvalid) ? acc[0] * na : NEG_INF;
-    sc[j][1] = (ta < nvalid) ? acc[1] * na : NEG_INF;
-    sc[j][2] = (tb < nvalid) ? acc[2] * nb : NEG_INF;
-    sc[j][3] = (tb < nvalid) ? acc[3] * nb : NEG_INF;
+    if constexpr (VER) {
+      sc[j][0] = (ta < nv0) ? acc[0] * na : NEG_INF;
+      sc[j][1] = (ta < nv1) ? acc[1] * na : NEG_INF;
+      sc[j][2] = (tb < nv0) ? acc[2] * nb : NEG_INF;
+      sc[j][3] = (tb < nv1) ? acc[3] * nb : NEG_INF;
+    } else {
+      sc[j][0] = (ta < nvalid) ? acc[0] * na : NEG_INF;
+      sc[j][1] = (ta < nvalid) ? acc[1] * na : NEG_INF;
+      sc[j][2] = (tb < nvalid) ? acc[2] * nb : NEG_INF;
+      sc[j][3] = (tb < nvalid) ? acc[3] * nb : NEG_INF;
+    }
   }
 
   // ---- online softmax with a lazily moved reference maximum -------------
@@ -544,7 +577,10 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
   }
 }
 
-template <int D>
+// VER: packed verifier (a.L > 1 query tokens, per-row causal limits; each CTA
+// holds 8 of the KV head's G * L (token, head) rows); otherwise decode.  APP:
+// the step's new K/V row is appended first (a.knew, a.vnew).
+template <int D, bool VER, bool APP>
 __global__ void __launch_bounds__(TQ_WARPS * 32, 1)
 tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
                  const Tq4Params prm) {
@@ -559,11 +595,22 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem_raw + L::BAR_OFF);
   int* misc = reinterpret_cast<int*>(smem_raw + L::MISC_OFF);
 
-  const int kvh = blockIdx.y;
+  const int kvh = VER ? (int)blockIdx.y / a.NT : (int)blockIdx.y;
+  const int nt = VER ? (int)blockIdx.y % a.NT : 0;
+  const int rows = VER ? min(8, a.G * a.L - 8 * nt) : a.G;
+  // row k of this CTA: query token (8 nt + k) / G, head (8 nt + k) % G; its
+  // q, out and partial row within the request
+  auto row_of = [&](int k) {
+    if constexpr (VER) {
+      const int gr = 8 * nt + k;
+      return (gr / a.G) * a.Hq + kvh * a.G + gr % a.G;
+    } else {
+      return kvh * a.G + k;
+    }
+  };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
   const bool direct = (a.num_splits == 1);
-  const int rows = a.G;
   const bool aligned = (smem_u32(smem_raw) & 1023) == 0;
   // setup that reads only kernel parameters
   if (aligned) {
@@ -608,7 +655,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   if (split >= nsplit) {
     if (direct && split == 0) {
       for (int i = threadIdx.x; i < rows * D; i += blockDim.x)
-        a.out[((int64_t)b * a.HqL + kvh * a.G + i / D) * D + i % D] = 0;
+        a.out[((int64_t)b * a.HqL + row_of(i / D)) * D + i % D] = 0;
     }
     return;
   }
@@ -622,6 +669,28 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   const int my_n = (n_cta > warp) ? (n_cta - warp + TQ_WARPS - 1) / TQ_WARPS : 0;
   auto chunk_of = [&](int it) { return c_begin + warp + it * TQ_WARPS; };
 
+  if (APP && split == nsplit - 1) {   // owns the last chunk
+    // the step's new K (warp 0) and V (warp 1) rows go to position ctx - 1
+    // before this split's copies read the page
+    if (warp < 2 && ctx > 0) {
+      const int pos = ctx - 1;
+      float rho;
+      const uint32_t word = tq4_encode<D>((warp ? a.vnew : a.knew) + ((int64_t)b * a.Hkv + kvh) * D,
+                                          warp, prm, lane, rho);
+      const int pidx = pos >> a.log2P;
+      const int page = (pidx < a.pt_stride) ? a.page_table[(int64_t)b * a.pt_stride + pidx] : -1;
+      if (page < 0 || page >= a.num_pages) {
+        if (lane == 0) flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+      } else {
+        tq4_store<D>(const_cast<uint8_t*>(a.pool) + (int64_t)page * a.page_bytes, a.codes_region,
+                     a.sb_region, warp, (int64_t)kvh * a.P + (pos & (a.P - 1)), lane, word, rho);
+      }
+    }
+    fence_proxy_async_global();
+    __syncthreads();
+    fence_proxy_async_global();
+  }
+
   // ---- rotated queries q' = H S_K q / sqrt(D) (rows >= G stay zero) -------
   // warp h < 8 transforms head row h with shuffles (E elements per lane)
   constexpr int E = D / 32;
@@ -630,7 +699,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
 #pragma unroll
     for (int e = 0; e < E; ++e) x[e] = 0.f;
     if (warp < rows) {
-      load_bf16<E>(a.q + ((int64_t)b * a.HqL + kvh * a.G + warp) * D + lane * E, x);
+      load_bf16<E>(a.q + ((int64_t)b * a.HqL + row_of(warp)) * D + lane * E, x);
       const uint32_t sb = prm.sk[(lane * E) >> 5] >> ((lane * E) & 31);
 #pragma unroll
       for (int e = 0; e < E; ++e)
@@ -722,6 +791,13 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   for (int g = 0; g < NCH; ++g) koff[g] = swz<L::CB>(ld_t, 2 * g + ld_ch);
   const uint32_t lut_lane = smem_u32(lut_w) + 4u * lane;
 
+  // verifier causal limits: token i of L sees positions < ctx - L + 1 + i
+  int lim0 = ctx, lim1 = ctx;
+  if constexpr (VER) {
+    const int ctx_all = ctx - a.L + 1;
+    lim0 = min(ctx, ctx_all + (8 * nt + 2 * c) / a.G);
+    lim1 = min(ctx, ctx_all + (8 * nt + 2 * c + 1) / a.G);
+  }
   int done = 0;
   for (int it = 0; it < my_n; ++it) {
     const int s = it % TQ_STAGES;
@@ -735,7 +811,9 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     const int tokbase = chunk_of(it) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * TQ_STAGES + s) * 2 * L::CODE_BUF);
     const uint8_t* kn = norms + (warp * TQ_STAGES + s) * 2 * L::NORM_BUF;
-    tq4_chunk<D>(st, bq, kc, kn, lut_lane, koff, cS, r, ok ? min(ctx - tokbase, DTOK) : 0);
+    const int nv = ok ? min(ctx - tokbase, DTOK) : 0;
+    tq4_chunk<D, VER>(st, bq, kc, kn, lut_lane, koff, cS, r, nv,
+                      ok ? min(lim0 - tokbase, nv) : 0, ok ? min(lim1 - tokbase, nv) : 0);
     __syncwarp();
     if (it + TQ_STAGES < my_n) {
       fence_proxy_async_smem();
@@ -826,7 +904,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     const uint32_t sb = prm.sv[(lane * E) >> 5] >> ((lane * E) & 31);
 #pragma unroll
     for (int e = 0; e < E; ++e) x[e] *= ((sb >> e) & 1u) ? -osc : osc;
-    const int fr = kvh * a.G + h;
+    const int fr = row_of(h);
     const int d0 = lane * E;
     if (direct) {
       uint32_t w[E / 2];
@@ -854,11 +932,36 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   }
 }
 
+template <int D, bool VER, bool APP>
+static int launch_tq4_split(const cudaLaunchConfig_t& cfg0, const CUtensorMap& tmap,
+                            const DecodeArgs& a, const Tq4Params& prm) {
+  static bool attr = false;   // one per instantiation
+  if (!attr) {
+    if (cudaFuncSetAttribute(tq4_split_kernel<D, VER, APP>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Tq4Smem<D>::TOTAL) != cudaSuccess)
+      return JF_ERR_CUDA;
+    attr = true;
+  }
+  cudaLaunchConfig_t cfg = cfg0;
+  cfg.dynamicSmemBytes = Tq4Smem<D>::TOTAL;
+  return cudaLaunchKernelEx(&cfg, tq4_split_kernel<D, VER, APP>, tmap, a, prm) == cudaSuccess
+             ? JF_OK : JF_ERR_CUDA;
+}
+
+template <int D>
+static int launch_tq4_split_any(const cudaLaunchConfig_t& cfg, const CUtensorMap& tmap,
+                                const DecodeArgs& a, const Tq4Params& prm) {
+  if (a.L > 1) return launch_tq4_split<D, true, false>(cfg, tmap, a, prm);
+  if (a.knew) return launch_tq4_split<D, false, true>(cfg, tmap, a, prm);
+  return launch_tq4_split<D, false, false>(cfg, tmap, a, prm);
+}
+
 int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
                       const Tq4Params& prm, const int32_t* page_table, int32_t pt_stride,
                       const int32_t* context_lens, int32_t batch, const void* q, int32_t Hq,
                       float softmax_scale, void* out, void* workspace, int32_t num_splits,
-                      cudaStream_t stream) {
+                      cudaStream_t stream, const void* k_new, const void* v_new, int32_t q_len) {
   DecodeArgs a{};
   a.pool = static_cast<const uint8_t*>(pool.base);
   a.num_pages = g.num_pages;
@@ -871,18 +974,18 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   a.Hkv = g.Hkv;
   a.Hq = Hq;
   a.G = Hq / g.Hkv;
-  a.L = 1;
-  a.NT = 1;
-  a.HqL = Hq;
+  a.L = q_len;
+  a.NT = (a.G * q_len + 7) / 8;
+  a.HqL = q_len * Hq;
   a.page_table = page_table;
   a.pt_stride = pt_stride;
   a.ctx = context_lens;
   a.q = static_cast<const uint16_t*>(q);
-  a.knew = nullptr;
-  a.vnew = nullptr;
+  a.knew = static_cast<const uint16_t*>(k_new);
+  a.vnew = static_cast<const uint16_t*>(v_new);
   a.out = static_cast<uint16_t*>(out);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  const int64_t rows = (int64_t)batch * Hq * num_splits;
+  const int64_t rows = (int64_t)batch * q_len * Hq * num_splits;
   a.status = reinterpret_cast<int32_t*>(ws);
   a.part_ml = reinterpret_cast<float*>(ws + 256);
   a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
@@ -892,7 +995,7 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   a.balanced = (batch > 1 && batch <= 1024 && num_splits > 1) ? 1 : 0;
   a.budget = 1;
   if (a.balanced) {   // one CTA per SM in all
-    const int slots = (sm_count() + g.Hkv - 1) / g.Hkv;
+    const int slots = (sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
     const int64_t fit = (int64_t)batch * num_splits - batch;
     const int64_t cap = fit < slots ? fit : slots;
     a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);
@@ -901,35 +1004,15 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + batch), (unsigned)g.Hkv, 1u)
-                           : dim3((unsigned)num_splits, (unsigned)g.Hkv, (unsigned)batch);
+  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + batch), (unsigned)(g.Hkv * a.NT), 1u)
+                           : dim3((unsigned)num_splits, (unsigned)(g.Hkv * a.NT), (unsigned)batch);
   cfg.blockDim = dim3(TQ_WARPS * 32);
   cfg.stream = stream;
   cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  cudaError_t e;
-  if (g.D == 256) {
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(tq4_split_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               Tq4Smem<256>::TOTAL) != cudaSuccess)
-        return JF_ERR_CUDA;
-      attr = true;
-    }
-    cfg.dynamicSmemBytes = Tq4Smem<256>::TOTAL;
-    e = cudaLaunchKernelEx(&cfg, tq4_split_kernel<256>, tmap, a, prm);
-  } else {
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(tq4_split_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               Tq4Smem<128>::TOTAL) != cudaSuccess)
-        return JF_ERR_CUDA;
-      attr = true;
-    }
-    cfg.dynamicSmemBytes = Tq4Smem<128>::TOTAL;
-    e = cudaLaunchKernelEx(&cfg, tq4_split_kernel<128>, tmap, a, prm);
-  }
-  if (e != cudaSuccess) return JF_ERR_CUDA;
+  const int st = (g.D == 256) ? launch_tq4_split_any<256>(cfg, tmap, a, prm)
+                              : launch_tq4_split_any<128>(cfg, tmap, a, prm);
+  if (st) return st;
   if (num_splits > 1) return launch_decode_merge(a, g.D, batch, stream);
   return JF_OK;
 }

@@ -153,11 +153,13 @@ def test_tq4_bad_codecs_and_unsupported_entry_points():
     assert dec(_tq4_pool(bad)) == B.JF_ERR_INVALID_ARG
     assert L.jf_kv_quantize_append(ctypes.byref(_tq4_pool(bad)), FAKE, 4, 1, FAKE, FAKE, FAKE,
                                    FAKE, 5, None, None) == B.JF_ERR_INVALID_ARG
-    # entry points without TQ4 support
-    assert L.jf_paged_verify_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 2, 8, 0.1, FAKE, FAKE,
-                                  1 << 20, 4, None) == B.JF_ERR_UNSUPPORTED
-    assert L.jf_paged_decode_append_attn(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, FAKE, FAKE, 8,
-                                         0.1, FAKE, FAKE, 1 << 20, 4, None) == B.JF_ERR_UNSUPPORTED
+    # the verifier and the fused step validate the codec too; the no-workspace
+    # decode does not take TQ4 pools
+    assert L.jf_paged_verify_attn(ctypes.byref(_tq4_pool(bad)), FAKE, 4, FAKE, 1, FAKE, 2, 8, 0.1,
+                                  FAKE, FAKE, 1 << 20, 4, None) == B.JF_ERR_INVALID_ARG
+    assert L.jf_paged_decode_append_attn(ctypes.byref(_tq4_pool(bad)), FAKE, 4, FAKE, 1, FAKE,
+                                         FAKE, FAKE, 8, 0.1, FAKE, FAKE, 1 << 20, 4,
+                                         None) == B.JF_ERR_INVALID_ARG
     assert L.jf_prefill_chunk_attn(ctypes.byref(p), FAKE, FAKE, 0, 16, 8, 0.1, 1, FAKE, FAKE, 256,
                                    None) == B.JF_ERR_WORKSPACE_TOO_SMALL   # TQ4 needs more
     assert L.jf_paged_decode_attn_noalloc(ctypes.byref(p), FAKE, 4, FAKE, 1, FAKE, 8, 0.1, FAKE, 4,

@@ -260,16 +260,101 @@ def test_tq4_decode_after_gpu_append_and_split_invariance():
         assert_attention_close(o, ref)
 
 
-def test_tq4_rejected_by_entry_points_without_tq4_support():
+def test_tq4_no_workspace_decode_is_rejected():
     case = make_case(3, 8, 2, 128, 64, [100])
     pool = gpu_pool(case)
-    ws = jf.verify_workspace(1, 2, 8, 2, 128, 2, device=DEV)
-    q2 = torch.zeros(1, 2, 8, 128, dtype=torch.bfloat16, device=DEV)
+    q = torch.zeros(1, 8, 128, dtype=torch.bfloat16, device=DEV)
     with pytest.raises(jf.JfError) as e:
-        jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
-                                torch.tensor([100], dtype=torch.int32, device=DEV), q2, 0.1,
-                                torch.empty_like(q2), ws, 2)
+        jf.jf_paged_decode_attn_noalloc(pool, case.page_table.to(DEV),
+                                        torch.tensor([100], dtype=torch.int32, device=DEV), q,
+                                        0.1, torch.empty_like(q), 2)
     assert e.value.status == jf.binding.JF_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,L,splits", [
+    (24, 4, 256, 256, [5000], 2, None),
+    (24, 4, 256, 128, [3000, 40], 4, None),       # G * L = 24: 3 n-tiles, batch plan
+    (8, 2, 128, 64, [700], 3, 5),
+    (16, 2, 256, 256, [2100, 4], 4, 3),           # G * L = 32; a context of exactly q_len
+])
+def test_tq4_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
+    case = make_case(900 + sum(ctx) + L, Hq, Hkv, D, P, ctx)
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    B = len(ctx)
+    q = synth.normal_bf16(synth.generator(910 + L), (B, L, Hq, D))
+    if splits is None:
+        splits = jf.default_verify_splits(B, L, Hq, Hkv, format=jf.JF_FMT_TQ4)
+    ws = jf.verify_workspace(B, L, Hq, Hkv, D, splits, device=DEV)
+    ws[256:] = 0xFF
+    out = torch.full((B, L, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    scale = 1 / math.sqrt(D)
+    jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
+                            torch.tensor(ctx, dtype=torch.int32, device=DEV), q.to(DEV), scale,
+                            out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    ref = np.stack([OT.prefill_chunk(ref_pool, lay, case.page_table[b].numpy(), bits(q[b]),
+                                     ctx[b] - L, scale) for b in range(B)])
+    assert_attention_close(out, ref)
+
+
+def test_tq4_verifier_with_one_token_is_decode():
+    case = make_case(78, 24, 4, 256, 256, [3333, 1234])
+    _, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    out_d = gpu_decode(case, pool, 9)
+    ws = jf.verify_workspace(2, 1, 24, 4, 256, 9, device=DEV)
+    out_v = torch.empty((2, 1, 24, 256), dtype=torch.bfloat16, device=DEV)
+    jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
+                            torch.tensor(case.ctx, dtype=torch.int32, device=DEV),
+                            case.q.view(2, 1, 24, 256).to(DEV), 1 / 16, out_v, ws, 9)
+    torch.cuda.synchronize()
+    assert torch.equal(out_v.view(2, 24, 256), out_d)
+
+
+@pytest.mark.parametrize("Hq,Hkv,D,P,ctx,splits", [
+    (24, 4, 256, 256, [5000, 257, 1], 38),   # new rows mid-page, at slot 0 of a page, alone
+    (8, 2, 128, 64, [64, 65, 999], 4),
+    (16, 2, 256, 128, [3000], 1),            # one split writes and reads directly
+])
+def test_tq4_fused_append_decode_equals_append_then_decode(Hq, Hkv, D, P, ctx, splits):
+    case = make_case(950 + sum(ctx), Hq, Hkv, D, P, ctx)
+    lay = oracle_layout(case)
+    req, pos = case.req.numpy(), case.pos.numpy()
+    last = np.array([np.nonzero(req == b)[0].max() for b in range(len(ctx))])
+    keep = np.setdiff1d(np.arange(len(req)), last)
+    prefix = OQ.new_pool(lay, case.num_pages, fill=0xFF)
+    OQ.append(prefix, lay, case.page_table.numpy(), req[keep], pos[keep], bits(case.k[keep]),
+              bits(case.v[keep]))
+    full = OQ.new_pool(lay, case.num_pages, fill=0xFF)
+    OQ.append(full, lay, case.page_table.numpy(), req, pos, bits(case.k), bits(case.v))
+    k_new = case.k[last].contiguous()
+    v_new = case.v[last].contiguous()
+    B = len(ctx)
+    pt = case.page_table.to(DEV)
+    ctx_t = torch.tensor(ctx, dtype=torch.int32, device=DEV)
+    scale = 1 / math.sqrt(D)
+    pool_a = pool_from_numpy(case, prefix)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool_a, pt, torch.arange(B, dtype=torch.int32, device=DEV),
+                             (ctx_t - 1).contiguous(), k_new.to(DEV), v_new.to(DEV), err)
+    out_a = torch.full((B, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws_a = jf.decode_workspace(B, Hq, Hkv, D, splits, device=DEV)
+    jf.jf_paged_decode_attn(pool_a, pt, ctx_t, case.q.to(DEV), scale, out_a, ws_a, splits)
+    pool_b = pool_from_numpy(case, prefix)
+    out_b = torch.full((B, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws_b = jf.decode_workspace(B, Hq, Hkv, D, splits, device=DEV)
+    ws_b[256:] = 0xFF
+    jf.jf_paged_decode_append_attn(pool_b, pt, ctx_t, k_new.to(DEV), v_new.to(DEV),
+                                   case.q.to(DEV), scale, out_b, ws_b, splits)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws_a) == 0 and jf.workspace_status(ws_b) == 0
+    assert torch.equal(pool_a.data, pool_b.data)
+    assert np.array_equal(pool_b.data.cpu().numpy(), full)       # bit-exact encode on append
+    assert torch.equal(out_a, out_b)
+    ref = OT.paged_decode(full, lay, case.page_table.numpy(), ctx, bits(case.q), scale)
+    assert_attention_close(out_b, ref)
 
 
 def test_tq4_decode_full_window_256k_one_head():
