@@ -437,9 +437,10 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     Tile ta, tb, tcur;
     bool ok = true;
     int pg_next = page_of(2);
+    // The loads of tile j + 2 are issued after tile j's arrive: a release
+    // waits for every earlier access of the warp, so loads still in flight
+    // would hold the arrive back by a memory latency.
     auto step = [&](int j, const Tile& cur, Tile& nxt) {
-      if (j + 2 < ntiles) load_tile(j + 2, pg_next, nxt);
-      pg_next = page_of(j + 3);
       const int kbuf = j % PF_KVBUF;
       if (j >= PF_KVBUF &&
           !tc::wait_cluster(&pv_done[kbuf], ((j - PF_KVBUF) / PF_KVBUF) & 1)) { ok = false; return; }
@@ -447,6 +448,8 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) tc::arrive_cluster(&kv_full[kbuf], 0);
+      if (j + 2 < ntiles) load_tile(j + 2, pg_next, nxt);
+      pg_next = page_of(j + 3);
     };
     if (ntiles > 0) load_tile(0, page_of(0), ta);
     if (ntiles > 1) load_tile(1, page_of(1), tb);

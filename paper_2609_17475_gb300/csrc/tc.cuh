@@ -110,12 +110,18 @@ __device__ __forceinline__ void cluster_sync() {
                "barrier.cluster.wait.acquire.aligned;\n" ::: "memory");
 }
 
-// Release-arrive on the mbarrier at this shared offset in CTA `rank` of the
-// cluster (the own CTA included).
+// Arrive on the mbarrier at this shared offset in CTA `rank` of the cluster
+// (the own CTA included).  The data it publishes is this CTA's own shared
+// memory (made visible to the tensor core by fence.proxy.async first) or its
+// own TMEM (tcgen05.wait::st and tcgen05.fence::before_thread_sync first), so
+// a CTA-scope release is enough: it orders the shared-memory stores before
+// the arrive without draining the SM's outstanding global accesses, which a
+// cluster-scope release waits for (measured: ~1,000 cycles per arrive in the
+// prefill kernel under load).
 __device__ __forceinline__ void arrive_cluster(uint64_t* bar, uint32_t rank) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n"
+  asm volatile("mbarrier.arrive.release.cta.shared::cluster.b64 _, [%0];\n"
                ::"r"(remote) : "memory");
 }
 
