@@ -20,23 +20,31 @@
 // Warp roles (each CTA):
 //   warp 0      TMEM allocation (512 columns, pair-wide); in CTA 0, lane 0
 //               issues every tcgen05.mma.cta_group::2 of the pair:
-//                 S_j  = Q  K_j^T   (A = Q in TMEM, B = K_j smem, K-major)
-//                 O   += P_j V_j    (A = P_j in TMEM, B = V_j smem, MN-major)
+//                 S_i  = Q  [K_2i K_2i+1]^T  (A = Q in TMEM, B = the K halves
+//                        of tiles 2i and 2i + 1 in smem, K-major, N = 128)
+//                 O   += P_j V_j             (A = P_j in smem, K-major;
+//                        B = V_j smem, MN-major)
 //               and commits to the barrier of both CTAs (multicast).
-//               TMEM columns: O [0, D), two S/P buffers of 64, Q [D + 128, +D/2);
-//               P_j (fp16) overwrites the first half of S_j once it is read.
+//               TMEM columns: O [0, D), S of a tile pair [D, D + 128),
+//               Q [D + 128, +D/2).  S over two tiles keeps the MMA at N = 128
+//               (an N = 64 pair MMA takes as long as an N = 128 one).
 //   warps 1-8   dequantize this CTA's halves of 64-position K/V tiles from
 //               the pool (page-table lookup, 4-bit codes -> fp16 integers
 //               through the mantissa of fp16 1024, then x = code * scale +
-//               bias with one fused multiply-add) into four 128B-swizzled
-//               half-tile buffers, one item (one position's code bytes of a
-//               64-wide block) per thread, loads running two tiles ahead;
-//               each warp then arrives on CTA 0's tile barrier.
+//               bias with one fused multiply-add) into 128B-swizzled
+//               buffers, one item (one position's code bytes of a 64-wide
+//               block) per thread, loads running two tiles ahead; warps 1-4
+//               write K halves into two pair buffers (free again once S of
+//               the pair two back is done), warps 5-8 V halves into four
+//               tile buffers (free once P V of the tile four back is done),
+//               each arriving on CTA 0's K-pair or V-tile barrier.
 //   warps 9-12  one thread per row: Q row -> TMEM at the start; online
-//               softmax on S (tcgen05.ld), P back to TMEM as fp16
-//               (tcgen05.st) and an arrive on CTA 0's P barrier; the running
-//               maximum is moved only when it grows by more than 2^8, and
-//               then O is rescaled in TMEM; finally O / l -> bf16 output.
+//               softmax on S (tcgen05.ld; after loading the second tile of a
+//               pair it frees the S columns for the next pair's MMA), P as
+//               fp16 into a shared-memory row (two P buffers) and an arrive
+//               on CTA 0's P barrier; the running maximum is moved only when
+//               it grows by more than 2^8, and then O is rescaled in TMEM;
+//               finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
 // 0,4,1,5,2,6,3,7 (the pairs one 32-bit word of codes yields); Q uses the same
 // order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
@@ -89,18 +97,24 @@ struct PrefillArgs {
   PfReq req[PF_MAX_REQ];
 };
 
-// Each CTA of a pair holds half of every K/V tile: K rows 32 r .. 32 r + 31
-// (all of head_dim, K-major) and V columns D/2 r .. D/2 (r + 1) (all 64
-// positions, MN-major), r = its rank in the pair.
+// Each CTA of a pair holds half of every K/V tile: K positions 32 r .. 32 r +
+// 31 (all of head_dim, K-major) and V columns D/2 r .. D/2 (r + 1) (all 64
+// positions, MN-major), r = its rank in the pair.  The K halves of tiles 2i
+// and 2i + 1 share a pair buffer (rows 32 (j & 1) + t), so one N = 128 MMA
+// computes S for both.  P of a tile is this CTA's 128 rows x 64 positions
+// (fp16, K-major).
 template <int D, int FMT>
 struct PfSmem {
-  static constexpr int KT_BYTES = (PF_BN / 2) * D * 2;   // [D/64][32 rows][128 B]
+  static constexpr int KP_BYTES = PF_BN * D * 2;         // [D/64][64 rows][128 B]
   static constexpr int VT_BYTES = PF_BN * (D / 2) * 2;   // [D/128][64 rows][128 B]
+  static constexpr int P_BYTES = PF_BM * PF_BN * 2;      // [128 rows][128 B]
   static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = PF_KVBUF * KT_BYTES;
-  static constexpr int OFF_BAR = OFF_V + PF_KVBUF * VT_BYTES;
+  static constexpr int OFF_V = 2 * KP_BYTES;
+  static constexpr int OFF_P = OFF_V + PF_KVBUF * VT_BYTES;
+  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
   static constexpr int OFF_LUT = OFF_BAR + 256;   // TQ4 centroid table (lane-replicated)
   static constexpr int TOTAL = 1024 + OFF_LUT + (FMT == JF_FMT_TQ4 ? 256 * 32 * 4 : 0);
+  static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
 
 __device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
@@ -162,7 +176,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   // (64 positions x NKB/2 blocks x 2/UPI units): one per dequant thread
   static_assert((PF_BN / 2) * NKB * 2 / UPI == 128 && PF_BN * (NKB / 2) * 2 / UPI == 128,
                 "one item per dequant thread");
-  constexpr uint32_t IDQK = tc::idesc_f16_f32(2 * PF_BM, PF_BN, 0, 0);
+  constexpr uint32_t IDQK = tc::idesc_f16_f32(2 * PF_BM, 2 * PF_BN, 0, 0);   // a tile pair
   constexpr uint32_t IDPV = tc::idesc_f16_f32(2 * PF_BM, D, 0, 1);
 
   extern __shared__ uint8_t smraw[];
@@ -170,12 +184,15 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
                                            ~static_cast<uintptr_t>(1023));
   uint8_t* sK = sm + L::OFF_K;
   uint8_t* sV = sm + L::OFF_V;
+  uint8_t* sP = sm + L::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::OFF_BAR);
-  uint64_t* kv_full = bars + 0;                // [PF_KVBUF] on CTA 0: both CTAs' halves stored
-  uint64_t* pv_done = bars + PF_KVBUF;         // [PF_KVBUF] both CTAs: P V of the tile done
-  uint64_t* s_full = bars + 2 * PF_KVBUF;      // [2] both CTAs: S ready
-  uint64_t* p_full = bars + 2 * PF_KVBUF + 2;  // [2] on CTA 0: both CTAs' P stored
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * PF_KVBUF + 4);
+  uint64_t* k_full = bars + 0;     // [2] on CTA 0: K halves of a tile pair stored
+  uint64_t* v_full = bars + 2;     // [PF_KVBUF] on CTA 0: both CTAs' V halves stored
+  uint64_t* pv_done = bars + 6;    // [PF_KVBUF] both CTAs: P V of the tile done
+  uint64_t* s_full = bars + 10;    // [2] both CTAs: S of pair i done (index i & 1)
+  uint64_t* s_free = bars + 12;    // on CTA 0: both CTAs' softmax warps loaded S
+  uint64_t* p_full = bars + 13;    // [4] on CTA 0: both CTAs' P stored (tile j & 3)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = tc::cluster_rank();
@@ -211,14 +228,17 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   const int ntiles = je - jb;
 
   if (threadIdx.x == 0) {
+    static_assert(PF_KVBUF == 4, "barrier layout");
     for (int i = 0; i < PF_KVBUF; ++i) {
-      mbar_init(&kv_full[i], 2 * PF_DQ_WARPS);
+      mbar_init(&v_full[i], PF_DQ_WARPS);        // the 4 V warps of each CTA
       mbar_init(&pv_done[i], 1);
-    }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&s_full[i], 1);
       mbar_init(&p_full[i], 2 * PF_SM_WARPS);
     }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&k_full[i], 2 * PF_DQ_WARPS);    // the 4 K warps of each CTA, twice
+      mbar_init(&s_full[i], 1);
+    }
+    mbar_init(s_free, 2 * PF_SM_WARPS);
     fence_barrier_init();
   }
   if constexpr (TQ) {   // centroid pair of code byte b for lane l: word b * 32 + l
@@ -233,7 +253,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   tc::fence_after();
   const uint32_t tbase = *tmem_slot;
   const uint32_t tO = tbase;
-  const uint32_t tS = tbase + D;               // two buffers of PF_BN columns
+  const uint32_t tS = tbase + D;               // S of a tile pair, 2 PF_BN columns
   const uint32_t tQ = tbase + D + 2 * PF_BN;   // D/2 columns of f16 pairs
 
   // ---- softmax warps: their Q row -> TMEM (fp16, pre-multiplied by
@@ -313,33 +333,43 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   if (warp == 0) {
     // ================= MMA issuer (CTA 0 of the pair) =================
     if (rank == 0 && lane == 0) {
-      const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV);
+      const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV), paddr = smem_u32(sP);
       bool ok = true;
       auto pv = [&](int j) {   // j: local tile index within this split
-        const int sb = j & 1, kb = j % PF_KVBUF;
-        if (!tc::wait_cluster(&p_full[sb], (j >> 1) & 1)) { ok = false; return; }
+        const int kb = j % PF_KVBUF;
+        if (!tc::wait_cluster(&v_full[kb], (j / PF_KVBUF) & 1) ||
+            !tc::wait_cluster(&p_full[j & 3], (j >> 2) & 1)) { ok = false; return; }
         tc::fence_after();
 #pragma unroll
         for (int k = 0; k < PF_BN / 16; ++k)
-          tc::mma2_ts(tO, tS + sb * PF_BN + 8 * k,
+          tc::mma2_ss(tO, tc::sdesc_sw128(paddr + (j & 1) * L::P_BYTES + k * 32, 16, 1024),
                       tc::sdesc_sw128(vaddr + kb * L::VT_BYTES + k * 2048, PF_BN * 128, 1024),
                       IDPV, (j > 0 || k > 0) ? 1u : 0u);
         tc::commit2_both(&pv_done[kb]);
       };
-      for (int j = 0; j < ntiles && ok; ++j) {
-        const int sb = j & 1, kb = j % PF_KVBUF;
-        if (!tc::wait_cluster(&kv_full[kb], (j / PF_KVBUF) & 1)) { ok = false; break; }
-        tc::fence_after();
+      // Pair i: S of tiles 2i, 2i + 1 (S column n = K row n of CTA 0 for n <
+      // 64, row n - 64 of CTA 1 otherwise: position 32 rank + n % 32 of tile
+      // 2i + (n % 64) / 32).  S of the next pair goes first once the softmax
+      // warps have loaded this pair's S; the P V of this pair's tiles follow.
+      // (one call site each: the issuer's code shares the SM's instruction
+      // cache with the other roles)
+      const int npairs = (ntiles + 1) >> 1;
+      int jn = 0;   // next tile whose P V is due
+      for (int i = 0; i <= npairs && ok; ++i) {
+        if (i < npairs) {
+          if (!tc::wait_cluster(&k_full[i & 1], (i >> 1) & 1) ||
+              (i >= 1 && !tc::wait_cluster(s_free, (i - 1) & 1))) { ok = false; break; }
+          tc::fence_after();
 #pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks)
-          tc::mma2_ts(tS + sb * PF_BN, tQ + 8 * ks,
-                      tc::sdesc_sw128(kaddr + kb * L::KT_BYTES + (ks >> 2) * ((PF_BN / 2) * 128) +
-                                          (ks & 3) * 32, 16, 1024),
-                      IDQK, ks ? 1u : 0u);
-        tc::commit2_both(&s_full[sb]);
-        if (j >= 1) pv(j - 1);
+          for (int ks = 0; ks < D / 16; ++ks)
+            tc::mma2_ts(tS, tQ + 8 * ks,
+                        tc::sdesc_sw128(kaddr + (i & 1) * L::KP_BYTES + (ks >> 2) * (PF_BN * 128) +
+                                            (ks & 3) * 32, 16, 1024),
+                        IDQK, ks ? 1u : 0u);
+          tc::commit2_both(&s_full[i & 1]);
+        }
+        for (const int upto = i < npairs ? 2 * i : ntiles; jn < upto && ok; ++jn) pv(jn);
       }
-      if (ok && ntiles > 0) pv(ntiles - 1);
       if (!ok) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
     }
     __syncwarp();
@@ -356,9 +386,8 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     const int u0 = (UPI == 2) ? 0 : (is_v ? rest : rest & 1);
     const int kb = is_v ? (NKB / 2) * (int)rank + kbl : kbl;
     const int tpos = is_v ? t : (PF_BN / 2) * (int)rank + t;   // position within the tile
-    uint8_t* dst_base = is_v ? sV + kbl * (PF_BN * 128) + t * 128
-                             : sK + kbl * ((PF_BN / 2) * 128) + t * 128;
-    const int tile_bytes = is_v ? L::VT_BYTES : L::KT_BYTES;
+    // V tile buffers [D/128][64 rows][128 B]; K pair buffers [D/64][64 rows][128 B]
+    uint8_t* dst_base = (is_v ? sV : sK) + kbl * (PF_BN * 128) + t * 128;
     const int64_t code_off = (is_v ? a.codes_region : 0) + kb * 32 + u0 * 16;
     // affine: the block's scale/bias word; TQ4: the vector's fp16 norm
     const int64_t sb_off = a.sb_base + (is_v ? a.sb_region : 0) + (TQ ? 0 : kb * 4);
@@ -437,17 +466,27 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     Tile ta, tb, tcur;
     bool ok = true;
     int pg_next = page_of(2);
-    // The loads of tile j + 2 are issued after tile j's arrive: a release
-    // waits for every earlier access of the warp, so loads still in flight
-    // would hold the arrive back by a memory latency.
+    // K warps: tile j's half goes to rows 32 (j & 1) .. of pair buffer
+    // (j / 2) % 2, free once S of the pair two back is done; V warps: tile
+    // buffer j % PF_KVBUF, free once P V of tile j - PF_KVBUF is done.  The
+    // loads of tile j + 2 are issued after tile j's arrive: a release waits
+    // for every earlier access of the warp, so loads still in flight would
+    // hold the arrive back by a memory latency.
+    // (one call of store per step: the roles share the SM's instruction cache)
     auto step = [&](int j, const Tile& cur, Tile& nxt) {
-      const int kbuf = j % PF_KVBUF;
-      if (j >= PF_KVBUF &&
-          !tc::wait_cluster(&pv_done[kbuf], ((j - PF_KVBUF) / PF_KVBUF) & 1)) { ok = false; return; }
-      store(dst_base + kbuf * tile_bytes, cur);
+      const int kbuf = j % PF_KVBUF, pb = (j >> 1) & 1;
+      uint64_t* const free_bar = is_v ? &pv_done[kbuf] : &s_full[pb];
+      const uint32_t free_par = is_v ? ((j - PF_KVBUF) / PF_KVBUF) & 1 : (((j >> 1) - 2) >> 1) & 1;
+      if (j >= 4 && !tc::wait_cluster(free_bar, free_par)) { ok = false; return; }
+      store(dst_base + (is_v ? kbuf * L::VT_BYTES : pb * L::KP_BYTES + (j & 1) * (32 * 128)), cur);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) tc::arrive_cluster(&kv_full[kbuf], 0);
+      if (lane == 0) {
+        uint64_t* const full_bar = is_v ? &v_full[kbuf] : &k_full[pb];
+        tc::arrive_cluster(full_bar, 0);
+        // a last K half without a partner tile arrives for it too
+        if (!is_v && (j & 1) == 0 && j + 1 == ntiles) tc::arrive_cluster(full_bar, 0);
+      }
       if (j + 2 < ntiles) load_tile(j + 2, pg_next, nxt);
       pg_next = page_of(j + 3);
     };
@@ -469,13 +508,20 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
-      const int b = j & 1;
-      if (!tc::wait_cluster(&s_full[b], (j >> 1) & 1)) { ok = false; break; }
+      // tile j's S: positions 0..31 in columns 32 (j & 1) .., 32..63 in
+      // columns 64 + 32 (j & 1) .. of its pair's S
+      const int pi = j >> 1;
+      if (!tc::wait_cluster(&s_full[pi & 1], (pi >> 1) & 1)) { ok = false; break; }
       tc::fence_after();
       uint32_t s0[32], s1[32];
-      tc::ld32(tS + b * PF_BN + lane_off, s0);
-      tc::ld32(tS + b * PF_BN + 32 + lane_off, s1);
+      tc::ld32(tS + (j & 1) * 32 + lane_off, s0);
+      tc::ld32(tS + 64 + (j & 1) * 32 + lane_off, s1);
       tc::wait_ld();
+      if (j & 1) {   // the pair's S is in registers: the next pair's MMA may overwrite it
+        tc::fence_before();
+        __syncwarp();
+        if (lane == 0) tc::arrive_cluster(s_free, 0);
+      }
       const int key0 = (jb + j) * PF_BN;
       float x[PF_BN];
       float mt = -INFINITY;
@@ -521,6 +567,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
             for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
             tc::st32(tO + c0 + lane_off, o);
           }
+          tc::wait_st();   // O is rescaled before P_j's arrive lets P V add to it
         }
         l *= f;
         m_ref = nref;
@@ -536,11 +583,23 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         p[c] = pack_f16x2(p0, p1);
       }
       l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      tc::st32(tS + b * PF_BN + lane_off, p);   // P_j overwrites the S_j columns just read
-      tc::wait_st();
+      // P_j -> this row of P buffer j & 1 (K-major, 128-byte swizzle), once
+      // P V of tile j - 2 has read that buffer
+      if (j >= 2 && !tc::wait_cluster(&pv_done[(j - 2) % PF_KVBUF], ((j - 2) / PF_KVBUF) & 1)) {
+        ok = false;
+        break;
+      }
+      {
+        uint8_t* prow = sP + (j & 1) * L::P_BYTES + r * 128;
+#pragma unroll
+        for (int m = 0; m < 8; ++m)
+          *reinterpret_cast<uint4*>(prow + ((m ^ (r & 7)) << 4)) =
+              make_uint4(p[4 * m], p[4 * m + 1], p[4 * m + 2], p[4 * m + 3]);
+      }
+      fence_proxy_async_smem();
       tc::fence_before();
       __syncwarp();
-      if (lane == 0) tc::arrive_cluster(&p_full[b], 0);
+      if (lane == 0) tc::arrive_cluster(&p_full[j & 3], 0);
     }
     // epilogue: O / l -> bf16 (one split) or the unnormalized partial
     // (m, l, O) in fp32 (several), undoing the d order 0,4,1,5,2,6,3,7
