@@ -20,14 +20,15 @@
 // Warp roles (each CTA):
 //   warp 0      TMEM allocation (512 columns, pair-wide); in CTA 0, lane 0
 //               issues every tcgen05.mma.cta_group::2 of the pair:
-//                 S_i  = Q  [K_2i K_2i+1]^T  (A = Q in TMEM, B = the K halves
+//                 S_i  = Q  [K_2i K_2i+1]^T  (A = Q in smem, B = the K halves
 //                        of tiles 2i and 2i + 1 in smem, K-major, N = 128)
-//                 O   += P_j V_j             (A = P_j in smem, K-major;
-//                        B = V_j smem, MN-major)
+//                 O   += P_j V_j             (A = P_j in TMEM, B = V_j smem,
+//                        MN-major)
 //               and commits to the barrier of both CTAs (multicast).
-//               TMEM columns: O [0, D), S of a tile pair [D, D + 128),
-//               Q [D + 128, +D/2).  S over two tiles keeps the MMA at N = 128
-//               (an N = 64 pair MMA takes as long as an N = 128 one).
+//               TMEM columns: O [0, D), two S/P buffers of a tile pair
+//               [D, D + 256); P_j (fp16) overwrites S columns already read.
+//               S over two tiles keeps the MMA at N = 128 (an N = 64 pair
+//               MMA takes as long as an N = 128 one).
 //   warps 1-8   dequantize this CTA's halves of 64-position K/V tiles from
 //               the pool (page-table lookup, 4-bit codes -> fp16 integers
 //               through the mantissa of fp16 1024, then x = code * scale +
@@ -38,13 +39,13 @@
 //               the pair two back is done), warps 5-8 V halves into four
 //               tile buffers (free once P V of the tile four back is done),
 //               each arriving on CTA 0's K-pair or V-tile barrier.
-//   warps 9-12  one thread per row: Q row -> TMEM at the start; online
-//               softmax on S (tcgen05.ld; after loading the second tile of a
-//               pair it frees the S columns for the next pair's MMA), P as
-//               fp16 into a shared-memory row (two P buffers) and an arrive
-//               on CTA 0's P barrier; the running maximum is moved only when
-//               it grows by more than 2^8, and then O is rescaled in TMEM;
-//               finally O / l -> bf16 output.
+//   warps 9-16  two per row quarter, each thread half a row (32 of a
+//               tile's 64 positions): Q -> shared memory at the start; online
+//               softmax on S (tcgen05.ld), the two halves exchanging their
+//               tile maxima, P back to TMEM as fp16 (tcgen05.st) and an
+//               arrive on CTA 0's P barrier; the running maximum is moved
+//               only when it grows by more than 2^8, and then O is rescaled
+//               in TMEM; finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
 // 0,4,1,5,2,6,3,7 (the pairs one 32-bit word of codes yields); Q uses the same
 // order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
@@ -60,7 +61,7 @@ namespace jfkv {
 constexpr int PF_BM = 128;   // MMA rows per CTA (256 per CTA pair)
 constexpr int PF_BN = 64;    // positions per K/V tile
 constexpr int PF_DQ_WARPS = 8;
-constexpr int PF_SM_WARPS = 4;
+constexpr int PF_SM_WARPS = 8;   // two per TMEM lane quarter, each half a tile's positions
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
 constexpr int PF_KVBUF = 4;     // K/V half-tile buffers in shared memory
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
@@ -97,22 +98,26 @@ struct PrefillArgs {
   PfReq req[PF_MAX_REQ];
 };
 
-// Each CTA of a pair holds half of every K/V tile: K positions 32 r .. 32 r +
-// 31 (all of head_dim, K-major) and V columns D/2 r .. D/2 (r + 1) (all 64
-// positions, MN-major), r = its rank in the pair.  The K halves of tiles 2i
-// and 2i + 1 share a pair buffer (rows 32 (j & 1) + t), so one N = 128 MMA
-// computes S for both.  P of a tile is this CTA's 128 rows x 64 positions
-// (fp16, K-major).
+// Each CTA of a pair holds its 128 query rows (fp16, K-major) and half of
+// every K/V tile: K positions 32 r .. 32 r + 31 (all of head_dim, K-major)
+// and V columns D/2 r .. D/2 (r + 1) (all 64 positions, MN-major), r = its
+// rank in the pair.  The K halves of tiles 2i and 2i + 1 share a pair buffer
+// (rows 32 (j & 1) + t), so one N = 128 MMA computes S for both.  TQ4 keeps
+// three V buffers (its centroid table takes the fourth's room).
 template <int D, int FMT>
 struct PfSmem {
+  static constexpr int VB = FMT == JF_FMT_TQ4 ? 3 : 4;   // V tile buffers
+  static constexpr int Q_BYTES = PF_BM * D * 2;          // [D/64][128 rows][128 B]
   static constexpr int KP_BYTES = PF_BN * D * 2;         // [D/64][64 rows][128 B]
   static constexpr int VT_BYTES = PF_BN * (D / 2) * 2;   // [D/128][64 rows][128 B]
-  static constexpr int P_BYTES = PF_BM * PF_BN * 2;      // [128 rows][128 B]
-  static constexpr int OFF_K = 0;
-  static constexpr int OFF_V = 2 * KP_BYTES;
-  static constexpr int OFF_P = OFF_V + PF_KVBUF * VT_BYTES;
-  static constexpr int OFF_BAR = OFF_P + 2 * P_BYTES;
-  static constexpr int OFF_LUT = OFF_BAR + 256;   // TQ4 centroid table (lane-replicated)
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = Q_BYTES;
+  static constexpr int OFF_V = OFF_K + 2 * KP_BYTES;
+  static constexpr int OFF_BAR = OFF_V + VB * VT_BYTES;
+  // half-row exchange: [2 tile parities][2 halves][128 rows] floats, then
+  // [4 quarters][2 tile parities] mbarriers
+  static constexpr int OFF_X = OFF_BAR + 256;
+  static constexpr int OFF_LUT = OFF_X + 2 * 2 * PF_BM * 4 + 64;   // TQ4 centroid table
   static constexpr int TOTAL = 1024 + OFF_LUT + (FMT == JF_FMT_TQ4 ? 256 * 32 * 4 : 0);
   static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
@@ -183,16 +188,19 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smraw) + 1023) &
                                            ~static_cast<uintptr_t>(1023));
   uint8_t* sK = sm + L::OFF_K;
+  uint8_t* sQ = sm + L::OFF_Q;
   uint8_t* sV = sm + L::OFF_V;
-  uint8_t* sP = sm + L::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L::OFF_BAR);
   uint64_t* k_full = bars + 0;     // [2] on CTA 0: K halves of a tile pair stored
-  uint64_t* v_full = bars + 2;     // [PF_KVBUF] on CTA 0: both CTAs' V halves stored
-  uint64_t* pv_done = bars + 6;    // [PF_KVBUF] both CTAs: P V of the tile done
-  uint64_t* s_full = bars + 10;    // [2] both CTAs: S of pair i done (index i & 1)
-  uint64_t* s_free = bars + 12;    // on CTA 0: both CTAs' softmax warps loaded S
-  uint64_t* p_full = bars + 13;    // [4] on CTA 0: both CTAs' P stored (tile j & 3)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  uint64_t* v_full = bars + 2;     // [VB] on CTA 0: both CTAs' V halves stored (tile j % VB)
+  uint64_t* pv_done = bars + 6;    // [4] both CTAs: P V of tile j done (j & 3)
+  uint64_t* s_full = bars + 10;    // [2] both CTAs: S of pair i done (i & 1)
+  // [4] on CTA 0: both CTAs' P stored (tile j & 3).  S of the next pair is
+  // issued before P V of this one, so a CTA's softmax can run up to 3 tiles
+  // past the tile P V waits for: four barriers keep one CTA's later arrivals
+  // out of the phase the other CTA has not reached.
+  uint64_t* p_full = bars + 12;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = tc::cluster_rank();
@@ -228,9 +236,8 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   const int ntiles = je - jb;
 
   if (threadIdx.x == 0) {
-    static_assert(PF_KVBUF == 4, "barrier layout");
-    for (int i = 0; i < PF_KVBUF; ++i) {
-      mbar_init(&v_full[i], PF_DQ_WARPS);        // the 4 V warps of each CTA
+    for (int i = 0; i < 4; ++i) {
+      if (i < L::VB) mbar_init(&v_full[i], PF_DQ_WARPS);   // the 4 V warps of each CTA
       mbar_init(&pv_done[i], 1);
       mbar_init(&p_full[i], 2 * PF_SM_WARPS);
     }
@@ -238,7 +245,8 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       mbar_init(&k_full[i], 2 * PF_DQ_WARPS);    // the 4 K warps of each CTA, twice
       mbar_init(&s_full[i], 1);
     }
-    mbar_init(s_free, 2 * PF_SM_WARPS);
+    for (int i = 0; i < 8; ++i)   // the 64 threads of a row quarter's two softmax warps
+      mbar_init(reinterpret_cast<uint64_t*>(sm + L::OFF_X + 2 * 2 * PF_BM * 4) + i, 64);
     fence_barrier_init();
   }
   if constexpr (TQ) {   // centroid pair of code byte b for lane l: word b * 32 + l
@@ -253,17 +261,23 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   tc::fence_after();
   const uint32_t tbase = *tmem_slot;
   const uint32_t tO = tbase;
-  const uint32_t tS = tbase + D;               // S of a tile pair, 2 PF_BN columns
-  const uint32_t tQ = tbase + D + 2 * PF_BN;   // D/2 columns of f16 pairs
+  const uint32_t tS = tbase + D;               // two S/P buffers of 2 PF_BN columns
 
-  // ---- softmax warps: their Q row -> TMEM (fp16, pre-multiplied by
-  // softmax_scale * log2(e), d order 0,4,1,5,2,6,3,7 in every 8) ------------
+  // ---- softmax warps: their half of the Q row -> shared memory (fp16,
+  // pre-multiplied by softmax_scale * log2(e), d order 0,4,1,5,2,6,3,7 in
+  // every 8; K-major, 128-byte swizzle: the 16-byte chunk m of row r at
+  // block m / 8, chunk (m % 8) ^ (r % 8)) -------------------------------------
   const int quarter = warp & 3;                // TMEM lanes this warp may access
+  const int half = warp > PF_DQ_WARPS ? (warp - 1 - PF_DQ_WARPS) >> 2 : 0;   // positions 32 half ..
   const int r = quarter * 32 + lane;
   const bool row_ok = r < rows;
   const int qi = row_ok ? r / a.G : 0;
   const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
   int qe = 0;                                  // per-row power of two kept out of fp16
+  auto q_chunk = [&](int m) -> uint4* {
+    return reinterpret_cast<uint4*>(sQ + (m >> 3) * (PF_BM * 128) + r * 128 +
+                                    (((m & 7) ^ (r & 7)) << 4));
+  };
   if (TQ && warp > PF_DQ_WARPS) {
     // rotated fp32 query row, natural d order (the centroid pairs are too)
     const float* qrow = a.qrot + ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
@@ -277,19 +291,17 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     qmax *= fabsf(a.scale_log2);
     qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
     const float qs = ldexpf(a.scale_log2, -qe);
-#pragma unroll 1
-    for (int c0 = 0; c0 < D / 2; c0 += 32) {   // 32 TMEM columns = 64 values
-      uint32_t v[32];
-#pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        float4 w = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (row_ok) w = *reinterpret_cast<const float4*>(qrow + 2 * c0 + 4 * k);
-        v[2 * k + 0] = pack_f16x2(w.x * qs, w.y * qs);
-        v[2 * k + 1] = pack_f16x2(w.z * qs, w.w * qs);
+#pragma unroll 4
+    for (int m = half * (D / 16); m < (half + 1) * (D / 16); ++m) {   // natural d order
+      float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
+      if (row_ok) {
+        w0 = *reinterpret_cast<const float4*>(qrow + 8 * m);
+        w1 = *reinterpret_cast<const float4*>(qrow + 8 * m + 4);
       }
-      tc::st32(tQ + c0 + lane_off, v);
+      *q_chunk(m) = make_uint4(pack_f16x2(w0.x * qs, w0.y * qs), pack_f16x2(w0.z * qs, w0.w * qs),
+                               pack_f16x2(w1.x * qs, w1.y * qs), pack_f16x2(w1.z * qs, w1.w * qs));
     }
-    tc::wait_st();
+    fence_proxy_async_smem();
   } else if (warp > PF_DQ_WARPS) {
     const uint16_t* qrow = rq.q + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
     float qmax = 0.f;
@@ -305,64 +317,60 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     qmax *= a.scale_log2;
     qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
     const float qs = ldexpf(a.scale_log2, -qe);
-#pragma unroll 1
-    for (int c0 = 0; c0 < D / 2; c0 += 32) {   // 32 TMEM columns = 64 values = 8 blocks of 8
-      uint32_t v[32];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        uint4 w = make_uint4(0, 0, 0, 0);
-        if (row_ok) w = *reinterpret_cast<const uint4*>(qrow + 2 * c0 + 8 * k);
-        const float e0 = bf16lo_to_f32(w.x) * qs, e1 = bf16hi_to_f32(w.x) * qs;
-        const float e2 = bf16lo_to_f32(w.y) * qs, e3 = bf16hi_to_f32(w.y) * qs;
-        const float e4 = bf16lo_to_f32(w.z) * qs, e5 = bf16hi_to_f32(w.z) * qs;
-        const float e6 = bf16lo_to_f32(w.w) * qs, e7 = bf16hi_to_f32(w.w) * qs;
-        v[4 * k + 0] = pack_f16x2(e0, e4);
-        v[4 * k + 1] = pack_f16x2(e1, e5);
-        v[4 * k + 2] = pack_f16x2(e2, e6);
-        v[4 * k + 3] = pack_f16x2(e3, e7);
-      }
-      tc::st32(tQ + c0 + lane_off, v);
+#pragma unroll 4
+    for (int m = half * (D / 16); m < (half + 1) * (D / 16); ++m) {
+      uint4 w = make_uint4(0, 0, 0, 0);
+      if (row_ok) w = *reinterpret_cast<const uint4*>(qrow + 8 * m);
+      const float e0 = bf16lo_to_f32(w.x) * qs, e1 = bf16hi_to_f32(w.x) * qs;
+      const float e2 = bf16lo_to_f32(w.y) * qs, e3 = bf16hi_to_f32(w.y) * qs;
+      const float e4 = bf16lo_to_f32(w.z) * qs, e5 = bf16hi_to_f32(w.z) * qs;
+      const float e6 = bf16lo_to_f32(w.w) * qs, e7 = bf16hi_to_f32(w.w) * qs;
+      *q_chunk(m) = make_uint4(pack_f16x2(e0, e4), pack_f16x2(e1, e5), pack_f16x2(e2, e6),
+                               pack_f16x2(e3, e7));
     }
-    tc::wait_st();
+    fence_proxy_async_smem();
   }
   tc::fence_before();
   __syncthreads();
-  tc::cluster_sync();   // both CTAs' Q rows are in TMEM before the first MMA
+  tc::cluster_sync();   // both CTAs' Q rows are in shared memory before the first MMA
   tc::fence_after();
 
   if (warp == 0) {
     // ================= MMA issuer (CTA 0 of the pair) =================
     if (rank == 0 && lane == 0) {
-      const uint32_t kaddr = smem_u32(sK), vaddr = smem_u32(sV), paddr = smem_u32(sP);
+      const uint32_t qaddr = smem_u32(sQ), kaddr = smem_u32(sK), vaddr = smem_u32(sV);
       bool ok = true;
+      // P_j (fp16, 32 columns) sits in the columns of its pair's S buffer
+      // that held S of positions 0..31 of tile j
       auto pv = [&](int j) {   // j: local tile index within this split
-        const int kb = j % PF_KVBUF;
-        if (!tc::wait_cluster(&v_full[kb], (j / PF_KVBUF) & 1) ||
+        const int kb = j % L::VB;
+        if (!tc::wait_cluster(&v_full[kb], (j / L::VB) & 1) ||
             !tc::wait_cluster(&p_full[j & 3], (j >> 2) & 1)) { ok = false; return; }
         tc::fence_after();
+        const uint32_t tp = tS + ((j >> 1) & 1) * (2 * PF_BN) + (j & 1) * 32;
 #pragma unroll
         for (int k = 0; k < PF_BN / 16; ++k)
-          tc::mma2_ss(tO, tc::sdesc_sw128(paddr + (j & 1) * L::P_BYTES + k * 32, 16, 1024),
+          tc::mma2_ts(tO, tp + 8 * k,
                       tc::sdesc_sw128(vaddr + kb * L::VT_BYTES + k * 2048, PF_BN * 128, 1024),
                       IDPV, (j > 0 || k > 0) ? 1u : 0u);
-        tc::commit2_both(&pv_done[kb]);
+        tc::commit2_both(&pv_done[j & 3]);
       };
-      // Pair i: S of tiles 2i, 2i + 1 (S column n = K row n of CTA 0 for n <
-      // 64, row n - 64 of CTA 1 otherwise: position 32 rank + n % 32 of tile
-      // 2i + (n % 64) / 32).  S of the next pair goes first once the softmax
-      // warps have loaded this pair's S; the P V of this pair's tiles follow.
-      // (one call site each: the issuer's code shares the SM's instruction
-      // cache with the other roles)
+      // Pair i: S of tiles 2i, 2i + 1 into S buffer i & 1 (S column n = K row
+      // n of CTA 0 for n < 64, row n - 64 of CTA 1 otherwise: position 32 rank
+      // + n % 32 of tile 2i + (n % 64) / 32), then P V of the previous pair's
+      // tiles; the buffer's last readers (P V of pair i - 2) were issued
+      // before it.  One call site each: the issuer's code shares the SM's
+      // instruction cache with the other roles.
       const int npairs = (ntiles + 1) >> 1;
       int jn = 0;   // next tile whose P V is due
       for (int i = 0; i <= npairs && ok; ++i) {
         if (i < npairs) {
-          if (!tc::wait_cluster(&k_full[i & 1], (i >> 1) & 1) ||
-              (i >= 1 && !tc::wait_cluster(s_free, (i - 1) & 1))) { ok = false; break; }
+          if (!tc::wait_cluster(&k_full[i & 1], (i >> 1) & 1)) { ok = false; break; }
           tc::fence_after();
 #pragma unroll
           for (int ks = 0; ks < D / 16; ++ks)
-            tc::mma2_ts(tS, tQ + 8 * ks,
+            tc::mma2_ss(tS + (i & 1) * (2 * PF_BN),
+                        tc::sdesc_sw128(qaddr + (ks >> 2) * (PF_BM * 128) + (ks & 3) * 32, 16, 1024),
                         tc::sdesc_sw128(kaddr + (i & 1) * L::KP_BYTES + (ks >> 2) * (PF_BN * 128) +
                                             (ks & 3) * 32, 16, 1024),
                         IDQK, ks ? 1u : 0u);
@@ -468,16 +476,16 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     int pg_next = page_of(2);
     // K warps: tile j's half goes to rows 32 (j & 1) .. of pair buffer
     // (j / 2) % 2, free once S of the pair two back is done; V warps: tile
-    // buffer j % PF_KVBUF, free once P V of tile j - PF_KVBUF is done.  The
+    // buffer j % VB, free once P V of tile j - VB is done.  The
     // loads of tile j + 2 are issued after tile j's arrive: a release waits
     // for every earlier access of the warp, so loads still in flight would
     // hold the arrive back by a memory latency.
     // (one call of store per step: the roles share the SM's instruction cache)
     auto step = [&](int j, const Tile& cur, Tile& nxt) {
-      const int kbuf = j % PF_KVBUF, pb = (j >> 1) & 1;
-      uint64_t* const free_bar = is_v ? &pv_done[kbuf] : &s_full[pb];
-      const uint32_t free_par = is_v ? ((j - PF_KVBUF) / PF_KVBUF) & 1 : (((j >> 1) - 2) >> 1) & 1;
-      if (j >= 4 && !tc::wait_cluster(free_bar, free_par)) { ok = false; return; }
+      const int kbuf = j % L::VB, pb = (j >> 1) & 1;
+      uint64_t* const free_bar = is_v ? &pv_done[(j - L::VB) & 3] : &s_full[pb];
+      const uint32_t free_par = is_v ? ((j - L::VB) >> 2) & 1 : (((j >> 1) - 2) >> 1) & 1;
+      if (j >= (is_v ? L::VB : 4) && !tc::wait_cluster(free_bar, free_par)) { ok = false; return; }
       store(dst_base + (is_v ? kbuf * L::VT_BYTES : pb * L::KP_BYTES + (j & 1) * (32 * 128)), cur);
       fence_proxy_async_smem();
       __syncwarp();
@@ -507,46 +515,54 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
+    // The two warps of a row quarter share each row: this one takes positions
+    // 32 half .. 32 half + 31 of every tile (S columns 64 half + 32 (j & 1) ..
+    // of its pair's S buffer), the same lazy maximum (they exchange their
+    // tile maxima), half of O's columns and P columns 32 (j & 1) + 16 half ..
+    // (S columns both halves have read once the maxima are exchanged); l is
+    // summed per half.
+    float* const xch = reinterpret_cast<float*>(sm + L::OFF_X);   // [parity][half][row]
+    uint64_t* const xbar = reinterpret_cast<uint64_t*>(sm + L::OFF_X + 2 * 2 * PF_BM * 4) +
+                           quarter * 2;                            // [parity]
+    // partner's value of this row for exchange k (bounded wait, no hang if
+    // the partner gave up)
+    auto exchange = [&](int k, float v, float& other) -> bool {
+      xch[((k & 1) * 2 + half) * PF_BM + r] = v;
+      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(&xbar[k & 1])) : "memory");
+      if (!mbar_wait_bounded(&xbar[k & 1], (k >> 1) & 1)) return false;
+      other = xch[((k & 1) * 2 + (half ^ 1)) * PF_BM + r];
+      return true;
+    };
     for (int j = 0; j < ntiles; ++j) {
-      // tile j's S: positions 0..31 in columns 32 (j & 1) .., 32..63 in
-      // columns 64 + 32 (j & 1) .. of its pair's S
       const int pi = j >> 1;
       if (!tc::wait_cluster(&s_full[pi & 1], (pi >> 1) & 1)) { ok = false; break; }
       tc::fence_after();
-      uint32_t s0[32], s1[32];
-      tc::ld32(tS + (j & 1) * 32 + lane_off, s0);
-      tc::ld32(tS + 64 + (j & 1) * 32 + lane_off, s1);
+      const uint32_t tb = tS + (pi & 1) * (2 * PF_BN);   // the pair's S/P buffer
+      uint32_t s0[32];
+      tc::ld32(tb + half * 64 + (j & 1) * 32 + lane_off, s0);
       tc::wait_ld();
-      if (j & 1) {   // the pair's S is in registers: the next pair's MMA may overwrite it
-        tc::fence_before();
-        __syncwarp();
-        if (lane == 0) tc::arrive_cluster(s_free, 0);
-      }
-      const int key0 = (jb + j) * PF_BN;
-      float x[PF_BN];
-      float mt = -INFINITY;
+      const int key0 = (jb + j) * PF_BN + 32 * half;
+      float x[32];
+      float mt;
       {
         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        if (key0 + PF_BN - 1 <= limit) {       // every position of the tile visible
+        if (key0 + 31 <= limit) {       // every position of the half tile visible
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            x[c] = __uint_as_float(s0[c]);
-            x[c + 32] = __uint_as_float(s1[c]);
-          }
+          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(s0[c]);
         } else {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) : -INFINITY;
-            x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) : -INFINITY;
-          }
+          for (int c = 0; c < 32; ++c) x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) : -INFINITY;
         }
         if (qe != 0) {
 #pragma unroll
-          for (int c = 0; c < PF_BN; ++c) x[c] *= smul;
+          for (int c = 0; c < 32; ++c) x[c] *= smul;
         }
 #pragma unroll
-        for (int c = 0; c < PF_BN; ++c) m4[c & 3] = fmaxf(m4[c & 3], x[c]);
-        mt = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        for (int c = 0; c < 32; ++c) m4[c & 3] = fmaxf(m4[c & 3], x[c]);
+        const float mh = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        float mo;
+        if (!exchange(j, mh, mo)) { ok = false; break; }
+        mt = fmaxf(mh, mo);
       }
       const bool need = mt > m_ref + PF_TAU;
       if (__any_sync(0xffffffffu, need)) {
@@ -559,7 +575,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
           }
           tc::fence_after();
 #pragma unroll 1
-          for (int c0 = 0; c0 < D; c0 += 32) {
+          for (int c0 = half * (D / 2); c0 < (half + 1) * (D / 2); c0 += 32) {
             uint32_t o[32];
             tc::ld32(tO + c0 + lane_off, o);
             tc::wait_ld();
@@ -572,10 +588,10 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         l *= f;
         m_ref = nref;
       }
-      uint32_t p[32];
+      uint32_t p[16];
       float l4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
+      for (int c = 0; c < 16; ++c) {
         // -inf - m_ref -> exp2 = 0; m_ref is finite once any position was visible
         const float p0 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c] - m_ref);
         const float p1 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c + 1] - m_ref);
@@ -583,23 +599,16 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         p[c] = pack_f16x2(p0, p1);
       }
       l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      // P_j -> this row of P buffer j & 1 (K-major, 128-byte swizzle), once
-      // P V of tile j - 2 has read that buffer
-      if (j >= 2 && !tc::wait_cluster(&pv_done[(j - 2) % PF_KVBUF], ((j - 2) / PF_KVBUF) & 1)) {
-        ok = false;
-        break;
-      }
-      {
-        uint8_t* prow = sP + (j & 1) * L::P_BYTES + r * 128;
-#pragma unroll
-        for (int m = 0; m < 8; ++m)
-          *reinterpret_cast<uint4*>(prow + ((m ^ (r & 7)) << 4)) =
-              make_uint4(p[4 * m], p[4 * m + 1], p[4 * m + 2], p[4 * m + 3]);
-      }
-      fence_proxy_async_smem();
+      tc::st16(tb + (j & 1) * 32 + 16 * half + lane_off, p);
+      tc::wait_st();
       tc::fence_before();
       __syncwarp();
       if (lane == 0) tc::arrive_cluster(&p_full[j & 3], 0);
+    }
+    {   // the row's sum: both halves' parts
+      float lo = 0.f;
+      if (ok && !exchange(ntiles, l, lo)) ok = false;
+      l += lo;
     }
     // epilogue: O / l -> bf16 (one split) or the unnormalized partial
     // (m, l, O) in fp32 (several), undoing the d order 0,4,1,5,2,6,3,7
@@ -607,7 +616,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     const int64_t prow = ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) *
                          a.num_splits + blockIdx.z;
     if (ntiles == 0) {   // an empty history range: a neutral partial
-      if (split && row_ok) {
+      if (split && row_ok && half == 0) {
         a.part_ml[prow * 2 + 0] = -INFINITY;
         a.part_ml[prow * 2 + 1] = 0.f;
         float4* po = reinterpret_cast<float4*>(a.part_o + prow * D);
@@ -619,12 +628,12 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       const float inv = split ? 1.f : (l > 0.f ? 1.f / l : 0.f);
       uint16_t* orow = rq.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
       float* prow_o = split ? a.part_o + prow * D : nullptr;
-      if (split && row_ok) {
+      if (split && row_ok && half == 0) {
         a.part_ml[prow * 2 + 0] = m_ref;
         a.part_ml[prow * 2 + 1] = l;
       }
 #pragma unroll 1
-      for (int c0 = 0; c0 < D; c0 += 32) {
+      for (int c0 = half * (D / 2); c0 < (half + 1) * (D / 2); c0 += 32) {
         uint32_t o[32];
         tc::ld32(tO + c0 + lane_off, o);
         tc::wait_ld();

@@ -173,6 +173,15 @@ __device__ __forceinline__ void st32(uint32_t taddr, const uint32_t (&v)[32]) {
       : "memory");
 }
 
+// 32 lanes x 16 columns of 32-bit words
+__device__ __forceinline__ void st16(uint32_t taddr, const uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+      "%13,%14,%15,%16};\n"
+      ::"r"(taddr), JF_W8(0), JF_W8(8)
+      : "memory");
+}
+
 #undef JF_R8
 #undef JF_W8
 
