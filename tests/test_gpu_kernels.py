@@ -440,6 +440,25 @@ def test_prefill_matches_oracle(Hq, Hkv, D, P, q_start, C, causal):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("D", [128, 256])
+@pytest.mark.parametrize("total", [1, 64, 65, 128, 192, 257, 320, 450, 576])
+def test_prefill_history_tile_counts(D, total):
+    """1 to 9 history tiles of 64 positions: S runs over tile pairs (a lone
+    last tile, pair buffers reused once and twice), P over single tiles."""
+    Hq, Hkv, P = (24, 4, 256) if D == 256 else (8, 2, 128)
+    C = min(total, 24)
+    case = make_case(700 + total + D, Hq, Hkv, D, P, [total], outliers=True)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    from paper_2609_17475_gb300 import synth
+    q = synth.normal_bf16(synth.generator(701 + total), (C, Hq, D))
+    scale = 1 / math.sqrt(D)
+    out = gpu_prefill(case, pool, q, total - C, True, scale)
+    ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q), total - C,
+                           scale, causal=True)
+    assert_attention_close(out, ref)
+
+
 def test_prefill_32k_prefix_sampled_rows():
     """The last 2,048-query chunk of the 32K prompt (24/4/256, P 256): sampled
     query rows checked against the oracle's decode at ctx = position + 1."""

@@ -430,6 +430,28 @@ def test_tq4_prefill_matches_oracle(Hq, Hkv, D, P, q_start, C, causal):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("total", [1, 65, 257, 450, 833])
+def test_tq4_prefill_history_tile_counts(total):
+    """1 to 14 history tiles on the TQ4 instance (three V buffers): a lone
+    last tile of a pair, buffers reused several times."""
+    Hq, Hkv, D, P = 24, 4, 256, 256
+    C = min(total, 24)
+    case = make_case(750 + total, Hq, Hkv, D, P, [total], outliers=True)
+    lay, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    q = synth.normal_bf16(synth.generator(9 + total), (C, Hq, D))
+    scale = 1 / math.sqrt(D)
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    ws = jf.prefill_batch_workspace(C, Hq, D, 1, device=DEV, format=jf.JF_FMT_TQ4)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), total - C, scale, True,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    ref = OT.prefill_chunk(ref_pool, lay, case.page_table[0].numpy(), bits(q), total - C, scale,
+                           causal=True)
+    assert_attention_close(out, ref)
+
+
 @pytest.mark.parametrize("spans,splits", [
     ([(3000, 64), (0, 40), (700, 150)], 1),
     ([(3000, 64), (0, 40), (700, 150)], 5),
