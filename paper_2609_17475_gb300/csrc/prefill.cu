@@ -36,9 +36,10 @@
 //               buffers, one item (one position's code bytes of a 64-wide
 //               block) per thread, loads running two tiles ahead; warps 1-4
 //               write K halves into two pair buffers (free again once S of
-//               the pair two back is done), warps 5-8 V halves into four
-//               tile buffers (free once P V of the tile four back is done),
-//               each arriving on CTA 0's K-pair or V-tile barrier.
+//               the pair two back is done), warps 5-8 V halves into VB tile
+//               buffers (four; three for TQ4; free once P V of the tile VB
+//               back is done), each arriving on CTA 0's K-pair or V-tile
+//               barrier.
 //   warps 9-16  two per row quarter, each thread half a row (32 of a
 //               tile's 64 positions): Q -> shared memory at the start; online
 //               softmax on S (tcgen05.ld), the two halves exchanging their
@@ -63,7 +64,7 @@ constexpr int PF_BN = 64;    // positions per K/V tile
 constexpr int PF_DQ_WARPS = 8;
 constexpr int PF_SM_WARPS = 8;   // two per TMEM lane quarter, each half a tile's positions
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
-constexpr int PF_KVBUF = 4;     // K/V half-tile buffers in shared memory
+constexpr int PF_KVBUF = 4;     // P V completion barriers, by tile index mod 4
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
 
 // One request's chunk in a launch: its query tiles are CTAs tile0 ..
