@@ -36,17 +36,15 @@
 //               buffers, one item (one position's code bytes of a 64-wide
 //               block) per thread, loads running two tiles ahead; warps 1-4
 //               write K halves into two pair buffers (free again once S of
-//               the pair two back is done), warps 5-8 V halves into VB tile
-//               buffers (four; three for TQ4; free once P V of the tile VB
-//               back is done), each arriving on CTA 0's K-pair or V-tile
-//               barrier.
-//   warps 9-16  two per row quarter, each thread half a row (32 of a
-//               tile's 64 positions): Q -> shared memory at the start; online
-//               softmax on S (tcgen05.ld), the two halves exchanging their
-//               tile maxima, P back to TMEM as fp16 (tcgen05.st) and an
-//               arrive on CTA 0's P barrier; the running maximum is moved
-//               only when it grows by more than 2^8, and then O is rescaled
-//               in TMEM; finally O / l -> bf16 output.
+//               the pair two back is done), warps 5-8 V halves into four
+//               tile buffers (free once P V of the tile four back is done),
+//               each arriving on CTA 0's K-pair or V-tile barrier.
+//   warps 9-12  one thread per row: Q row -> shared memory at the start;
+//               online softmax on S (tcgen05.ld), P back to TMEM as fp16
+//               over S columns already read (tcgen05.st) and an arrive on
+//               CTA 0's P barrier; the running maximum is moved only when it
+//               grows by more than 2^8, and then O is rescaled in TMEM;
+//               finally O / l -> bf16 output.
 // Within every 8 consecutive d the tiles store elements in the order
 // 0,4,1,5,2,6,3,7 (the pairs one 32-bit word of codes yields); Q uses the same
 // order, so Q K^T is unchanged, and the epilogue undoes it for O.  Q is
@@ -62,7 +60,7 @@ namespace jfkv {
 constexpr int PF_BM = 128;   // MMA rows per CTA (256 per CTA pair)
 constexpr int PF_BN = 64;    // positions per K/V tile
 constexpr int PF_DQ_WARPS = 8;
-constexpr int PF_SM_WARPS = 8;   // two per TMEM lane quarter, each half a tile's positions
+constexpr int PF_SM_WARPS = 4;   // one per TMEM lane quarter, one row per thread
 constexpr int PF_THREADS = 32 * (1 + PF_DQ_WARPS + PF_SM_WARPS);
 constexpr int PF_KVBUF = 4;     // P V completion barriers, by tile index mod 4
 constexpr float PF_TAU = 8.f;   // log2 headroom before the running max moves
@@ -103,11 +101,10 @@ struct PrefillArgs {
 // every K/V tile: K positions 32 r .. 32 r + 31 (all of head_dim, K-major)
 // and V columns D/2 r .. D/2 (r + 1) (all 64 positions, MN-major), r = its
 // rank in the pair.  The K halves of tiles 2i and 2i + 1 share a pair buffer
-// (rows 32 (j & 1) + t), so one N = 128 MMA computes S for both.  TQ4 keeps
-// three V buffers (its centroid table takes the fourth's room).
+// (rows 32 (j & 1) + t), so one N = 128 MMA computes S for both.
 template <int D, int FMT>
 struct PfSmem {
-  static constexpr int VB = FMT == JF_FMT_TQ4 ? 3 : 4;   // V tile buffers
+  static constexpr int VB = 4;                           // V tile buffers
   static constexpr int Q_BYTES = PF_BM * D * 2;          // [D/64][128 rows][128 B]
   static constexpr int KP_BYTES = PF_BN * D * 2;         // [D/64][64 rows][128 B]
   static constexpr int VT_BYTES = PF_BN * (D / 2) * 2;   // [D/128][64 rows][128 B]
@@ -115,10 +112,7 @@ struct PfSmem {
   static constexpr int OFF_K = Q_BYTES;
   static constexpr int OFF_V = OFF_K + 2 * KP_BYTES;
   static constexpr int OFF_BAR = OFF_V + VB * VT_BYTES;
-  // half-row exchange: [2 tile parities][2 halves][128 rows] floats, then
-  // [4 quarters][2 tile parities] mbarriers
-  static constexpr int OFF_X = OFF_BAR + 256;
-  static constexpr int OFF_LUT = OFF_X + 2 * 2 * PF_BM * 4 + 64;   // TQ4 centroid table
+  static constexpr int OFF_LUT = OFF_BAR + 256;   // TQ4 centroid table (lane-replicated)
   static constexpr int TOTAL = 1024 + OFF_LUT + (FMT == JF_FMT_TQ4 ? 256 * 32 * 4 : 0);
   static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
@@ -246,8 +240,6 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       mbar_init(&k_full[i], 2 * PF_DQ_WARPS);    // the 4 K warps of each CTA, twice
       mbar_init(&s_full[i], 1);
     }
-    for (int i = 0; i < 8; ++i)   // the 64 threads of a row quarter's two softmax warps
-      mbar_init(reinterpret_cast<uint64_t*>(sm + L::OFF_X + 2 * 2 * PF_BM * 4) + i, 64);
     fence_barrier_init();
   }
   if constexpr (TQ) {   // centroid pair of code byte b for lane l: word b * 32 + l
@@ -264,12 +256,11 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
   const uint32_t tO = tbase;
   const uint32_t tS = tbase + D;               // two S/P buffers of 2 PF_BN columns
 
-  // ---- softmax warps: their half of the Q row -> shared memory (fp16,
+  // ---- softmax warps: their Q row -> shared memory (fp16,
   // pre-multiplied by softmax_scale * log2(e), d order 0,4,1,5,2,6,3,7 in
   // every 8; K-major, 128-byte swizzle: the 16-byte chunk m of row r at
   // block m / 8, chunk (m % 8) ^ (r % 8)) -------------------------------------
   const int quarter = warp & 3;                // TMEM lanes this warp may access
-  const int half = warp > PF_DQ_WARPS ? (warp - 1 - PF_DQ_WARPS) >> 2 : 0;   // positions 32 half ..
   const int r = quarter * 32 + lane;
   const bool row_ok = r < rows;
   const int qi = row_ok ? r / a.G : 0;
@@ -293,7 +284,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
     const float qs = ldexpf(a.scale_log2, -qe);
 #pragma unroll 4
-    for (int m = half * (D / 16); m < (half + 1) * (D / 16); ++m) {   // natural d order
+    for (int m = 0; m < D / 8; ++m) {   // natural d order
       float4 w0 = make_float4(0.f, 0.f, 0.f, 0.f), w1 = w0;
       if (row_ok) {
         w0 = *reinterpret_cast<const float4*>(qrow + 8 * m);
@@ -319,7 +310,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
     const float qs = ldexpf(a.scale_log2, -qe);
 #pragma unroll 4
-    for (int m = half * (D / 16); m < (half + 1) * (D / 16); ++m) {
+    for (int m = 0; m < D / 8; ++m) {
       uint4 w = make_uint4(0, 0, 0, 0);
       if (row_ok) w = *reinterpret_cast<const uint4*>(qrow + 8 * m);
       const float e0 = bf16lo_to_f32(w.x) * qs, e1 = bf16hi_to_f32(w.x) * qs;
@@ -516,67 +507,50 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     const float smul = ldexpf(1.f, qe);   // S = (scaled Q) K^T * 2^qe
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
-    // The two warps of a row quarter share each row: this one takes positions
-    // 32 half .. 32 half + 31 of every tile (S columns 64 half + 32 (j & 1) ..
-    // of its pair's S buffer), the same lazy maximum (they exchange their
-    // tile maxima), half of O's columns and P columns 32 (j & 1) + 16 half ..
-    // (S columns both halves have read once the maxima are exchanged); l is
-    // summed per half.
-    float* const xch = reinterpret_cast<float*>(sm + L::OFF_X);   // [parity][half][row]
-    uint64_t* const xbar = reinterpret_cast<uint64_t*>(sm + L::OFF_X + 2 * 2 * PF_BM * 4) +
-                           quarter * 2;                            // [parity]
-    // partner's value of this row for exchange k (bounded wait, no hang if
-    // the partner gave up)
-    auto exchange = [&](int k, float v, float& other) -> bool {
-      xch[((k & 1) * 2 + half) * PF_BM + r] = v;
-      asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(smem_u32(&xbar[k & 1])) : "memory");
-      if (!mbar_wait_bounded(&xbar[k & 1], (k >> 1) & 1)) return false;
-      other = xch[((k & 1) * 2 + (half ^ 1)) * PF_BM + r];
-      return true;
-    };
     for (int j = 0; j < ntiles; ++j) {
+      // tile j's S: positions 0..31 in columns 32 (j & 1) .., 32..63 in
+      // columns 64 + 32 (j & 1) .. of its pair's S/P buffer; P_j (fp16)
+      // goes to columns 32 (j & 1) .. once both are read
       const int pi = j >> 1;
       if (!tc::wait_cluster(&s_full[pi & 1], (pi >> 1) & 1)) { ok = false; break; }
       tc::fence_after();
-      const uint32_t tb = tS + (pi & 1) * (2 * PF_BN);   // the pair's S/P buffer
-      uint32_t s0[32];
-      tc::ld32(tb + half * 64 + (j & 1) * 32 + lane_off, s0);
+      const uint32_t tb = tS + (pi & 1) * (2 * PF_BN);
+      uint32_t s0[32], s1[32];
+      tc::ld32(tb + (j & 1) * 32 + lane_off, s0);
+      tc::ld32(tb + 64 + (j & 1) * 32 + lane_off, s1);
       tc::wait_ld();
-      const int key0 = (jb + j) * PF_BN + 32 * half;
-      float x[32];
+      const int key0 = (jb + j) * PF_BN;
+      float x[PF_BN];
       float mt;
       {
         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        if (key0 + 31 <= limit) {       // every position of the half tile visible
+        if (key0 + PF_BN - 1 <= limit) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(s0[c]);
+          for (int c = 0; c < 32; ++c) { x[c] = __uint_as_float(s0[c]); x[c + 32] = __uint_as_float(s1[c]); }
         } else {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) : -INFINITY;
+          for (int c = 0; c < 32; ++c) {
+            x[c] = (key0 + c <= limit) ? __uint_as_float(s0[c]) : -INFINITY;
+            x[c + 32] = (key0 + c + 32 <= limit) ? __uint_as_float(s1[c]) : -INFINITY;
+          }
         }
         if (qe != 0) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[c] *= smul;
+          for (int c = 0; c < PF_BN; ++c) x[c] *= smul;
         }
 #pragma unroll
-        for (int c = 0; c < 32; ++c) m4[c & 3] = fmaxf(m4[c & 3], x[c]);
-        const float mh = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-        float mo;
-        if (!exchange(j, mh, mo)) { ok = false; break; }
-        mt = fmaxf(mh, mo);
+        for (int c = 0; c < PF_BN; ++c) m4[c & 3] = fmaxf(m4[c & 3], x[c]);
+        mt = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       }
       const bool need = mt > m_ref + PF_TAU;
       if (__any_sync(0xffffffffu, need)) {
         const float nref = need ? mt : m_ref;
         const float f = (need && m_ref != -INFINITY) ? fast_exp2(m_ref - nref) : 1.f;
         if (j > 0) {
-          if (!tc::wait_cluster(&pv_done[(j - 1) % PF_KVBUF], ((j - 1) / PF_KVBUF) & 1)) {
-            ok = false;
-            break;
-          }
+          if (!tc::wait_cluster(&pv_done[(j - 1) % PF_KVBUF], ((j - 1) / PF_KVBUF) & 1)) { ok = false; break; }
           tc::fence_after();
 #pragma unroll 1
-          for (int c0 = half * (D / 2); c0 < (half + 1) * (D / 2); c0 += 32) {
+          for (int c0 = 0; c0 < D; c0 += 32) {
             uint32_t o[32];
             tc::ld32(tO + c0 + lane_off, o);
             tc::wait_ld();
@@ -584,32 +558,25 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
             for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
             tc::st32(tO + c0 + lane_off, o);
           }
-          tc::wait_st();   // O is rescaled before P_j's arrive lets P V add to it
         }
         l *= f;
         m_ref = nref;
       }
-      uint32_t p[16];
+      uint32_t p[32];
       float l4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        // -inf - m_ref -> exp2 = 0; m_ref is finite once any position was visible
+      for (int c = 0; c < 32; ++c) {
         const float p0 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c] - m_ref);
         const float p1 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c + 1] - m_ref);
         l4[c & 3] += p0 + p1;
         p[c] = pack_f16x2(p0, p1);
       }
       l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      tc::st16(tb + (j & 1) * 32 + 16 * half + lane_off, p);
+      tc::st32(tb + (j & 1) * 32 + lane_off, p);
       tc::wait_st();
       tc::fence_before();
       __syncwarp();
       if (lane == 0) tc::arrive_cluster(&p_full[j & 3], 0);
-    }
-    {   // the row's sum: both halves' parts
-      float lo = 0.f;
-      if (ok && !exchange(ntiles, l, lo)) ok = false;
-      l += lo;
     }
     // epilogue: O / l -> bf16 (one split) or the unnormalized partial
     // (m, l, O) in fp32 (several), undoing the d order 0,4,1,5,2,6,3,7
@@ -617,7 +584,7 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
     const int64_t prow = ((int64_t)(rq.row0 + q0 + qi) * a.Hq + kvh * a.G + r % a.G) *
                          a.num_splits + blockIdx.z;
     if (ntiles == 0) {   // an empty history range: a neutral partial
-      if (split && row_ok && half == 0) {
+      if (split && row_ok) {
         a.part_ml[prow * 2 + 0] = -INFINITY;
         a.part_ml[prow * 2 + 1] = 0.f;
         float4* po = reinterpret_cast<float4*>(a.part_o + prow * D);
@@ -629,12 +596,12 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       const float inv = split ? 1.f : (l > 0.f ? 1.f / l : 0.f);
       uint16_t* orow = rq.out + ((int64_t)(q0 + qi) * a.Hq + kvh * a.G + r % a.G) * D;
       float* prow_o = split ? a.part_o + prow * D : nullptr;
-      if (split && row_ok && half == 0) {
+      if (split && row_ok) {
         a.part_ml[prow * 2 + 0] = m_ref;
         a.part_ml[prow * 2 + 1] = l;
       }
 #pragma unroll 1
-      for (int c0 = half * (D / 2); c0 < (half + 1) * (D / 2); c0 += 32) {
+      for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t o[32];
         tc::ld32(tO + c0 + lane_off, o);
         tc::wait_ld();
