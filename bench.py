@@ -130,6 +130,16 @@ def dist_env():
     return world, rank, local
 
 
+def max_over_ranks(value, world, device):
+    """The largest `value` over all ranks (the slowest replica's time); the
+    value itself when one process runs."""
+    if world <= 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
@@ -222,11 +232,8 @@ def run_ours(args, world, rank, local):
             e1.record(stream)
         stream.synchronize()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
         torch.distributed.barrier()
     clocks = clk.summary()
 
@@ -278,7 +285,7 @@ def run_ours(args, world, rank, local):
             e2e_step()
         f1.record(stream)
     stream.synchronize()
-    e2e_ms = f0.elapsed_time(f1) / e2e_steps
+    e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world, dev)
     h2d = qh.numel() * 2 + kh.numel() * 2 + vh.numel() * 2
     d2h = oh.numel() * 2
     torch.cuda.synchronize()
