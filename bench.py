@@ -662,6 +662,30 @@ def _bench_rows(jf, synth, dev, stream, peaks_gbs, peak_tf, only=None):
     out["a1a4_prompt_32k_16_chunks"] = {
         "ms": t_pf_all, "TFLOPs_attention": flops_all / (t_pf_all / 1e3) / 1e12,
         "prompt_positions_per_s": prompt / (t_pf_all / 1e3)}
+    # the same calls with the workspace that lets a chunk balance its waves
+    # (whole waves of CTA pairs, then the last query tiles with split histories)
+    pwb = torch.zeros(max(jf.jf_prefill_chunk_workspace_bytes(pool, c * chunk, chunk, Hq)
+                          for c in range(prompt // chunk)), dtype=torch.uint8, device=dev)
+    t_bal = _event_time(lambda: jf.jf_prefill_chunk_attn(pool, pt[0], qc, q_last, scale, True, oc,
+                                                         pwb, stream=stream), 10, stream)
+
+    def prefill_all_balanced():
+        for c in range(prompt // chunk):
+            pos = torch.arange(c * chunk, (c + 1) * chunk, dtype=torch.int32, device=dev)
+            jf.jf_kv_quantize_append(pool, pt, zero_req, pos, kc, vc, err, stream=stream)
+            jf.jf_prefill_chunk_attn(pool, pt[0], qc, c * chunk, scale, True, oc, pwb,
+                                     stream=stream)
+    t_all_bal = _event_time(prefill_all_balanced, 3, stream)
+    check("a1+a4 prompt, balanced", pwb)
+    out["a4_prefill_chunk_2048_at_30720"]["balanced"] = {
+        "ms": t_bal, "TFLOPs": flops / (t_bal / 1e3) / 1e12,
+        "frac_tensor": flops / (t_bal / 1e3) / 1e12 / peak_tf,
+        "workspace_bytes": pwb.numel(), "launches": "prefill (whole waves) + prefill (split "
+                                                    "tail) + merge"}
+    out["a1a4_prompt_32k_16_chunks"]["balanced"] = {
+        "ms": t_all_bal, "TFLOPs_attention": flops_all / (t_all_bal / 1e3) / 1e12,
+        "prompt_positions_per_s": prompt / (t_all_bal / 1e3)}
+    del pwb
     # decode loop of the 32K+6K workload: 6,144 x (append 1 row, decode) in one CUDA graph
     q1 = torch.randn(1, Hq, D, generator=g, device=dev).to(torch.bfloat16)
     o1 = torch.empty_like(q1)

@@ -266,6 +266,15 @@ int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_tabl
  *   workspace       affine pool: >= jf_prefill_workspace_bytes() (an int32
  *                   status word); TQ4 pool: >= jf_prefill_batch_workspace_bytes(
  *                   JF_FMT_TQ4, chunk_len, Hq, D, 1), 256-byte aligned.
+ * Wave balance: the kernel runs one CTA per SM, two per pair.  A chunk over
+ * a long prefix (q_start >= 4 chunk_len) whose CTA pairs would leave the last
+ * wave partly empty runs, when the workspace holds
+ * jf_prefill_chunk_workspace_bytes(...) bytes (256-byte aligned), as two
+ * launches: its first query tiles as whole waves, then the rest with their
+ * history split across pairs and merged (as jf_prefill_batch_attn with
+ * num_splits > 1).  With a smaller workspace it runs as one launch.  Both
+ * forms compute the same attention; the summation order, and so the last
+ * bits, differ.
  * TQ4 pools (Sec. 3.1: page lookup, unpacking, centroid lookup, inverse
  * rotation and norm restoration fused into the attention's operand path):
  * the queries are rotated once (q' = H S_K q / sqrt(D), fp32 in the
@@ -277,6 +286,13 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
                           const void* q, int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
                           float softmax_scale, int32_t causal, void* out, void* workspace,
                           size_t workspace_bytes, void* stream);
+
+/* Workspace bytes with which jf_prefill_chunk_attn runs this chunk in its
+ * wave-balanced form on a GPU with num_sms SMs (0: the current device's);
+ * the plain minimum when the chunk runs as one launch anyway.  Host only
+ * (with num_sms > 0 it touches no device).  0 for invalid arguments. */
+size_t jf_prefill_chunk_workspace_bytes(const jf_kv_pool* pool, int32_t q_start,
+                                        int32_t chunk_len, int32_t num_q_heads, int32_t num_sms);
 
 /*
  * Prefill chunks of several requests in one launch (Sec. 3.3: the scheduler

@@ -11,4 +11,5 @@ from .binding import (  # noqa: F401
     status_string, version, verify_workspace, default_verify_splits, workspace_status,
     JF_FMT_AFFINE4_G64, JF_FMT_TQ4, Tq4Codec, jf_kv_page_bytes_fmt, jf_tq4_codebook,
     jf_prefill_batch_attn, jf_reservation_pages, prefill_batch_workspace, default_prefill_splits,
+    jf_prefill_chunk_workspace_bytes, prefill_chunk_workspace,
 )

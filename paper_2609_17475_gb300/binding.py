@@ -33,7 +33,7 @@ EXPORTS = [
     "jf_kv_checkpoint", "jf_kv_restore", "jf_status_string", "jf_version",
     "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
     "jf_kv_page_bytes_fmt", "jf_tq4_codebook", "jf_prefill_batch_attn", "jf_reservation_pages",
-    "jf_prefill_batch_workspace_bytes",
+    "jf_prefill_batch_workspace_bytes", "jf_prefill_chunk_workspace_bytes",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -91,6 +91,7 @@ def lib() -> ctypes.CDLL:
             "jf_prefill_batch_attn": (ctypes.c_int, [PP, P, I32, I32, P, P, P, I32, F32, I32, I32,
                                                      P, P, SZ, P]),
             "jf_prefill_batch_workspace_bytes": (SZ, [I32, I64, I32, I32, I32]),
+            "jf_prefill_chunk_workspace_bytes": (SZ, [PP, I32, I32, I32, I32]),
             "jf_reservation_pages": (I64, [I64, I64, I64, I32]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
@@ -396,6 +397,25 @@ def prefill_batch_workspace(total_rows: int, num_q_heads: int, head_dim: int, nu
                             device="cuda", format: int = JF_FMT_AFFINE4_G64) -> torch.Tensor:
     n = int(lib().jf_prefill_batch_workspace_bytes(int(format), int(total_rows), num_q_heads,
                                                    head_dim, num_splits))
+    if n == 0:
+        raise ValueError("invalid workspace geometry")
+    return torch.zeros(n, dtype=torch.uint8, device=device)
+
+
+def jf_prefill_chunk_workspace_bytes(pool: "KVPool", q_start: int, chunk_len: int,
+                                     num_q_heads: int, num_sms: int = 0) -> int:
+    """Workspace bytes for jf_prefill_chunk_attn's wave-balanced form (the
+    plain minimum when the chunk runs as one launch); num_sms 0: the current
+    device's."""
+    return int(lib().jf_prefill_chunk_workspace_bytes(ctypes.byref(pool.c_struct()), int(q_start),
+                                                      int(chunk_len), int(num_q_heads),
+                                                      int(num_sms)))
+
+
+def prefill_chunk_workspace(pool: "KVPool", q_start: int, chunk_len: int, num_q_heads: int,
+                            device="cuda") -> torch.Tensor:
+    """A zeroed workspace with which jf_prefill_chunk_attn balances its waves."""
+    n = jf_prefill_chunk_workspace_bytes(pool, q_start, chunk_len, num_q_heads)
     if n == 0:
         raise ValueError("invalid workspace geometry")
     return torch.zeros(n, dtype=torch.uint8, device=device)

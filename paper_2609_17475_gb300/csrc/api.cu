@@ -36,6 +36,7 @@ int launch_prefill_batch(const Geom&, const jf_kv_pool&, const int32_t* const*, 
                          int32_t, void*, void*, cudaStream_t, int32_t, int64_t,
                          const Tq4Params*);
 size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S, int fmt);
+int sm_count();
 }  // namespace jfkv
 
 using namespace jfkv;
@@ -243,6 +244,87 @@ int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_tabl
                        stream);
 }
 
+}  // extern "C"
+
+namespace {
+
+// The prefill kernel's geometry: 128 MMA rows per CTA (128 / G queries), two
+// CTAs per pair, one CTA per SM, 64-position history tiles.
+constexpr int64_t kPfRows = 128;
+constexpr int64_t kPfTile = 64;
+
+// Wave balance of one chunk over a long prefix (q_start >= 4 chunk_len, so
+// its CTA pairs carry nearly equal work W, the prefix's history tiles).
+// Pairs run num_sms / 2 at a time.  When the last wave would be partly
+// empty, the query tiles that fill it become a tail: the head's pairs run as
+// whole waves, and the tail's history is split k ways, so the tail costs
+// ceil(pieces / slots) rounds of W / k instead of one more W.  The estimate
+// adds a fixed cost for the split launch and its merge and a cost per round
+// (0.07 W + 0.03 W per round, fitted on a 2,048-query chunk after 30,720
+// positions at 24 / 4 heads, D = 256); the smallest k within 0.05 W of the
+// best is taken, only if it beats the unsplit tail by 0.05 W and leaves
+// every piece 8 history tiles or more.  head = chunk_len, k = 1: one launch.
+struct PfTailPlan {
+  int32_t head, k;
+};
+
+PfTailPlan prefill_tail_plan(int64_t G, int64_t Hkv, int64_t q_start, int64_t chunk_len,
+                             int64_t num_sms) {
+  PfTailPlan p{(int32_t)chunk_len, 1};
+  if (G < 1 || G > kPfRows || Hkv < 1 || num_sms < 2 || chunk_len < 1 || q_start < 4 * chunk_len)
+    return p;
+  const int64_t slots = num_sms / 2;
+  const int64_t qpp = 2 * (kPfRows / G);                // queries per CTA pair
+  const int64_t pph = (chunk_len + qpp - 1) / qpp;      // pairs per KV head
+  const int64_t rem = (pph * Hkv) % slots;
+  if (pph * Hkv <= slots || rem == 0) return p;
+  const int64_t t_tail = (rem + Hkv - 1) / Hkv;         // tail pairs per KV head
+  if (t_tail >= pph) return p;
+  const int64_t c_head = (pph - t_tail) * qpp;
+  const int64_t min_tiles = (q_start + c_head + kPfTile) / kPfTile;   // first tail query's
+  double est[9] = {0};
+  double best = 1e30;
+  for (int s = 2; s <= 8 && min_tiles / s >= 8; ++s) {
+    const int64_t rounds = (t_tail * Hkv * s + slots - 1) / slots;
+    est[s] = (double)rounds / s + 0.07 + 0.03 * (double)rounds;
+    if (est[s] < best) best = est[s];
+  }
+  if (best > 0.95) return p;
+  for (int s = 2; s <= 8; ++s)
+    if (est[s] > 0 && est[s] <= best + 0.05) return PfTailPlan{(int32_t)c_head, s};
+  return p;
+}
+
+// Workspace of the balanced form: the head launch (unsplit) and the tail
+// launch (k splits) run one after the other on the same workspace.
+size_t prefill_tail_workspace(const PfTailPlan& p, int64_t chunk_len, int64_t Hq, int64_t D,
+                              int fmt) {
+  const size_t h = prefill_workspace_bytes(p.head, Hq, D, 1, fmt);
+  const size_t t = prefill_workspace_bytes(chunk_len - p.head, Hq, D, p.k, fmt);
+  return h > t ? h : t;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t jf_prefill_chunk_workspace_bytes(const jf_kv_pool* pool, int32_t q_start,
+                                        int32_t chunk_len, int32_t num_q_heads, int32_t num_sms) {
+  if (check_pool_any(pool)) return 0;
+  if (q_start < 0 || chunk_len < 0 || num_q_heads < 1 || num_sms < 0) return 0;
+  if (num_q_heads % pool->num_kv_heads) return 0;
+  const bool tq = pool->format == JF_FMT_TQ4;
+  const size_t one = tq ? prefill_workspace_bytes(chunk_len, num_q_heads, pool->head_dim, 1,
+                                                  JF_FMT_TQ4)
+                        : jf_prefill_workspace_bytes();
+  const PfTailPlan p = prefill_tail_plan(num_q_heads / pool->num_kv_heads, pool->num_kv_heads,
+                                         q_start, chunk_len, num_sms ? num_sms : sm_count());
+  if (p.k == 1) return one;
+  const size_t bal = prefill_tail_workspace(p, chunk_len, num_q_heads, pool->head_dim,
+                                            pool->format);
+  return bal > one ? bal : one;
+}
+
 int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row, const void* q,
                           int32_t q_start, int32_t chunk_len, int32_t num_q_heads,
                           float softmax_scale, int32_t causal, void* out, void* workspace,
@@ -264,18 +346,37 @@ int jf_prefill_chunk_attn(const jf_kv_pool* pool, const int32_t* page_table_row,
   if (chunk_len == 0) return JF_OK;
   const Geom g = make_geom(*pool);
   if (num_q_heads / pool->num_kv_heads > 128) return JF_ERR_UNSUPPORTED;
+  Tq4Params prm;
   if (tq) {
-    Tq4Params prm;
     st = tq4_make_params(pool->tq4, g.D, &prm);
     if (st) return st;
-    const int64_t row0 = 0;
-    return launch_prefill_batch(g, *pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1,
-                                num_q_heads, softmax_scale, causal, out, workspace,
-                                static_cast<cudaStream_t>(stream), 1, chunk_len, &prm);
   }
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int64_t row0 = 0;
+  const PfTailPlan p = prefill_tail_plan(num_q_heads / pool->num_kv_heads, pool->num_kv_heads,
+                                         q_start, chunk_len, sm_count());
+  if (p.k > 1 && aligned(workspace, 256) &&
+      workspace_bytes >= prefill_tail_workspace(p, chunk_len, num_q_heads, g.D, pool->format)) {
+    // the head's query tiles as whole waves, then the tail's with split histories
+    const size_t row_bytes = (size_t)num_q_heads * g.D * 2;
+    const int32_t t_start = q_start + p.head, t_len = chunk_len - p.head;
+    const void* q_t = static_cast<const uint8_t*>(q) + (size_t)p.head * row_bytes;
+    void* out_t = static_cast<uint8_t*>(out) + (size_t)p.head * row_bytes;
+    st = launch_prefill_batch(g, *pool, &page_table_row, &q_start, &p.head, q, &row0, 1,
+                              num_q_heads, softmax_scale, causal, out, workspace, s, 1, p.head,
+                              tq ? &prm : nullptr);
+    if (st) return st;
+    return launch_prefill_batch(g, *pool, &page_table_row, &t_start, &t_len, q_t, &row0, 1,
+                                num_q_heads, softmax_scale, causal, out_t, workspace, s, p.k,
+                                t_len, tq ? &prm : nullptr);
+  }
+  if (tq)
+    return launch_prefill_batch(g, *pool, &page_table_row, &q_start, &chunk_len, q, &row0, 1,
+                                num_q_heads, softmax_scale, causal, out, workspace, s, 1,
+                                chunk_len, &prm);
   CUtensorMap tmap{};
   return launch_prefill(g, *pool, tmap, page_table_row, q, q_start, chunk_len, num_q_heads,
-                        softmax_scale, causal, out, workspace, static_cast<cudaStream_t>(stream));
+                        softmax_scale, causal, out, workspace, s);
 }
 
 size_t jf_prefill_batch_workspace_bytes(int32_t format, int64_t total_rows, int32_t num_q_heads,

@@ -194,3 +194,30 @@ def test_prefill_batch_rejects_bad_arguments():
     assert need(1, 32, 8, 128, 1) == 256 + (32 * 8 * 8 + 255) // 256 * 256 + 2 * 32 * 8 * 128 * 4
     assert need(5, 32, 8, 128, 1) == 0
     assert call(splits=4, wsb=n - 1) == B.JF_ERR_WORKSPACE_TOO_SMALL
+
+
+def test_prefill_chunk_workspace_plans_the_wave_balance():
+    """Host-only (num_sms given): a 2,048-query chunk after 30,720 positions at
+    24/4/256 has 49 CTA pairs per KV head, 196 in all; 152 SMs run 76 at a time,
+    so the last wave would hold 44.  The tail of 11 pairs per KV head (the last
+    452 queries) is split 3 ways: its workspace holds 3 partials per row."""
+    p = _pool(num_kv_heads=4, head_dim=256, num_pages=128)
+    f = lambda qs, c, hq=24, sms=152: B.lib().jf_prefill_chunk_workspace_bytes(
+        ctypes.byref(p), qs, c, hq, sms)
+    rows = 452 * 24 * 3
+    assert f(30720, 2048) == 256 + -(-rows * 8 // 256) * 256 + rows * 256 * 4
+    assert f(30720, 2048) == B.lib().jf_prefill_batch_workspace_bytes(0, 452, 24, 256, 3)
+    minimal = B.jf_prefill_workspace_bytes()
+    assert f(0, 2048) == minimal            # short prefix: unequal pairs, one launch
+    assert f(30720, 798) == minimal         # 76 pairs: one wave
+    assert f(30720, 1596) == minimal        # 152 pairs: two whole waves
+    assert f(30720, 2394) == minimal        # 228 pairs: three whole waves
+    assert f(30720, 2048, sms=196 * 2) == minimal   # all pairs at once
+    assert f(30720, 2048, hq=23) == 0       # Hq % Hkv
+    assert f(-1, 2048) == 0
+    # a TQ4 pool's minimum (its rotated queries and partials) already covers
+    # the balanced form's two launches
+    codec = _codec(256)
+    t = _tq4_pool(codec, num_kv_heads=4, head_dim=256, num_pages=128)
+    g = B.lib().jf_prefill_chunk_workspace_bytes(ctypes.byref(t), 30720, 2048, 24, 152)
+    assert g == B.lib().jf_prefill_batch_workspace_bytes(1, 2048, 24, 256, 1)

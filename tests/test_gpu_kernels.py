@@ -481,6 +481,53 @@ def test_prefill_32k_prefix_sampled_rows():
             assert_attention_close(out[i:i + 1, kvh * G:(kvh + 1) * G], ref)
 
 
+def _whole_waves(pairs):
+    slots = torch.cuda.get_device_properties(0).multi_processor_count // 2
+    return pairs <= slots or pairs % slots == 0
+
+
+# rows on both sides of the head/tail boundaries the wave balance can choose
+# for this chunk (1,596 on 152 SMs) and the chunk's ends
+BALANCE_ROWS = (0, 1, 1511, 1512, 1553, 1554, 1595, 1596, 1597, 1800, 2047)
+
+
+def test_prefill_wave_balanced_chunk():
+    """2,048 queries after 30,720 positions (24/4/256, P 256): 196 CTA pairs,
+    not whole waves of the pairs the GPU runs at once.  With the workspace
+    jf_prefill_chunk_workspace_bytes asks for, the chunk runs as whole waves
+    plus a tail whose histories are split; sampled rows against the oracle,
+    every row against the one-launch form (minimal workspace)."""
+    Hq, Hkv, D, P, C = 24, 4, 256, 256, 2048
+    q_start = 32768 - C
+    if _whole_waves(Hkv * -(-C // 42)):
+        pytest.skip("the chunk fills whole waves on this GPU")
+    case = make_case(406, Hq, Hkv, D, P, [32768])
+    pool = gpu_append(case)
+    from paper_2609_17475_gb300 import synth
+    q = synth.normal_bf16(synth.generator(407), (C, Hq, D))
+    ws = jf.prefill_chunk_workspace(pool, q_start, C, Hq, device=DEV)
+    assert ws.numel() > jf.jf_prefill_workspace_bytes()
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), q_start, 1 / 16, True,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    one = gpu_prefill(case, pool, q, q_start, True, 1 / 16)
+    assert torch.isfinite(out.float()).all()
+    diff = (out.float() - one.float()).abs()
+    assert diff.max().item() <= 1e-2 and diff.mean().item() <= 1e-4, (diff.max(), diff.mean())
+    G = Hq // Hkv
+    for kvh in (0, 3):
+        L1 = OA.PoolLayout(1, P, D)
+        opool = OA.new_pool(L1, case.num_pages)
+        OA.append(opool, L1, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
+                  bits(case.k[:, kvh:kvh + 1]), bits(case.v[:, kvh:kvh + 1]))
+        for i in BALANCE_ROWS:
+            ref = OT.paged_decode(opool, L1, case.page_table.numpy(), [q_start + i + 1],
+                                  bits(q[i:i + 1, kvh * G:(kvh + 1) * G]), 1 / 16)
+            assert_attention_close(out[i:i + 1, kvh * G:(kvh + 1) * G], ref)
+
+
 def test_prefill_poison_pages_never_leak():
     case = make_case(77, 8, 2, 128, 64, [300], num_pages=12)
     ref_pool = case.oracle_pool(fill=0xFF)

@@ -402,6 +402,41 @@ def test_tq4_decode_full_window_256k_one_head():
                                   opool[page, o1:o1 + 2 * geo.page_size])
 
 
+def test_tq4_prefill_wave_balanced_chunk():
+    """2,048 queries after 30,720 TQ4 positions (24/4/256, P 256): 196 CTA
+    pairs, not whole waves, and the TQ4 minimum workspace already holds the
+    balanced form (whole waves, then a tail with split histories), so the
+    plain call runs it; sampled rows against the oracle's decode."""
+    Hq, Hkv, D, P, C = 24, 4, 256, 256, 2048
+    q_start = 32768 - C
+    slots = torch.cuda.get_device_properties(0).multi_processor_count // 2
+    pairs = Hkv * -(-C // 42)
+    if pairs <= slots or pairs % slots == 0:
+        pytest.skip("the chunk fills whole waves on this GPU")
+    case = make_case(408, Hq, Hkv, D, P, [32768])
+    pool = gpu_append(case)
+    q = synth.normal_bf16(synth.generator(409), (C, Hq, D))
+    ws = jf.prefill_batch_workspace(C, Hq, D, 1, device=DEV, format=jf.JF_FMT_TQ4)
+    assert jf.jf_prefill_chunk_workspace_bytes(pool, q_start, C, Hq) == ws.numel()
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device=DEV)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), q_start, 1 / 16, True,
+                             out, ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    assert torch.isfinite(out.float()).all()
+    sk, sv = signs(D)
+    G = Hq // Hkv
+    L1 = OQ.Tq4Layout(1, P, D, OQ.make_codec(D, sk, sv))
+    for kvh in (1, 2):
+        opool = OQ.new_pool(L1, case.num_pages)
+        OQ.append(opool, L1, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
+                  bits(case.k[:, kvh:kvh + 1]), bits(case.v[:, kvh:kvh + 1]))
+        for i in (0, 1511, 1512, 1553, 1554, 1595, 1596, 1597, 2047):
+            ref = OT.paged_decode(opool, L1, case.page_table.numpy(), [q_start + i + 1],
+                                  bits(q[i:i + 1, kvh * G:(kvh + 1) * G]), 1 / 16)
+            assert_attention_close(out[i:i + 1, kvh * G:(kvh + 1) * G], ref)
+
+
 # --------------------------------------------------------------------------
 # prefill chunk attention over TQ4 pages
 # --------------------------------------------------------------------------
