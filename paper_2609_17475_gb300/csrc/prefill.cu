@@ -199,18 +199,22 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = tc::cluster_rank();
+  // CTA pairs in launch order: the KV heads of one pair of query tiles are
+  // consecutive, so every head's longest tiles start in the first wave
+  const int pair = (int)(blockIdx.x >> 1);
+  const int kvh = pair % a.Hkv;
+  const int tile = (pair / a.Hkv) * 2 + (int)(blockIdx.x & 1);
   // this CTA's request (tile ranges ascend with the request index)
   int ri = 0;
   for (int i = 1; i < a.nreq; ++i)
-    if ((int)blockIdx.x >= a.req[i].tile0) ri = i;
+    if (tile >= a.req[i].tile0) ri = i;
   const PfReq& rq = a.req[ri];
   const int32_t* const pt = rq.pt;
   const int q_start = rq.q_start, C = rq.C;
-  const int bx = (int)blockIdx.x - rq.tile0;
+  const int bx = tile - rq.tile0;
   // query tile of this CTA and of its partner: latest (longest) tiles first
   const int qt = rq.n_tiles2 - 1 - bx;
   const int qt_partner = rq.n_tiles2 - 1 - (bx ^ 1);
-  const int kvh = blockIdx.y;
   const int q0 = qt * a.QPC;
   const int nq = max(0, min(a.QPC, C - q0));
   const int rows = nq * a.G;
@@ -844,8 +848,8 @@ int launch_prefill_batch(const Geom& g, const jf_kv_pool& pool, const int32_t* c
     tiles += r.n_tiles2;
   }
   a.nreq = n;
-  if (tiles > 0x7FFFFFFF || g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
-  dim3 grid((unsigned)tiles, (unsigned)g.Hkv, (unsigned)num_splits);
+  if (tiles * g.Hkv > 0x7FFFFFFF || g.Hkv > 65535) return JF_ERR_UNSUPPORTED;
+  dim3 grid((unsigned)(tiles * g.Hkv), 1u, (unsigned)num_splits);
   const int64_t rows = total_rows * Hq;
   const int64_t rblocks = (rows + 7) / 8;   // 8 warps per CTA, one row each
   if (rblocks > 0x7FFFFFFF) return JF_ERR_UNSUPPORTED;
