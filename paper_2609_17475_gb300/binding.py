@@ -336,14 +336,23 @@ def verify_workspace(batch, q_len, num_q_heads, num_kv_heads, head_dim, num_spli
                             device=device)
 
 
+def _num_sms(device, num_sms) -> int:
+    """num_sms when given (planning for a GPU of that size), else the SM count
+    of `device` (the current one when None)."""
+    if num_sms is not None:
+        return int(num_sms)
+    dev = device if device is not None else torch.cuda.current_device()
+    return torch.cuda.get_device_properties(dev).multi_processor_count
+
+
 def default_verify_splits(batch: int, q_len: int, num_q_heads: int, num_kv_heads: int,
-                          device=None, format: int = JF_FMT_AFFINE4_G64) -> int:
+                          device=None, format: int = JF_FMT_AFFINE4_G64,
+                          num_sms: Optional[int] = None) -> int:
     """Split cap for the verifier: each split of a KV head runs
     ceil(G * q_len / 8) CTAs, so fewer splits fill the GPU (two split CTAs per
     SM for the affine format, one for TQ4)."""
     nt = -(-(num_q_heads // num_kv_heads) * q_len // 8)
-    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    slots = (1 if format == JF_FMT_TQ4 else 2) * props.multi_processor_count
+    slots = (1 if format == JF_FMT_TQ4 else 2) * _num_sms(device, num_sms)
     per = slots // (batch * num_kv_heads * nt)   # one full wave
     return max(1, per if batch == 1 else per + 2)
 
@@ -422,7 +431,7 @@ def prefill_chunk_workspace(pool: "KVPool", q_start: int, chunk_len: int, num_q_
 
 
 def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: int,
-                           device=None) -> int:
+                           device=None, num_sms: Optional[int] = None) -> int:
     """History splits for a launch.  The kernel runs one CTA per SM, two per
     pair, so SMs / 2 pairs run at once; each candidate split count is scored
     by its makespan when the pairs' history tiles (64 positions each, plus a
@@ -440,8 +449,7 @@ def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: i
             work += [-(-(int(s0) + last) // 64)] * num_kv_heads
     if not work:
         return 1
-    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    slots = max(1, props.multi_processor_count // 2)
+    slots = max(1, _num_sms(device, num_sms) // 2)
     longest = max(work)
     scores = []
     for S in [1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 12, 14, 16, 20, 24, 32, 48, 64]:
@@ -525,14 +533,13 @@ def jf_kv_restore(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
 
 
 def default_num_splits(batch: int, num_kv_heads: int, device=None,
-                       format: int = JF_FMT_AFFINE4_G64) -> int:
+                       format: int = JF_FMT_AFFINE4_G64, num_sms: Optional[int] = None) -> int:
     """Split cap per (request, KV head) so the split grid fills every SM slot
     once (two split CTAs per SM for the affine format, one for TQ4, whose
     centroid table takes a CTA's spare shared memory).  A batch plans its
     splits over all requests together, and its workspace then needs room for
     about two more splits per request than an even share (rounding up per
     request)."""
-    props = torch.cuda.get_device_properties(device if device is not None else torch.cuda.current_device())
-    target = (1 if format == JF_FMT_TQ4 else 2) * props.multi_processor_count
+    target = (1 if format == JF_FMT_TQ4 else 2) * _num_sms(device, num_sms)
     per = -(-target // (batch * num_kv_heads))
     return max(1, per if batch == 1 else per + 2)

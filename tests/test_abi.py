@@ -221,3 +221,23 @@ def test_prefill_chunk_workspace_plans_the_wave_balance():
     t = _tq4_pool(codec, num_kv_heads=4, head_dim=256, num_pages=128)
     g = B.lib().jf_prefill_chunk_workspace_bytes(ctypes.byref(t), 30720, 2048, 24, 152)
     assert g == B.lib().jf_prefill_batch_workspace_bytes(1, 2048, 24, 256, 1)
+
+
+def test_split_planners_on_a_152_sm_gpu():
+    """The host split planners with the SM count given (no device touched),
+    against the split counts the benchmark runs on a 152-SM GB300."""
+    # decode: one wave of 2 split CTAs per SM (affine), 1 per SM (TQ4)
+    assert B.default_num_splits(1, 4, num_sms=152) == 76
+    assert B.default_num_splits(1, 4, num_sms=152, format=B.JF_FMT_TQ4) == 38
+    assert B.default_num_splits(2, 4, num_sms=152) == 38 + 2      # batch: even share + 2
+    # verifier: ceil(G q_len / 8) CTAs per split (24 / 4 heads: 2, 3, 3)
+    assert [B.default_verify_splits(1, L, 24, 4, num_sms=152) for L in (2, 3, 4)] == [38, 25, 25]
+    assert [B.default_verify_splits(1, L, 24, 4, num_sms=152, format=B.JF_FMT_TQ4)
+            for L in (2, 3, 4)] == [19, 12, 12]
+    # prefill history splits (24 / 4 heads, 42 queries per CTA pair)
+    ps = lambda qs, cl: B.default_prefill_splits(qs, cl, 24, 4, num_sms=152)
+    assert ps([32704], [64]) == 9          # 4 pairs walking 512 tiles each
+    assert ps([30720], [2048]) == 3
+    assert ps([4096 * (b + 1) - 64 for b in range(8)], [64] * 8) == 2
+    assert ps([4096 * (b + 1) - 512 for b in range(8)], [512] * 8) == 1
+    assert ps([0], [0]) == 1               # nothing to schedule
