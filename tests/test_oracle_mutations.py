@@ -3,7 +3,10 @@
 Each case plants one mistake in the oracle (on the CPU, via monkeypatch) and
 checks that at least one pin test now fails: a dropped term, a wrong divisor,
 the wrong tie direction, swapped nibbles, a transposed GQA map, a missing
-softmax scale, an off-by-one causal bound, a wrong page lookup.
+softmax scale, an off-by-one causal bound, a wrong page lookup, a merge
+without the max rescale, split ranges that drop a position, checkpoint
+records in physical instead of logical order, restore into the wrong pages,
+and a reservation without the output cap or rounded down.
 """
 import numpy as np
 import pytest
@@ -200,3 +203,65 @@ def test_tq4_quantile_offset_is_caught(monkeypatch):
         return np.array([x[np.searchsorted(cdf, k / 16.0)] for k in range(16)])
     monkeypatch.setattr(Q, "quantile_init", bad)
     assert _fails(TT.test_quantile_start_is_the_beta_quantile, 256)
+
+
+# -- split merge (Eq. 3 workspace), checkpoint / restore (Sec. 3.4), Eq. 7 -----
+import oracle.checkpoint as C
+import oracle.reservation as R
+from tests import test_oracle_reservation as TR
+
+
+def test_merge_without_max_rescale_is_caught(monkeypatch):
+    def bad(parts):
+        return sum(o for _, _, o in parts) / sum(l for _, l, _ in parts)
+    monkeypatch.setattr(T, "merge_partials", bad)
+    assert _fails(TA.test_split_merge_equals_plain_softmax, 3)
+
+
+def test_merge_rescaling_only_the_sums_is_caught(monkeypatch):
+    def bad(parts):
+        m_star = max(m for m, _, _ in parts)
+        return (sum(o for _, _, o in parts) /
+                sum(np.exp(m - m_star) * l for m, l, _ in parts))
+    monkeypatch.setattr(T, "merge_partials", bad)
+    assert _fails(TA.test_split_merge_equals_plain_softmax, 2)
+
+
+def test_split_bounds_dropping_the_last_position_are_caught(monkeypatch):
+    orig = T.split_bounds
+
+    def bad(ctx, num_splits):
+        b = orig(ctx, num_splits)
+        return b[:-1] + [(b[-1][0], b[-1][1] - 1)] if b[-1][1] - 1 > b[-1][0] else b
+    monkeypatch.setattr(T, "split_bounds", bad)
+    assert _fails(TA.test_split_bounds_cover_exactly)
+
+
+def test_checkpoint_in_physical_page_order_is_caught(monkeypatch):
+    orig = C.checkpoint
+
+    def bad(pool, page_table_row, num_pages):
+        return orig(pool, np.sort(np.asarray(page_table_row)[:num_pages]), num_pages)
+    monkeypatch.setattr(C, "checkpoint", bad)
+    assert _fails(TA.test_checkpoint_bytes_and_restore_round_trip)
+
+
+def test_restore_to_logical_slots_is_caught(monkeypatch):
+    def bad(pool, page_table_row, num_pages, blob):
+        pb = pool.shape[1]
+        for k in range(num_pages):
+            pool[k] = blob[k * pb:(k + 1) * pb]
+    monkeypatch.setattr(C, "restore", bad)
+    assert _fails(TA.test_checkpoint_bytes_and_restore_round_trip)
+
+
+def test_reservation_without_the_output_cap_is_caught(monkeypatch):
+    monkeypatch.setattr(R, "reservation_pages",
+                        lambda p, o, g_out=8192, page_size=256: -(-(p + o) // page_size))
+    assert _fails(TR.test_paper_policy_numbers)
+
+
+def test_reservation_rounding_down_is_caught(monkeypatch):
+    monkeypatch.setattr(R, "reservation_pages",
+                        lambda p, o, g_out=8192, page_size=256: (p + min(o, g_out)) // page_size)
+    assert _fails(TR.test_reservation_matches_brute_force_and_library, 257, 0, 8192, 256)
