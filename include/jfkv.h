@@ -57,6 +57,10 @@ extern "C" {
 #define JF_DEV_ERR_POSITION   2   /* position beyond the page-table row, or
                                      a request index out of range          */
 #define JF_DEV_ERR_TIMEOUT    4   /* a bounded wait on a copy gave up      */
+#define JF_DEV_ERR_LAYOUT     8   /* the kernel's dynamic shared-memory
+                                     window was not 1024-byte aligned (the
+                                     swizzled copies need it); the CTA did
+                                     no work                               */
 
 /* ---- formats -------------------------------------------------------- */
 #define JF_FMT_AFFINE4_G64 0      /* affine 4-bit, 64-element groups (above) */

@@ -20,9 +20,9 @@ What the paper fixes (Sec. 3.1 Eq. 4; App. A.1 Table 3; Sec. 2 Eq. 2)
   FP16 norm; Eq. 2 counts 16 * 2 * 4 * (128 + 2) bytes per position for the
   paper's 16 layers x 4 KV heads.
 * Signs: NumPy ``default_rng(seed + d * 7919)`` sampling +-1; K seed 0, V
-  seed 1.  Random draws are inputs here: ``tq4_signs`` in the product
-  package's seeded-input module draws them, and every function below takes the
-  sign vectors as arguments.
+  seed 1.  ``sign_vector`` is this module's reading of that rule; the codec
+  functions take sign vectors as arguments, and the tests require the seeded
+  inputs the CUDA path is given to equal ``sign_vector``'s.
 
 Readings taken where the paper is silent
 ----------------------------------------
@@ -34,8 +34,9 @@ Readings taken where the paper is silent
   centroid); the loop ends after the update whose largest change is below
   1e-6, or after 100 updates.  The fp64 result is rounded to fp32.
 * Encoding thresholds are fp32: t_k = fp32(fp32(c_k + c_{k+1}) * 0.5).
-* Sign draw: ``rng.choice([-1.0, 1.0], size=d)``, which is the same draw as
-  ``2 * rng.integers(0, 2, size=d) - 1``.
+* Sign draw: one ``rng.integers(0, 2)`` per coordinate, 0 -> -1 and 1 -> +1
+  (``2 * rng.integers(0, 2, size=d) - 1``, which is also the draw
+  ``rng.choice([-1, 1], size=d)`` makes).
 * H_d is Sylvester's ordering, H[i, j] = (-1)^popcount(i & j).
 * The index decision is exact: with u = H_d S x (exact in fp64 for bf16
   inputs whose nonzero magnitudes span less than 2^37) and
@@ -136,6 +137,17 @@ def hadamard(d: int) -> np.ndarray:
         pop += bits & 1
         bits >>= 1
     return np.where(pop % 2 == 0, 1.0, -1.0)
+
+
+SEED_K, SEED_V = 0, 1   # Table 3's default K and V seeds
+
+
+def sign_vector(seed: int, d: int) -> np.ndarray:
+    """The random-sign diagonal S of Table 3 for head_dim d, fp64 [d] of +-1:
+    NumPy ``default_rng(seed + d * 7919)``, one uniform bit per coordinate,
+    0 -> -1 and 1 -> +1 (module header: sign draw)."""
+    rng = np.random.default_rng(int(seed) + int(d) * 7919)
+    return (2 * rng.integers(0, 2, size=int(d)) - 1).astype(np.float64)
 
 
 @dataclasses.dataclass(frozen=True)

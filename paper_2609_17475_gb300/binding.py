@@ -24,6 +24,7 @@ JF_ERR_CUDA = -4
 JF_DEV_ERR_PAGE_ID = 1
 JF_DEV_ERR_POSITION = 2
 JF_DEV_ERR_TIMEOUT = 4
+JF_DEV_ERR_LAYOUT = 8
 JF_FMT_AFFINE4_G64 = 0
 JF_FMT_TQ4 = 1
 

@@ -187,4 +187,9 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// Host: raise a kernel's dynamic shared-memory limit to `bytes` on the
+// current device, once per (kernel, device); thread-safe.  The attribute is
+// per device, so a process that launches on several GPUs opts in on each.
+int smem_optin(const void* kernel, int bytes);
+
 }  // namespace jfkv

@@ -35,6 +35,9 @@
 //   o = sum_s 2^{m_s - m*} O_s / sum_s 2^{m_s - m*} l_s.
 #include <cmath>
 #include <cfloat>
+#include <mutex>
+#include <utility>
+#include <vector>
 
 #include "decode.cuh"
 #include "quant.cuh"
@@ -418,12 +421,12 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     nsplit = plan_sh[2];
     cps = plan_sh[3];
     if (b < 0) return;   // past the batch's last split
-    ctx = checked_ctx(a, b);
+    ctx = checked_ctx(a, b, split);
     nch = (ctx + DTOK - 1) / DTOK;
   } else {
     split = blockIdx.x;
     b = blockIdx.z;
-    ctx = checked_ctx(a, b);
+    ctx = checked_ctx(a, b, split);
     split_plan(ctx, a.num_splits, nch, cps, nsplit);
   }
   if (split >= nsplit) {
@@ -440,7 +443,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   auto chunk_of = [&](int it) { return c_begin + warp + it * DWARPS; };
 
   if (!aligned) {
-    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
+    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_LAYOUT);
     return;
   }
   if (a.knew != nullptr && split == nsplit - 1) {   // owns the last chunk
@@ -823,6 +826,8 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   }
   int ctx = ctx_raw;
   const int64_t cap = (int64_t)a.pt_stride * a.P;
+  if ((ctx < 0 || ctx > cap) && t == 0 && blockIdx.x == 0 && hq == 0)
+    flag_error(a.status, JF_DEV_ERR_POSITION);   // also covers requests with no split
   if (ctx < 0) ctx = 0;
   if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
@@ -901,6 +906,21 @@ int sm_count() {
   return cache[dev];
 }
 
+int smem_optin(const void* kernel, int bytes) {
+  static std::mutex mu;
+  static std::vector<std::pair<const void*, int>> done;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return JF_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(mu);
+  for (const auto& e : done)
+    if (e.first == kernel && e.second == dev) return JF_OK;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) !=
+      cudaSuccess)
+    return JF_ERR_CUDA;
+  done.emplace_back(kernel, dev);
+  return JF_OK;
+}
+
 // rows (positions) of one TMA box of the decode code tensor map
 int decode_box_rows() { return DTOK; }
 
@@ -932,15 +952,9 @@ template <int D>
 static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
                            cudaStream_t stream) {
   using L = DecodeSmem<D>;
-  static bool attr_done = false;
-  if (!attr_done) {
-    if (cudaFuncSetAttribute(decode_split_kernel<D, false>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, L::TOTAL) != cudaSuccess ||
-        cudaFuncSetAttribute(decode_split_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             L::TOTAL) != cudaSuccess)
-      return JF_ERR_CUDA;
-    attr_done = true;
-  }
+  if (smem_optin((const void*)decode_split_kernel<D, false>, L::TOTAL) != JF_OK ||
+      smem_optin((const void*)decode_split_kernel<D, true>, L::TOTAL) != JF_OK)
+    return JF_ERR_CUDA;
   // Both kernels use programmatic dependent launch: each may be scheduled
   // while the previous kernel in the stream drains, and waits (griddepcontrol)
   // before it reads anything that kernel wrote.

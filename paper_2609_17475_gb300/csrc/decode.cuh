@@ -103,11 +103,14 @@ static __device__ BalPlan balanced_plan(const DecodeArgs& a, int x, int want_b, 
   return p;
 }
 
-__device__ __forceinline__ int checked_ctx(const DecodeArgs& a, int b) {
+// Context length of request b clamped to [0, pt_stride * P].  An out-of-range
+// value is reported by the CTAs that own split 0 of request b (every request
+// with at least one chunk has one; the merge kernel reports the others).
+__device__ __forceinline__ int checked_ctx(const DecodeArgs& a, int b, int split) {
   int ctx = a.ctx[b];
   const int64_t cap = (int64_t)a.pt_stride * a.P;
   if (ctx < 0 || ctx > cap) {
-    if (threadIdx.x == 0 && blockIdx.x == 0) flag_error(a.status, JF_DEV_ERR_POSITION);
+    if (threadIdx.x == 0 && split == 0) flag_error(a.status, JF_DEV_ERR_POSITION);
     ctx = ctx < 0 ? 0 : (int)cap;
   }
   return ctx;

@@ -762,16 +762,11 @@ size_t prefill_workspace_bytes(int64_t rows, int64_t Hq, int64_t D, int64_t S, i
 }
 
 // One prefill launch of a given instantiation (its shared-memory opt-in is
-// set once per instantiation).
+// set once per instantiation and device).
 template <int D, int FMT>
 static int launch_pf(const dim3& grid, const PrefillArgs& a, cudaStream_t stream) {
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(prefill_kernel<D, FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             PfSmem<D, FMT>::TOTAL) != cudaSuccess)
-      return JF_ERR_CUDA;
-    attr = true;
-  }
+  if (smem_optin((const void*)prefill_kernel<D, FMT>, PfSmem<D, FMT>::TOTAL) != JF_OK)
+    return JF_ERR_CUDA;
   prefill_kernel<D, FMT><<<grid, PF_THREADS, PfSmem<D, FMT>::TOTAL, stream>>>(a);
   return cudaGetLastError() == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }

@@ -644,12 +644,12 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     nsplit = misc[2];
     cps = misc[3];
     if (b < 0) return;
-    ctx = checked_ctx(a, b);
+    ctx = checked_ctx(a, b, split);
     nch = (ctx + DTOK - 1) / DTOK;
   } else {
     split = blockIdx.x;
     b = blockIdx.z;
-    ctx = checked_ctx(a, b);
+    ctx = checked_ctx(a, b, split);
     split_plan(ctx, a.num_splits, nch, cps, nsplit);
   }
   if (split >= nsplit) {
@@ -660,7 +660,7 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     return;
   }
   if (!aligned) {
-    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
+    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_LAYOUT);
     return;
   }
   const int c_begin = split * cps;
@@ -935,14 +935,8 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
 template <int D, bool VER, bool APP>
 static int launch_tq4_split(const cudaLaunchConfig_t& cfg0, const CUtensorMap& tmap,
                             const DecodeArgs& a, const Tq4Params& prm) {
-  static bool attr = false;   // one per instantiation
-  if (!attr) {
-    if (cudaFuncSetAttribute(tq4_split_kernel<D, VER, APP>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             Tq4Smem<D>::TOTAL) != cudaSuccess)
-      return JF_ERR_CUDA;
-    attr = true;
-  }
+  if (smem_optin((const void*)tq4_split_kernel<D, VER, APP>, Tq4Smem<D>::TOTAL) != JF_OK)
+    return JF_ERR_CUDA;
   cudaLaunchConfig_t cfg = cfg0;
   cfg.dynamicSmemBytes = Tq4Smem<D>::TOTAL;
   return cudaLaunchKernelEx(&cfg, tq4_split_kernel<D, VER, APP>, tmap, a, prm) == cudaSuccess

@@ -358,6 +358,27 @@ def test_decode_reports_bad_page_id():
     assert jf.workspace_status(ws) & jf.binding.JF_DEV_ERR_PAGE_ID
 
 
+@pytest.mark.parametrize("splits", [1, 4])
+@pytest.mark.parametrize("bad", ["past_row", "negative"])
+def test_decode_flags_a_bad_context_of_a_later_request(splits, bad):
+    """A context length outside [0, pt_stride * P] of the last request of a
+    batch sets JF_DEV_ERR_POSITION (per-request and batch split plans)."""
+    case = make_case(81, 8, 2, 128, 64, [300, 500, 200])
+    pool = pool_from_numpy(case, case.oracle_pool())
+    pt = case.page_table
+    ctx = [300, 500, pt.shape[1] * 64 + 1 if bad == "past_row" else -5]
+    out = torch.empty(3, 8, 128, dtype=torch.bfloat16, device=DEV)
+    ws = jf.decode_workspace(3, 8, 2, 128, splits, device=DEV)
+    jf.jf_paged_decode_attn(pool, pt.to(DEV), torch.tensor(ctx, dtype=torch.int32, device=DEV),
+                            case.q.to(DEV), 0.1, out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) & jf.binding.JF_DEV_ERR_POSITION
+    # the valid requests are still right
+    ref = OT.paged_decode(case.oracle_pool(), case.layout, case.page_table.numpy(),
+                          [300, 500, 0], bits(case.q), 0.1)
+    assert_attention_close(out[:2], ref[:2])
+
+
 def test_decode_full_window_256k_sampled_heads():
     """The 256K full-window workload (24/4/256, 1,024 pages in a random physical
     order, 4 K channels per KV head x20) at full size, in the launch shape the

@@ -20,12 +20,17 @@ DEV = "cuda"
 
 
 def signs(D):
+    """Sign vectors for the CUDA path (seeded inputs; equal to the oracle's
+    ``sign_vector`` by a CPU test)."""
     return synth.tq4_signs(synth.TQ4_SEED_K, D), synth.tq4_signs(synth.TQ4_SEED_V, D)
 
 
+def oracle_codec(D):
+    return OQ.make_codec(D, OQ.sign_vector(OQ.SEED_K, D), OQ.sign_vector(OQ.SEED_V, D))
+
+
 def oracle_layout(case):
-    sk, sv = signs(case.D)
-    return OQ.Tq4Layout(case.Hkv, case.P, case.D, OQ.make_codec(case.D, sk, sv))
+    return OQ.Tq4Layout(case.Hkv, case.P, case.D, oracle_codec(case.D))
 
 
 def oracle_pool(case, fill=0):
@@ -143,7 +148,8 @@ def test_tq4_append_close_thresholds_take_the_exact_path_everywhere():
     assert np.diff(np.float32(16) * OQ.thresholds(c)).min() < 2 ** -12
     sk, sv = signs(D)
     case = make_case(21, 2 * Hkv, Hkv, D, 64, [300], num_pages=6)
-    lay = OQ.Tq4Layout(Hkv, 64, D, OQ.Codec(D, c, sk.astype(np.float64), sv.astype(np.float64)))
+    lay = OQ.Tq4Layout(Hkv, 64, D, OQ.Codec(D, c, OQ.sign_vector(OQ.SEED_K, D),
+                                            OQ.sign_vector(OQ.SEED_V, D)))
     ref = OQ.new_pool(lay, case.num_pages)
     OQ.append(ref, lay, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),
               bits(case.k), bits(case.v))
@@ -384,7 +390,7 @@ def test_tq4_decode_full_window_256k_one_head():
     torch.cuda.synchronize()
     assert int(err.item()) == 0 and jf.workspace_status(ws) == 0
     G, kvh = geo.group, 2
-    L1 = OQ.Tq4Layout(1, geo.page_size, geo.head_dim, OQ.make_codec(geo.head_dim, sk, sv))
+    L1 = OQ.Tq4Layout(1, geo.page_size, geo.head_dim, oracle_codec(geo.head_dim))
     opool = OQ.new_pool(L1, npages)
     OQ.append(opool, L1, pt.numpy(), req.numpy(), pos.numpy(),
               bits(k[:, kvh:kvh + 1]), bits(v[:, kvh:kvh + 1]))
@@ -426,7 +432,7 @@ def test_tq4_prefill_wave_balanced_chunk():
     assert torch.isfinite(out.float()).all()
     sk, sv = signs(D)
     G = Hq // Hkv
-    L1 = OQ.Tq4Layout(1, P, D, OQ.make_codec(D, sk, sv))
+    L1 = OQ.Tq4Layout(1, P, D, oracle_codec(D))
     for kvh in (1, 2):
         opool = OQ.new_pool(L1, case.num_pages)
         OQ.append(opool, L1, case.page_table.numpy(), case.req.numpy(), case.pos.numpy(),

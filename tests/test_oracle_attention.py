@@ -184,6 +184,25 @@ def test_page_permutation_invariance_is_exact():
     assert np.array_equal(a, b)
 
 
+def test_page_size_invariance_is_exact():
+    """The same logical rows in pools of 64-, 128- and 256-position pages
+    (each with its own shuffled page order) give bitwise the same output."""
+    Hq, Hkv, D, ctx = 8, 2, 256, [700, 130]
+    rng = np.random.default_rng(21)
+    kb = [bf16_bits(torch.randn(c, Hkv, D, generator=torch.Generator().manual_seed(c))
+                    .to(torch.bfloat16)) for c in ctx]
+    vb = [bf16_bits(torch.randn(c, Hkv, D, generator=torch.Generator().manual_seed(c + 1))
+                    .to(torch.bfloat16)) for c in ctx]
+    qb = bf16_bits(torch.randn(len(ctx), Hq, D, generator=torch.Generator().manual_seed(3))
+                   .to(torch.bfloat16))
+    outs = []
+    for P in (64, 128, 256):
+        L = A.PoolLayout(Hkv, P, D)
+        pool, pt = _pool_from_dense(L, kb, vb, ctx, rng)
+        outs.append(T.paged_decode(pool, L, pt, ctx, qb, 1 / 16))
+    assert np.array_equal(outs[0], outs[1]) and np.array_equal(outs[0], outs[2])
+
+
 @pytest.mark.parametrize("splits", [1, 2, 3, 7, 64])
 def test_split_merge_equals_plain_softmax(splits):
     Hq, Hkv, D, P, ctx = 4, 2, 128, 64, [257, 40]

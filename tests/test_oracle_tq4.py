@@ -33,8 +33,7 @@ GOLD = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "tq4_cas
 
 
 def _codec(d=256):
-    return tq4.make_codec(d, synth.tq4_signs(synth.TQ4_SEED_K, d),
-                          synth.tq4_signs(synth.TQ4_SEED_V, d))
+    return tq4.make_codec(d, tq4.sign_vector(tq4.SEED_K, d), tq4.sign_vector(tq4.SEED_V, d))
 
 
 def _density(d):
@@ -50,6 +49,34 @@ def _continuous_update(c, d):
         den = integrate.quad(f, t[k], t[k + 1], epsabs=1e-15, epsrel=1e-13)[0]
         out[k] = num / den
     return out
+
+
+# -- random signs (Table 3) ------------------------------------------------------
+@pytest.mark.parametrize("d", [3, 64, 128, 256])
+@pytest.mark.parametrize("seed", [0, 1, 7])
+def test_seeded_input_signs_equal_the_oracle_rule(seed, d):
+    """The sign vectors handed to the CUDA path (the seeded-input module) are
+    the oracle's reading of Table 3's rule, entry for entry."""
+    s = synth.tq4_signs(seed, d)
+    assert s.dtype == np.int8
+    assert np.array_equal(s.astype(np.float64), tq4.sign_vector(seed, d))
+    assert (synth.TQ4_SEED_K, synth.TQ4_SEED_V) == (tq4.SEED_K, tq4.SEED_V) == (0, 1)
+
+
+def test_sign_rule_seed_offset_is_d_times_7919():
+    """Table 3 seeds the generator with seed + d * 7919: the draw for (seed, d)
+    and for (seed + 7919, d - 1) start from the same generator state, so the
+    shorter vector is a prefix of the longer one; any other offset breaks it."""
+    for d in (64, 128, 256):
+        a = tq4.sign_vector(3, d)
+        b = tq4.sign_vector(3 + 7919, d - 1)
+        assert np.array_equal(a[:d - 1], b)
+        assert not np.array_equal(a[:d - 1], tq4.sign_vector(3 + 7918, d - 1))
+        assert set(np.unique(a)) == {-1.0, 1.0}
+        # K and V (seeds 0 and 1) get different diagonals; about half the signs are negative
+        k, v = tq4.sign_vector(0, d), tq4.sign_vector(1, d)
+        assert not np.array_equal(k, v)
+        assert abs(int((k < 0).sum()) - d // 2) < 4 * math.sqrt(d)
 
 
 # -- rotation ------------------------------------------------------------------
