@@ -57,6 +57,11 @@ extern "C" {
 #define JF_DEV_ERR_POSITION   2   /* position beyond the page-table row, or
                                      a request index out of range          */
 #define JF_DEV_ERR_TIMEOUT    4   /* a bounded wait on a copy gave up      */
+#define JF_DEV_ERR_RANGE     16   /* prefill met an affine K/V group whose
+                                     fp16 reconstruction can overflow
+                                     (|bias| + 15 scale >= 65504, or a
+                                     non-finite scale/bias word): outputs
+                                     reading it are not reliable           */
 #define JF_DEV_ERR_LAYOUT     8   /* the kernel's dynamic shared-memory
                                      window was not 1024-byte aligned (the
                                      swizzled copies need it); the CTA did
@@ -279,6 +284,13 @@ int jf_paged_decode_append_attn(const jf_kv_pool* pool, const int32_t* page_tabl
  * num_splits > 1).  With a smaller workspace it runs as one launch.  Both
  * forms compute the same attention; the summation order, and so the last
  * bits, differ.
+ * Numerics (affine pools): each 64-position K/V tile is rebuilt in shared
+ * memory as fp16 code * scale + bias (one rounding) for the tensor cores, and
+ * q * softmax_scale * log2(e) enters as fp16; accumulation and the softmax
+ * run in fp32.  A K or V group whose reconstruction can leave the fp16 range
+ * (|bias| + 15 scale >= 65504, or a non-finite scale/bias word) sets
+ * JF_DEV_ERR_RANGE in the status word; outputs that attend such a group are
+ * then not reliable.
  * TQ4 pools (Sec. 3.1: page lookup, unpacking, centroid lookup, inverse
  * rotation and norm restoration fused into the attention's operand path):
  * the queries are rotated once (q' = H S_K q / sqrt(D), fp32 in the
@@ -367,6 +379,20 @@ int jf_kv_checkpoint(const jf_kv_pool* pool, const int32_t* page_table_row, int3
  */
 int jf_kv_restore(const jf_kv_pool* pool, const int32_t* page_table_row, int32_t num_pages,
                   const void* src, size_t src_bytes, int32_t* err_flag, void* stream);
+
+/*
+ * Self-test of the bounded-wait give-up path (no paper counterpart; failure
+ * detection).  Every wait of the library's kernels on a copy is bounded: it
+ * polls a fixed number of times, then the kernel ORs JF_DEV_ERR_TIMEOUT into
+ * its status word and returns, so a copy that never lands costs an error bit
+ * instead of a hung GPU.  This call runs that path alone in one thread: it
+ * waits on a shared-memory barrier that completes only if arrive != 0, so
+ * with arrive == 0 the wait runs out (after 4,096 polls) and JF_DEV_ERR_TIMEOUT
+ * is ORed into *status; with arrive != 0 *status is left unchanged.  No copy
+ * or other CTA is involved and the CUDA context stays usable.
+ *   status  device int32
+ */
+int jf_selftest_bounded_wait(int32_t* status, int32_t arrive, void* stream);
 
 /*
  * Decode attention without a caller-supplied workspace.  The paper has no

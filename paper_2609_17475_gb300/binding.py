@@ -25,6 +25,7 @@ JF_DEV_ERR_PAGE_ID = 1
 JF_DEV_ERR_POSITION = 2
 JF_DEV_ERR_TIMEOUT = 4
 JF_DEV_ERR_LAYOUT = 8
+JF_DEV_ERR_RANGE = 16
 JF_FMT_AFFINE4_G64 = 0
 JF_FMT_TQ4 = 1
 
@@ -35,6 +36,7 @@ EXPORTS = [
     "jf_paged_decode_attn_noalloc", "jf_paged_decode_append_attn", "jf_paged_verify_attn",
     "jf_kv_page_bytes_fmt", "jf_tq4_codebook", "jf_prefill_batch_attn", "jf_reservation_pages",
     "jf_prefill_batch_workspace_bytes", "jf_prefill_chunk_workspace_bytes",
+    "jf_selftest_bounded_wait",
 ]
 JF_STATIC_WORKSPACE_BYTES = 8 << 20
 
@@ -94,6 +96,7 @@ def lib() -> ctypes.CDLL:
             "jf_prefill_batch_workspace_bytes": (SZ, [I32, I64, I32, I32, I32]),
             "jf_prefill_chunk_workspace_bytes": (SZ, [PP, I32, I32, I32, I32]),
             "jf_reservation_pages": (I64, [I64, I64, I64, I32]),
+            "jf_selftest_bounded_wait": (ctypes.c_int, [P, I32, P]),
             "jf_status_string": (ctypes.c_char_p, [ctypes.c_int]),
             "jf_version": (ctypes.c_char_p, []),
         }
@@ -111,6 +114,28 @@ def status_string(status: int) -> str:
 
 def version() -> str:
     return lib().jf_version().decode()
+
+
+# NVTX ranges around every call that enqueues work (named after the C entry
+# point), for timelines in Nsight tools: enabled by JFKV_NVTX=1 in the
+# environment when this module is imported; otherwise the functions are left
+# unwrapped and cost nothing.
+NVTX = os.environ.get("JFKV_NVTX", "0") not in ("", "0")
+
+
+def _traced(fn):
+    if not NVTX:
+        return fn
+    import functools
+
+    @functools.wraps(fn)
+    def wrapper(*args, **kwargs):
+        torch.cuda.nvtx.range_push(fn.__name__)
+        try:
+            return fn(*args, **kwargs)
+        finally:
+            torch.cuda.nvtx.range_pop()
+    return wrapper
 
 
 def _check(fn: str, status: int) -> None:
@@ -246,6 +271,7 @@ def workspace_status(workspace: torch.Tensor) -> int:
     return int(workspace[:4].view(torch.int32).item())
 
 
+@_traced
 def jf_kv_quantize_append(pool: KVPool, page_table: torch.Tensor, row_req: torch.Tensor,
                           row_pos: torch.Tensor, k: torch.Tensor, v: torch.Tensor,
                           err_flag: Optional[torch.Tensor] = None, stream=None) -> None:
@@ -266,6 +292,7 @@ def jf_kv_quantize_append(pool: KVPool, page_table: torch.Tensor, row_req: torch
     _check("jf_kv_quantize_append", st)
 
 
+@_traced
 def jf_paged_decode_attn(pool: KVPool, page_table: torch.Tensor, context_lens: torch.Tensor,
                          q: torch.Tensor, softmax_scale: float, out: torch.Tensor,
                          workspace: torch.Tensor, num_splits: int, stream=None) -> None:
@@ -284,6 +311,7 @@ def jf_paged_decode_attn(pool: KVPool, page_table: torch.Tensor, context_lens: t
     _check("jf_paged_decode_attn", st)
 
 
+@_traced
 def jf_paged_decode_append_attn(pool: KVPool, page_table: torch.Tensor,
                                 context_lens: torch.Tensor, k_new: torch.Tensor,
                                 v_new: torch.Tensor, q: torch.Tensor, softmax_scale: float,
@@ -312,6 +340,7 @@ def jf_paged_decode_append_attn(pool: KVPool, page_table: torch.Tensor,
     _check("jf_paged_decode_append_attn", st)
 
 
+@_traced
 def jf_paged_verify_attn(pool: KVPool, page_table: torch.Tensor, context_lens: torch.Tensor,
                          q: torch.Tensor, softmax_scale: float, out: torch.Tensor,
                          workspace: torch.Tensor, num_splits: int, stream=None) -> None:
@@ -358,6 +387,7 @@ def default_verify_splits(batch: int, q_len: int, num_q_heads: int, num_kv_heads
     return max(1, per if batch == 1 else per + 2)
 
 
+@_traced
 def jf_paged_decode_attn_noalloc(pool: KVPool, page_table: torch.Tensor,
                                  context_lens: torch.Tensor, q: torch.Tensor, softmax_scale: float,
                                  out: torch.Tensor, num_splits: int,
@@ -383,6 +413,7 @@ def jf_paged_decode_attn_noalloc(pool: KVPool, page_table: torch.Tensor,
     _check("jf_paged_decode_attn_noalloc", st)
 
 
+@_traced
 def jf_prefill_chunk_attn(pool: KVPool, page_table_row: torch.Tensor, q: torch.Tensor,
                           q_start: int, softmax_scale: float, causal: bool, out: torch.Tensor,
                           workspace: torch.Tensor, stream=None) -> None:
@@ -470,6 +501,7 @@ def default_prefill_splits(q_start, chunk_len, num_q_heads: int, num_kv_heads: i
     return next(S for S, t in scores if t <= 1.02 * best_t)
 
 
+@_traced
 def jf_prefill_batch_attn(pool: KVPool, page_table: torch.Tensor, q_start, chunk_len,
                           q: torch.Tensor, softmax_scale: float, causal: bool, out: torch.Tensor,
                           workspace: torch.Tensor, num_splits: int = 1, stream=None) -> None:
@@ -508,6 +540,15 @@ def jf_reservation_pages(prompt_len: int, output_len: int, g_out: int = 8192,
     return r
 
 
+def jf_selftest_bounded_wait(status: torch.Tensor, arrive: bool, stream=None) -> None:
+    """Run the bounded-wait give-up path alone (include/jfkv.h): with
+    arrive=False the wait runs out and JF_DEV_ERR_TIMEOUT is ORed into status."""
+    _need(status, torch.int32, "status")
+    _check("jf_selftest_bounded_wait",
+           lib().jf_selftest_bounded_wait(_ptr(status), 1 if arrive else 0, _stream(stream)))
+
+
+@_traced
 def jf_kv_checkpoint(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
                      dst: torch.Tensor, err_flag: Optional[torch.Tensor] = None,
                      stream=None) -> None:
@@ -521,6 +562,7 @@ def jf_kv_checkpoint(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
     _check("jf_kv_checkpoint", st)
 
 
+@_traced
 def jf_kv_restore(pool: KVPool, page_table_row: torch.Tensor, num_pages: int,
                   src: torch.Tensor, err_flag: Optional[torch.Tensor] = None,
                   stream=None) -> None:

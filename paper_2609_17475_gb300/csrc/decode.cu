@@ -44,7 +44,8 @@
 
 namespace jfkv {
 
-constexpr int DWARPS = 6;     // warps per split CTA (2 CTAs per SM)
+// Warps per split CTA (NW, a template parameter): 6 (two CTAs per SM) or 12
+// (one CTA per SM, the same warps per SM in one block).
 constexpr int DSTAGES = 2;    // stages per warp
 
 // (w >> 8) as an integer multiply-high, which runs on the FMA pipe and spares
@@ -85,14 +86,14 @@ __device__ __forceinline__ uint32_t hi_halves(uint32_t a, uint32_t b) {
   return __byte_perm(a, b, 0x7632);
 }
 
-template <int D>
+template <int D, int NW>
 struct DecodeSmem {
   static constexpr int CB = D / 2;
   static constexpr int NG = D / 64;
   static constexpr int SBB = 4 * NG;
   static constexpr int CODE_BUF = DTOK * CB;
   static constexpr int SB_BUF = DTOK * SBB;
-  static constexpr int NBUF = DWARPS * DSTAGES;
+  static constexpr int NBUF = NW * DSTAGES;
   static constexpr int CODES_BYTES = NBUF * 2 * CODE_BUF;
   static constexpr int SB_BYTES = NBUF * 2 * SB_BUF;
   static constexpr int QF_BYTES = NG * 2 * 32 * 16;   // query fragments [g][half][lane][4]
@@ -102,8 +103,9 @@ struct DecodeSmem {
   static constexpr int PLAN_BYTES = 16;                // batch plan broadcast
   static constexpr int TOTAL = CODES_BYTES + SB_BYTES + QF_BYTES + BAR_BYTES + PLAN_BYTES;
   static constexpr uint32_t STAGE_TX = 2 * CODE_BUF + 2 * SB_BUF;
-  static_assert(DWARPS * 8 * (D + 4) * 4 <= CODES_BYTES, "combine buffer must fit");
-  static_assert((DWARPS * 8 * 3 + 16) * 4 <= SB_BYTES, "combine (m, l), weights must fit");
+  static_assert(NW * 8 * (D + 4) * 4 <= CODES_BYTES, "combine buffer must fit");
+  static_assert((NW * 8 * 3 + 16) * 4 <= SB_BYTES, "combine (m, l), weights must fit");
+  static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
 
 // Per-warp online-softmax state.  Thread (r, c) of the warp owns query heads
@@ -357,11 +359,11 @@ __device__ __forceinline__ void append_new_row(const DecodeArgs& a, int b, int k
                      bh);
 }
 
-template <int D, bool VER>
-__global__ void __launch_bounds__(DWARPS * 32, 2)
+template <int D, bool VER, int NW>
+__global__ void __launch_bounds__(NW * 32, 12 / NW)
 decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
   // VER: packed verifier (a.L > 1, per-row causal limits); otherwise decode
-  using L = DecodeSmem<D>;
+  using L = DecodeSmem<D, NW>;
   constexpr int NG = L::NG;
   constexpr int SBB = L::SBB;
   constexpr float NEG_INF = -INFINITY;
@@ -389,7 +391,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   };
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;
-  const bool direct = (a.num_splits == 1);
+  const bool direct = (a.plan_splits == 1 && !a.balanced);
   int* plan_sh = reinterpret_cast<int*>(sbuf + L::SB_BYTES + L::QF_BYTES + L::BAR_BYTES);
   // the swizzled TMA boxes need a 1024-byte aligned window
   const bool aligned = (smem_u32(smem_raw) & 1023) == 0;
@@ -427,7 +429,7 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     split = blockIdx.x;
     b = blockIdx.z;
     ctx = checked_ctx(a, b, split);
-    split_plan(ctx, a.num_splits, nch, cps, nsplit);
+    split_plan(ctx, a.plan_splits, nch, cps, nsplit);
   }
   if (split >= nsplit) {
     if (direct && split == 0) {   // empty context: zero output
@@ -439,8 +441,8 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   const int c_begin = split * cps;
   const int c_end = min(c_begin + cps, nch);
   const int n_cta = c_end - c_begin;
-  const int my_n = (n_cta > warp) ? (n_cta - warp + DWARPS - 1) / DWARPS : 0;
-  auto chunk_of = [&](int it) { return c_begin + warp + it * DWARPS; };
+  const int my_n = (n_cta > warp) ? (n_cta - warp + NW - 1) / NW : 0;
+  auto chunk_of = [&](int it) { return c_begin + warp + it * NW; };
 
   if (!aligned) {
     if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_LAYOUT);
@@ -546,6 +548,9 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   int pg_next = load_pages(1);
 
   // ---- TMA producer (lane 0 of each warp feeds its own ring) -------------
+  // decode reads each page once per call: evict it from L2 first; the
+  // verifier's n-tile CTAs read the same pages, so L2 keeps them normally
+  const uint64_t l2pol = VER ? l2_evict_normal_policy() : l2_evict_first_policy();
   uint32_t valid = 0;
   auto issue = [&](int it) {
     const int s = it % DSTAGES;
@@ -567,10 +572,10 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
         const uint8_t* gsb = a.pool + (int64_t)page * a.page_bytes + a.sb_base +
                              ((int64_t)kvh * a.P + inp) * SBB;
         mbar_arrive_expect_tx(bar, L::STAGE_TX);
-        tma_load_5d(kc, &tmap, 0, inp, kvh, 0, page, bar);
-        tma_load_5d(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar);
-        bulk_g2s(ks, gsb, L::SB_BUF, bar);
-        bulk_g2s(ks + L::SB_BUF, gsb + a.sb_region, L::SB_BUF, bar);
+        tma_load_5d_hint(kc, &tmap, 0, inp, kvh, 0, page, bar, l2pol);
+        tma_load_5d_hint(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar, l2pol);
+        bulk_g2s_hint(ks, gsb, L::SB_BUF, bar, l2pol);
+        bulk_g2s_hint(ks + L::SB_BUF, gsb + a.sb_region, L::SB_BUF, bar, l2pol);
       }
     }
     valid = (valid & ~(1u << s)) | ((uint32_t)ok << s);
@@ -664,76 +669,78 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     Bs[g][0] = __shfl_sync(0xffffffffu, st.Bs[0], g * 4 + c);
     Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
   }
-  __syncthreads();   // every warp is past its last stage: reuse the rings
-  // Each warp's O (rows padded by 4 floats: the 128-bit stores of one
-  // quarter-warp hit 8 distinct bank groups) and (m, l) per head.
+  // This warp's ring is idle now (each of its copies has landed and been
+  // read), so its O rows (padded by 4 floats: the 128-bit stores of one
+  // quarter-warp hit 8 distinct bank groups) and (m, l) per head go into its
+  // own stage buffers at once, without waiting for the other warps.
   constexpr int SROW = D + 4;
-  float* so = reinterpret_cast<float*>(codes);    // [DWARPS][8][SROW]
-  float* sml = reinterpret_cast<float*>(sbuf);    // [DWARPS][8][2]
-  float* swt = sml + DWARPS * 8 * 2;              // [DWARPS][8] combine weights
-  float* shl = swt + DWARPS * 8;                  // [8][2] (M, L) per head
+  constexpr int WCODES = DSTAGES * 2 * L::CODE_BUF;   // one warp's code ring (bytes)
+  constexpr int WSB = DSTAGES * 2 * L::SB_BUF;        // one warp's scale/bias ring
+  static_assert(8 * SROW * 4 <= WCODES && 8 * 2 * 4 <= WSB, "combine rows fit a warp's ring");
   {
+    float* so = reinterpret_cast<float*>(codes + warp * WCODES);   // [8][SROW]
+    float* sml = reinterpret_cast<float*>(sbuf + warp * WSB);      // [8][2]
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf) {          // d block 64g + 32 hf + 4r + e
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {        // head 2c + hh
-          float4 v;
-          // 2^24 undoes the fp16 subnormal codes (2^20 for the hi nibbles)
-          v.x = fmaf(O[g][0][2 * hf + hh], 16777216.f, Bs[g][hh]);
-          v.y = fmaf(O[g][1][2 * hf + hh], 1048576.f, Bs[g][hh]);
-          v.z = fmaf(O[g][2][2 * hf + hh], 16777216.f, Bs[g][hh]);
-          v.w = fmaf(O[g][3][2 * hf + hh], 1048576.f, Bs[g][hh]);
-          *reinterpret_cast<float4*>(so + (warp * 8 + 2 * c + hh) * SROW + 64 * g + 32 * hf +
-                                     4 * r) = v;
+          if (2 * c + hh < rows) {
+            float4 v;
+            // 2^24 undoes the fp16 subnormal codes (2^20 for the hi nibbles)
+            v.x = fmaf(O[g][0][2 * hf + hh], 16777216.f, Bs[g][hh]);
+            v.y = fmaf(O[g][1][2 * hf + hh], 1048576.f, Bs[g][hh]);
+            v.z = fmaf(O[g][2][2 * hf + hh], 16777216.f, Bs[g][hh]);
+            v.w = fmaf(O[g][3][2 * hf + hh], 1048576.f, Bs[g][hh]);
+            *reinterpret_cast<float4*>(so + (2 * c + hh) * SROW + 64 * g + 32 * hf + 4 * r) = v;
+          }
         }
       }
     }
     if (r == 0) {
-      sml[(warp * 8 + 2 * c) * 2 + 0] = m0;
-      sml[(warp * 8 + 2 * c) * 2 + 1] = l0;
-      sml[(warp * 8 + 2 * c + 1) * 2 + 0] = m1;
-      sml[(warp * 8 + 2 * c + 1) * 2 + 1] = l1;
+      sml[(2 * c) * 2 + 0] = m0;
+      sml[(2 * c) * 2 + 1] = l0;
+      sml[(2 * c + 1) * 2 + 0] = m1;
+      sml[(2 * c + 1) * 2 + 1] = l1;
     }
   }
   __syncthreads();
 
   // ---- combine the warps of this CTA --------------------------------------
   // per head: M = max_w m_w, weights 2^(m_w - M) (divided by L when this CTA
-  // writes the final output), L = sum_w 2^(m_w - M) l_w
-  if (threadIdx.x < rows) {
-    const int h = threadIdx.x;
-    float M = NEG_INF;
-#pragma unroll
-    for (int w = 0; w < DWARPS; ++w) M = fmaxf(M, sml[(w * 8 + h) * 2]);
-    float f[DWARPS];
-    float L = 0.f;
-#pragma unroll
-    for (int w = 0; w < DWARPS; ++w) {
-      const float mw = sml[(w * 8 + h) * 2];
-      f[w] = (mw != NEG_INF) ? fast_exp2(mw - M) : 0.f;
-      L = fmaf(f[w], sml[(w * 8 + h) * 2 + 1], L);
-    }
-    const float inv = direct ? (L > 0.f ? 1.f / L : 0.f) : 1.f;
-#pragma unroll
-    for (int w = 0; w < DWARPS; ++w) swt[w * 8 + h] = f[w] * inv;
-    shl[h * 2 + 0] = M;
-    shl[h * 2 + 1] = L;
-  }
-  __syncthreads();
+  // writes the final output), L = sum_w 2^(m_w - M) l_w; every thread works
+  // out the weights of its own head.
   for (int idx = threadIdx.x; idx < rows * (D / 4); idx += blockDim.x) {
     const int h = idx / (D / 4), d = 4 * (idx % (D / 4));
+    float mw[NW], lw[NW];
+    float M = NEG_INF;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {
+      const float2 v = *reinterpret_cast<const float2*>(sbuf + w * WSB + h * 8);
+      mw[w] = v.x;
+      lw[w] = v.y;
+      M = fmaxf(M, v.x);
+    }
+    float f[NW];
+    float Lsum = 0.f;
+#pragma unroll
+    for (int w = 0; w < NW; ++w) {
+      f[w] = (mw[w] != NEG_INF) ? fast_exp2(mw[w] - M) : 0.f;
+      Lsum = fmaf(f[w], lw[w], Lsum);
+    }
+    const float inv = direct ? (Lsum > 0.f ? 1.f / Lsum : 0.f) : 1.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int w = 0; w < DWARPS; ++w) {
-      const float f = swt[w * 8 + h];
-      const float4 v = *reinterpret_cast<const float4*>(so + (w * 8 + h) * SROW + d);
-      if (f != 0.f) {
-        acc.x = fmaf(f, v.x, acc.x);
-        acc.y = fmaf(f, v.y, acc.y);
-        acc.z = fmaf(f, v.z, acc.z);
-        acc.w = fmaf(f, v.w, acc.w);
+    for (int w = 0; w < NW; ++w) {
+      const float fw = f[w] * inv;
+      const float4 v = *reinterpret_cast<const float4*>(
+          reinterpret_cast<const float*>(codes + w * WCODES) + h * SROW + d);
+      if (fw != 0.f) {
+        acc.x = fmaf(fw, v.x, acc.x);
+        acc.y = fmaf(fw, v.y, acc.y);
+        acc.z = fmaf(fw, v.z, acc.z);
+        acc.w = fmaf(fw, v.w, acc.w);
       }
     }
     const int fr = row_of(h);
@@ -752,29 +759,30 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
           : ((int64_t)blockIdx.z * a.HqL + fr) * a.num_splits + blockIdx.x;
       *reinterpret_cast<float4*>(a.part_o + row * D + d) = acc;
       if (d == 0) {
-        a.part_ml[row * 2 + 0] = shl[h * 2 + 0];
-        a.part_ml[row * 2 + 1] = shl[h * 2 + 1];
+        a.part_ml[row * 2 + 0] = M;
+        a.part_ml[row * 2 + 1] = Lsum;
       }
     }
   }
 }
 
 
-// One CTA per (32-wide slice of head_dim, query head, request); its 8 warps
-// take interleaved splits and reduce through shared memory, so the merge is
-// spread over the whole GPU.  The kernel is a chain of dependent loads, so it
-// issues them all at once: the context length, every (m, l) row and this
-// thread's partial outputs for up to MERGE_BATCH splits are loaded before any
-// is used; rows past the split plan are loaded (the workspace holds
-// num_splits rows) and then ignored.
+// Merge for one or a few requests: one CTA per (32-wide slice of head_dim,
+// query row, request); its 8 warps take interleaved splits and reduce through
+// shared memory, so even one request's merge is spread over the whole GPU.
+// The kernel is a chain of dependent loads, so it issues them all at once:
+// the context length, every (m, l) row and this thread's partial outputs for
+// up to MERGE_SG_BATCH splits are loaded before any is used; rows past the
+// split plan are loaded (the workspace holds num_splits rows) and then
+// ignored.
 constexpr int MERGE_THREADS = 256;
 constexpr int MERGE_DSLICE = 32;
 constexpr int MERGE_NSG = MERGE_THREADS / MERGE_DSLICE;   // split groups
-constexpr int MERGE_BATCH = 16;                           // splits per thread per batch
-constexpr int MERGE_MLB = MERGE_BATCH * MERGE_NSG / 32;   // (m, l) rows per lane per batch
+constexpr int MERGE_SG_BATCH = 16;                        // splits per thread per batch
+constexpr int MERGE_MLB = MERGE_SG_BATCH * MERGE_NSG / 32;   // (m, l) rows per lane per batch
 
 template <int D>
-__global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const DecodeArgs a) {
+__global__ void __launch_bounds__(MERGE_THREADS) decode_merge_sg_kernel(const DecodeArgs a) {
   __shared__ float red[MERGE_NSG][MERGE_DSLICE];
   // the next kernel in the stream may be scheduled now; it waits for this
   // grid to complete before it reads anything
@@ -785,12 +793,13 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   const int t = threadIdx.x, dd = t % MERGE_DSLICE, sg = t / MERGE_DSLICE;
   const int lane = t & 31;
   // partials of split s: row row0 + s * rs.  Per-request plans put them at
-  // ((b Hq + hq) S + s) and are known only after the context is read, so all
-  // S rows are loaded speculatively; the batch plan numbers splits globally
-  // (row (g0 + s) Hq + hq) and is worked out first.
+  // ((b Hq + hq) num_splits + s) and are known only after the context is
+  // read, so the plan's plan_splits rows are loaded speculatively; the batch
+  // plan numbers splits globally (row (g0 + s) Hq + hq) and is worked out
+  // first.
   __shared__ int plan_sh[2];
-  int S = a.num_splits;
-  int64_t row0 = ((int64_t)b * a.HqL + hq) * S;
+  int S = a.plan_splits;
+  int64_t row0 = ((int64_t)b * a.HqL + hq) * a.num_splits;
   int64_t rs = 1;
   int nsplit_bal = 0;
   if (a.balanced) {
@@ -812,14 +821,14 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 
   const int ctx_raw = a.ctx[b];
   float2 mlv[MERGE_MLB];
-  float ov[MERGE_BATCH], mv[MERGE_BATCH];
+  float ov[MERGE_SG_BATCH], mv[MERGE_SG_BATCH];
 #pragma unroll
   for (int k = 0; k < MERGE_MLB; ++k) {
     const int s = lane + 32 * k;
     mlv[k] = (s < S) ? ml[s * rs] : make_float2(-INFINITY, 0.f);
   }
 #pragma unroll
-  for (int u = 0; u < MERGE_BATCH; ++u) {
+  for (int u = 0; u < MERGE_SG_BATCH; ++u) {
     const int s = sg + MERGE_NSG * u;
     ov[u] = (s < S) ? po[s * rs * D] : 0.f;
     mv[u] = (s < S) ? ml[s * rs].x : -INFINITY;
@@ -831,7 +840,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
   if (ctx < 0) ctx = 0;
   if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
-  split_plan(ctx, a.num_splits, nch, cps, nsplit);
+  split_plan(ctx, a.plan_splits, nch, cps, nsplit);
   if (a.balanced) nsplit = nsplit_bal;
   uint16_t* orow = a.out + ((int64_t)b * a.HqL + hq) * D + d0;
   if (nsplit == 0) {
@@ -861,19 +870,19 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
 #pragma unroll
-    for (int u = 0; u < MERGE_BATCH; ++u)
+    for (int u = 0; u < MERGE_SG_BATCH; ++u)
       if (sg + MERGE_NSG * u < nsplit && mv[u] != -INFINITY)
         acc = fmaf(fast_exp2(mv[u] - M), ov[u], acc);
     // more splits than one batch covers
-    for (int s0 = sg + MERGE_NSG * MERGE_BATCH; s0 < nsplit; s0 += MERGE_NSG * MERGE_BATCH) {
+    for (int s0 = sg + MERGE_NSG * MERGE_SG_BATCH; s0 < nsplit; s0 += MERGE_NSG * MERGE_SG_BATCH) {
 #pragma unroll
-      for (int u = 0; u < MERGE_BATCH; ++u) {
+      for (int u = 0; u < MERGE_SG_BATCH; ++u) {
         const int s = s0 + MERGE_NSG * u;
         ov[u] = (s < nsplit) ? po[s * rs * D] : 0.f;
         mv[u] = (s < nsplit) ? ml[s * rs].x : -INFINITY;
       }
 #pragma unroll
-      for (int u = 0; u < MERGE_BATCH; ++u)
+      for (int u = 0; u < MERGE_SG_BATCH; ++u)
         if (mv[u] != -INFINITY) acc = fmaf(fast_exp2(mv[u] - M), ov[u], acc);
     }
   }
@@ -885,6 +894,106 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_kernel(const Decod
     for (int k = 0; k < MERGE_NSG; ++k) o += red[k][t];
     orow[t] = __bfloat16_as_ushort(__float2bfloat16_rn(L > 0.f ? o / L : 0.f));
   }
+}
+
+// Merge for batches (one CTA per query row and request).  D / 2 threads,
+// each owning two adjacent columns of the output row.  Every warp works out the row's
+// reference maximum M itself from the splits' (m, l) pairs (lane j holds
+// splits j and j + 32 of a batch), and each thread sums its two columns over
+// the splits in split order, the weights 2^(m_s - M) passed along by
+// shuffles:
+//   o = sum_s 2^{m_s - M} O_s / sum_s 2^{m_s - M} l_s.
+// A batch's loads are all issued before any is used.  Per-request plans are
+// known only once the context length is read, so the first batch of their
+// rows is loaded speculatively and rows past the plan are ignored (whatever
+// the workspace holds there).
+constexpr int MERGE_BATCH = 64;   // splits per batch: two per lane for the weights
+
+template <int D>
+__global__ void __launch_bounds__(D / 2) decode_merge_kernel(const DecodeArgs a) {
+  // the next kernel in the stream may be scheduled now; it waits for this
+  // grid to complete before it reads anything
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  // the split kernel's partials must be complete and visible
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  const int hq = blockIdx.x, b = blockIdx.y;
+  const int t = threadIdx.x, lane = t & 31;
+  int64_t row0, rs;   // partials of split s: row row0 + s * rs
+  int S, nsplit_bal = 0;
+  if (a.balanced) {   // every warp works the plan out itself
+    const BalPlan p = balanced_plan(a, -1, b, lane);
+    row0 = (int64_t)p.g0 * a.HqL + hq;
+    rs = a.HqL;
+    nsplit_bal = p.nsplit;
+    S = p.nsplit;
+  } else {
+    row0 = ((int64_t)b * a.HqL + hq) * a.num_splits;
+    rs = 1;
+    S = a.plan_splits;
+  }
+  const float2* ml = reinterpret_cast<const float2*>(a.part_ml) + row0;
+  const float2* po = reinterpret_cast<const float2*>(a.part_o + row0 * D) + t;
+  const int64_t ostride = rs * (D / 2);   // float2 elements between split rows
+
+  const int ctx_raw = a.ctx[b];
+  float2 ml0 = (lane < S) ? ml[lane * rs] : make_float2(-INFINITY, 0.f);
+  float2 ml1 = (lane + 32 < S) ? ml[(lane + 32) * rs] : make_float2(-INFINITY, 0.f);
+  float2 ov[MERGE_BATCH];
+#pragma unroll
+  for (int j = 0; j < MERGE_BATCH; ++j)
+    ov[j] = (j < S) ? po[j * ostride] : make_float2(0.f, 0.f);
+
+  int ctx = ctx_raw;
+  const int64_t cap = (int64_t)a.pt_stride * a.P;
+  if ((ctx < 0 || ctx > cap) && t == 0 && hq == 0)
+    flag_error(a.status, JF_DEV_ERR_POSITION);   // also covers requests with no split
+  if (ctx < 0) ctx = 0;
+  if (ctx > cap) ctx = (int)cap;
+  int nch, cps, nsplit;
+  split_plan(ctx, a.plan_splits, nch, cps, nsplit);
+  if (a.balanced) nsplit = nsplit_bal;
+  uint32_t* orow = reinterpret_cast<uint32_t*>(a.out + ((int64_t)b * a.HqL + hq) * D) + t;
+  if (nsplit == 0) {
+    *orow = 0u;
+    return;
+  }
+
+  // reference maximum over every split (each warp on its own)
+  float M = fmaxf(lane < nsplit ? ml0.x : -INFINITY, lane + 32 < nsplit ? ml1.x : -INFINITY);
+  for (int s = lane + MERGE_BATCH; s < nsplit; s += 32) M = fmaxf(M, ml[s * rs].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+
+  float L = 0.f;
+  float2 acc = make_float2(0.f, 0.f);
+  for (int s0 = 0; s0 < nsplit; s0 += MERGE_BATCH) {
+    if (s0 > 0) {   // the next batch (more splits than one batch covers)
+      ml0 = (s0 + lane < nsplit) ? ml[(s0 + lane) * rs] : make_float2(-INFINITY, 0.f);
+      ml1 = (s0 + lane + 32 < nsplit) ? ml[(s0 + lane + 32) * rs]
+                                      : make_float2(-INFINITY, 0.f);
+#pragma unroll
+      for (int j = 0; j < MERGE_BATCH; ++j)
+        ov[j] = (s0 + j < nsplit) ? po[(s0 + j) * ostride] : make_float2(0.f, 0.f);
+    }
+    const float w0 = (s0 + lane < nsplit && ml0.x != -INFINITY) ? fast_exp2(ml0.x - M) : 0.f;
+    const float w1 =
+        (s0 + lane + 32 < nsplit && ml1.x != -INFINITY) ? fast_exp2(ml1.x - M) : 0.f;
+    if (w0 != 0.f) L = fmaf(w0, ml0.y, L);   // rows past the plan hold anything
+    if (w1 != 0.f) L = fmaf(w1, ml1.y, L);
+#pragma unroll
+    for (int j = 0; j < MERGE_BATCH; ++j) {
+      const float w = __shfl_sync(0xffffffffu, j < 32 ? w0 : w1, j & 31);
+      if (s0 + j < nsplit && w != 0.f) {
+        acc.x = fmaf(w, ov[j].x, acc.x);
+        acc.y = fmaf(w, ov[j].y, acc.y);
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  *orow = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.x * inv)) |
+          ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.y * inv)) << 16);
 }
 
 // ---------------------------------------------------------------------------
@@ -930,30 +1039,39 @@ size_t decode_workspace_bytes(int64_t B, int64_t Hq, int64_t D, int64_t S) {
   return (size_t)(256 + ml + rows * D * 4);
 }
 
-// Merge phase: one CTA per (32-wide slice of head_dim, row, request), launched
-// with programmatic dependent launch after the split kernel.
+// Merge phase, launched with programmatic dependent launch after the split
+// kernel.
 int launch_decode_merge(const DecodeArgs& a, int D, int B, cudaStream_t stream) {
   cudaLaunchAttribute pdl[1];
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t mc = {};
-  mc.gridDim = dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.HqL, (unsigned)B);
-  mc.blockDim = dim3(MERGE_THREADS);
+  // a few rows: 32-column slices with 8 split groups each (more CTAs, fewer
+  // loads per thread); a batch: one CTA per row
+  const bool sg = (int64_t)B * a.HqL * (D / MERGE_DSLICE) <= 4 * (int64_t)sm_count();
+  mc.gridDim = sg ? dim3((unsigned)(D / MERGE_DSLICE), (unsigned)a.HqL, (unsigned)B)
+                  : dim3((unsigned)a.HqL, (unsigned)B, 1u);
+  mc.blockDim = dim3(sg ? (unsigned)MERGE_THREADS : (unsigned)(D / 2));
   mc.dynamicSmemBytes = 0;
   mc.stream = stream;
   mc.attrs = pdl;
   mc.numAttrs = 1;
-  const cudaError_t e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256>, a)
-                                   : cudaLaunchKernelEx(&mc, decode_merge_kernel<128>, a);
+  cudaError_t e;
+  if (sg)
+    e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<256>, a)
+                   : cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<128>, a);
+  else
+    e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256>, a)
+                   : cudaLaunchKernelEx(&mc, decode_merge_kernel<128>, a);
   return e == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }
 
-template <int D>
+template <int D, int NW>
 static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
                            cudaStream_t stream) {
-  using L = DecodeSmem<D>;
-  if (smem_optin((const void*)decode_split_kernel<D, false>, L::TOTAL) != JF_OK ||
-      smem_optin((const void*)decode_split_kernel<D, true>, L::TOTAL) != JF_OK)
+  using L = DecodeSmem<D, NW>;
+  if (smem_optin((const void*)decode_split_kernel<D, false, NW>, L::TOTAL) != JF_OK ||
+      smem_optin((const void*)decode_split_kernel<D, true, NW>, L::TOTAL) != JF_OK)
     return JF_ERR_CUDA;
   // Both kernels use programmatic dependent launch: each may be scheduled
   // while the previous kernel in the stream drains, and waits (griddepcontrol)
@@ -963,19 +1081,39 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
   // batch plan: a.budget + B CTAs per KV head cover every split (sum_b n_b <=
-  // T / cps + B <= budget + B); per-request plans: num_splits per request
+  // T / cps + B <= budget + B); per-request plans: plan_splits per request
   cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)(a.Hkv * a.NT), 1u)
-                           : dim3((unsigned)a.num_splits, (unsigned)(a.Hkv * a.NT), (unsigned)B);
-  cfg.blockDim = dim3(DWARPS * 32);
+                           : dim3((unsigned)a.plan_splits, (unsigned)(a.Hkv * a.NT), (unsigned)B);
+  cfg.blockDim = dim3(NW * 32);
   cfg.dynamicSmemBytes = L::TOTAL;
   cfg.stream = stream;
   cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  const cudaError_t e = (a.L > 1) ? cudaLaunchKernelEx(&cfg, decode_split_kernel<D, true>, tmap, a)
-                                  : cudaLaunchKernelEx(&cfg, decode_split_kernel<D, false>, tmap, a);
+  const cudaError_t e =
+      (a.L > 1) ? cudaLaunchKernelEx(&cfg, decode_split_kernel<D, true, NW>, tmap, a)
+                : cudaLaunchKernelEx(&cfg, decode_split_kernel<D, false, NW>, tmap, a);
   if (e != cudaSuccess) return JF_ERR_CUDA;
-  if (a.num_splits > 1) return launch_decode_merge(a, D, B, stream);
+  if (a.balanced || a.plan_splits > 1) return launch_decode_merge(a, D, B, stream);
   return JF_OK;
+}
+
+// Warps per split CTA for a call (the NW template parameter).  Two 6-warp
+// CTAs on one SM do not share it evenly: the CTA placed first keeps issue
+// priority and ends its share ~4 us (of ~50) before the other, so one request
+// (and a batch whose workspace has fewer partial rows than the 6-warp grid
+// has CTA slots) runs one 12-warp CTA per SM.  A batch with rows to spare
+// keeps the 6-warp CTAs: their pieces are half as long, so cutting unequal
+// requests into pieces leaves less unevenness.
+static int decode_warps(int batch, int num_splits, int Hkv, int NT) {
+  if (NT > 1) return 6;   // packed verifier: measured slower with 12-warp CTAs
+  const int64_t sms = sm_count();
+  if (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) {   // batch split plan
+    const int64_t slots6 = (2 * sms + Hkv * NT - 1) / (Hkv * NT);
+    const int64_t fit = (int64_t)batch * num_splits - batch;
+    return fit < slots6 ? 12 : 6;
+  }
+  // per-request plans: one 12-warp CTA per SM while they fit in one wave
+  return (batch == 1 || (int64_t)batch * Hkv * NT * num_splits <= sms) ? 12 : 6;
 }
 
 int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
@@ -1013,19 +1151,26 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   a.num_splits = num_splits;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.B = batch;
+  const int nw = decode_warps(batch, num_splits, g.Hkv, a.NT);
+  const int per_sm = 12 / nw;   // split CTAs resident per SM
+  const int slots = (per_sm * sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
+  // per-request plans: one CTA wave (12-warp CTAs) or the caller's cap
+  a.plan_splits = (nw == 12 && num_splits > slots) ? slots : num_splits;
   // Batches of up to BAL_MAX_B requests size their splits for the whole batch
-  // (balanced_plan): about 2 CTAs per SM in all, fewer than B * num_splits
+  // (balanced_plan): one CTA per slot in all, fewer than B * num_splits
   // (minus B/2 for rounding) so every split's partial row fits the workspace.
   a.balanced = (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) ? 1 : 0;
   a.budget = 1;
   if (a.balanced) {
-    const int slots = (2 * sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
     const int64_t fit = (int64_t)batch * num_splits - batch;
     const int64_t cap = fit < slots ? fit : slots;
     a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);
   }
-  if (g.D == 256) return launch_decode_t<256>(tmap, a, batch, stream);
-  return launch_decode_t<128>(tmap, a, batch, stream);
+  if (nw == 12)
+    return g.D == 256 ? launch_decode_t<256, 12>(tmap, a, batch, stream)
+                      : launch_decode_t<128, 12>(tmap, a, batch, stream);
+  return g.D == 256 ? launch_decode_t<256, 6>(tmap, a, batch, stream)
+                    : launch_decode_t<128, 6>(tmap, a, batch, stream);
 }
 
 }  // namespace jfkv

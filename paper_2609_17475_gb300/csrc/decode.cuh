@@ -30,7 +30,8 @@ struct DecodeArgs {
   float* part_ml;      // [B, Hq, S, 2]
   float* part_o;       // [B, Hq, S, D]
   int32_t* status;
-  int32_t num_splits;
+  int32_t num_splits;   // workspace rows per (request, query row): the row stride
+  int32_t plan_splits;  // per-request plans cut a request into at most this many splits
   float scale_log2;    // softmax_scale * log2(e)
   int32_t B;           // requests
   int32_t L;           // query tokens per request (1: decode; 2-4: packed verifier)

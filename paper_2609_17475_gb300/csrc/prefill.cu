@@ -449,6 +449,10 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
       } else {
         uint32_t s2, b2;
         sb_to_h2(x.sbw, s2, b2);
+        // K and V are rebuilt in fp16: a group whose values can leave its
+        // range (|bias| + 15 scale >= 65504, or a non-finite word) is reported
+        if (x.valid && !(fabsf(bf16hi_to_f32(x.sbw)) + 15.f * bf16lo_to_f32(x.sbw) < 65504.f))
+          flag_error(a.status, JF_DEV_ERR_RANGE);
 #pragma unroll
         for (int u = 0; u < UPI; ++u) {
           const uint32_t cw[4] = {x.c[u].x, x.c[u].y, x.c[u].z, x.c[u].w};

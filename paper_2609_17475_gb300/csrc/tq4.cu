@@ -750,6 +750,9 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
   };
   int pg_cur = load_pages(0);
   int pg_next = load_pages(1);
+  // decode reads each page once per call: evict it from L2 first; the
+  // verifier's n-tile CTAs read the same pages, so L2 keeps them normally
+  const uint64_t l2pol = VER ? l2_evict_normal_policy() : l2_evict_first_policy();
   uint32_t valid = 0;
   auto issue = [&](int it) {
     const int s = it % TQ_STAGES;
@@ -771,10 +774,10 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
         const uint8_t* gn = a.pool + (int64_t)page * a.page_bytes + a.sb_base +
                             ((int64_t)kvh * a.P + inp) * 2;
         mbar_arrive_expect_tx(bar, L::STAGE_TX);
-        tma_load_5d(kc, &tmap, 0, inp, kvh, 0, page, bar);
-        tma_load_5d(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar);
-        bulk_g2s(kn, gn, L::NORM_BUF, bar);
-        bulk_g2s(kn + L::NORM_BUF, gn + a.sb_region, L::NORM_BUF, bar);
+        tma_load_5d_hint(kc, &tmap, 0, inp, kvh, 0, page, bar, l2pol);
+        tma_load_5d_hint(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar, l2pol);
+        bulk_g2s_hint(kn, gn, L::NORM_BUF, bar, l2pol);
+        bulk_g2s_hint(kn + L::NORM_BUF, gn + a.sb_region, L::NORM_BUF, bar, l2pol);
       }
     }
     valid = (valid & ~(1u << s)) | ((uint32_t)ok << s);
@@ -984,6 +987,7 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   a.part_ml = reinterpret_cast<float*>(ws + 256);
   a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
   a.num_splits = num_splits;
+  a.plan_splits = num_splits;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.B = batch;
   a.balanced = (batch > 1 && batch <= 1024 && num_splits > 1) ? 1 : 0;

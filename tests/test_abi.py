@@ -241,3 +241,24 @@ def test_split_planners_on_a_152_sm_gpu():
     assert ps([4096 * (b + 1) - 64 for b in range(8)], [64] * 8) == 2
     assert ps([4096 * (b + 1) - 512 for b in range(8)], [512] * 8) == 1
     assert ps([0], [0]) == 1               # nothing to schedule
+
+
+def test_nvtx_ranges_wrap_every_enqueueing_call_when_enabled():
+    """JFKV_NVTX=1 wraps each call that enqueues work in an NVTX range named
+    after its C entry point; unset, the functions stay unwrapped."""
+    import subprocess
+    import sys
+    names = ["jf_kv_quantize_append", "jf_paged_decode_attn", "jf_paged_decode_append_attn",
+             "jf_paged_verify_attn", "jf_paged_decode_attn_noalloc", "jf_prefill_chunk_attn",
+             "jf_prefill_batch_attn", "jf_kv_checkpoint", "jf_kv_restore"]
+    code = ("import paper_2609_17475_gb300.binding as B; "
+            f"print(all(hasattr(getattr(B, n), '__wrapped__') for n in {names!r}), "
+            f"any(hasattr(getattr(B, n), '__wrapped__') for n in {names!r}))")
+    import os
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    on = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=root,
+                        env=dict(os.environ, JFKV_NVTX="1"))
+    off = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=root,
+                         env=dict(os.environ, JFKV_NVTX="0"))
+    assert on.stdout.split() == ["True", "True"], on.stderr
+    assert off.stdout.split() == ["False", "False"], off.stderr

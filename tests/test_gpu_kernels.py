@@ -379,6 +379,25 @@ def test_decode_flags_a_bad_context_of_a_later_request(splits, bad):
     assert_attention_close(out[:2], ref[:2])
 
 
+def test_bounded_wait_gives_up_and_reports_timeout():
+    """The give-up path of the kernels' bounded waits: a barrier nobody
+    arrives at makes the wait run out, JF_DEV_ERR_TIMEOUT is reported, and the
+    context stays usable (a decode afterwards is still right)."""
+    st = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.binding.jf_selftest_bounded_wait(st, True)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    jf.binding.jf_selftest_bounded_wait(st, False)
+    torch.cuda.synchronize()
+    assert int(st.item()) == jf.binding.JF_DEV_ERR_TIMEOUT
+    case = make_case(93, 8, 2, 128, 64, [500])
+    ref_pool = case.oracle_pool()
+    out = gpu_decode(case, pool_from_numpy(case, ref_pool), 3)
+    ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), case.ctx, bits(case.q),
+                          1 / math.sqrt(128))
+    assert_attention_close(out, ref)
+
+
 def test_decode_full_window_256k_sampled_heads():
     """The 256K full-window workload (24/4/256, 1,024 pages in a random physical
     order, 4 K channels per KV head x20) at full size, in the launch shape the
@@ -558,6 +577,25 @@ def test_prefill_poison_pages_never_leak():
     out = gpu_prefill(case, pool, q, 200, True, 0.1)
     ref = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q), 200, 0.1)
     assert_attention_close(out, ref)
+
+
+def test_prefill_flags_groups_beyond_fp16_range():
+    """A K group scaled far past the fp16 range sets JF_DEV_ERR_RANGE (the
+    call still completes); the same cache without it leaves the status clear."""
+    from paper_2609_17475_gb300 import synth
+    case = make_case(91, 8, 2, 128, 64, [300])
+    q = synth.normal_bf16(synth.generator(92), (40, 8, 128))
+    out = gpu_prefill(case, pool_from_numpy(case, case.oracle_pool()), q, 260, True, 0.1)
+    assert torch.isfinite(out.float()).all()
+    big = case.k.clone()
+    big[123, 1, 64:128] = (big[123, 1, 64:128].float() * 40000.0).to(torch.bfloat16)
+    case.k = big
+    pool = pool_from_numpy(case, case.oracle_pool())
+    ws = torch.zeros(jf.jf_prefill_workspace_bytes(), dtype=torch.uint8, device=DEV)
+    jf.jf_prefill_chunk_attn(pool, case.page_table[0].to(DEV), q.to(DEV), 260, 0.1, True,
+                             torch.empty_like(q, device=DEV), ws)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == jf.binding.JF_DEV_ERR_RANGE
 
 
 # --------------------------------------------------------------------------
