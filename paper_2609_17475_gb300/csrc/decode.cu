@@ -766,6 +766,415 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   }
 }
 
+// Decode of a batch under the span plan (decode.cuh): the same per-split
+// work as decode_split_kernel (one 12-warp CTA per SM), run over the
+// segments in which this CTA's piece meets the batch's requests.  A separate
+// kernel, so that the single-request kernel keeps its straight-line code
+// (the same body as a lambda there measured 1.3 us slower per 256K call).
+template <int D>
+__global__ void __launch_bounds__(12 * 32, 1)
+decode_span_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a) {
+  constexpr bool VER = false;
+  constexpr int NW = 12;
+  using L = DecodeSmem<D, NW>;
+  constexpr int NG = L::NG;
+  constexpr int SBB = L::SBB;
+  constexpr float NEG_INF = -INFINITY;
+
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* codes = smem_raw;
+  uint8_t* sbuf = codes + L::CODES_BYTES;
+  uint4* qsm = reinterpret_cast<uint4*>(sbuf + L::SB_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES + L::QF_BYTES);
+
+  // decode: one CTA per KV head holds its G query heads; verifier: NT CTAs
+  // each hold 8 of its G * L (token, head) rows
+  const int kvh = VER ? (int)blockIdx.y / a.NT : (int)blockIdx.y;
+  const int nt = VER ? (int)blockIdx.y % a.NT : 0;
+  const int rows = VER ? min(8, a.G * a.L - 8 * nt) : a.G;
+  // row k of this CTA: query token i = (8 nt + k) / G, head h = (8 nt + k) % G;
+  // its q, out and partial row within the request is i * Hq + kvh * G + h
+  auto row_of = [&](int k) {
+    if constexpr (VER) {
+      const int gr = 8 * nt + k;
+      return (gr / a.G) * a.Hq + kvh * a.G + gr % a.G;
+    } else {
+      return kvh * a.G + k;
+    }
+  };
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = lane >> 2, c = lane & 3;
+  int* plan_sh = reinterpret_cast<int*>(sbuf + L::SB_BYTES + L::QF_BYTES + L::BAR_BYTES);
+  // the swizzled TMA boxes need a 1024-byte aligned window
+  const bool aligned = (smem_u32(smem_raw) & 1023) == 0;
+  if (aligned) {   // setup that reads nothing a previous kernel writes
+    if (threadIdx.x == 0) prefetch_tensormap(&tmap);
+    if (lane == 0) {
+      for (int s = 0; s < DSTAGES; ++s) mbar_init(&bars[warp * DSTAGES + s], 1);
+      fence_barrier_init();
+    }
+  }
+  // launched with programmatic dependent launch: wait for the previous
+  // kernel (e.g. the append that wrote the newest position) before any read
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+
+  // this warp's ring: bit s holds the parity of the next wait on stage s
+  // (a CTA of the span plan runs its ring through several splits)
+  uint32_t ph = 0;
+  // One split: chunks [c_begin, c_end) of request b (context ctx); its
+  // partial rows are prow0 + prow_step * (row within the request), or the
+  // output rows when `direct`; owns_last: it holds the request's last chunk
+  // (where the fused append stores the step's row).  False when a bounded
+  // wait gave up.
+  auto run_split = [&](const int b, const int ctx, const int c_begin, const int c_end,
+                       const int64_t prow0, const int64_t prow_step, const bool direct,
+                       const bool owns_last) -> bool {
+    const int n_cta = c_end - c_begin;
+    const int my_n = (n_cta > warp) ? (n_cta - warp + NW - 1) / NW : 0;
+    auto chunk_of = [&](int it) { return c_begin + warp + it * NW; };
+
+    if (a.knew != nullptr && owns_last) {   // the split holding the last chunk
+      // the new row goes to the pool before this split's TMA reads it
+      append_new_row<D>(a, b, kvh, ctx - 1, warp, lane);
+      fence_proxy_async_global();
+      __syncthreads();
+      fence_proxy_async_global();
+    }
+    __syncwarp();
+
+    // ---- query fragments (B operand of QK^T) ---------------------------------
+    const bool head_ok = r < rows;
+    const uint16_t* qrow = a.q + ((int64_t)b * a.HqL + row_of(head_ok ? r : 0)) * D;
+    uint4 qlo[NG], qhi[NG];
+    float qmax = 0.f;
+  #pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      if (head_ok) {
+        qlo[g] = *reinterpret_cast<const uint4*>(qrow + 64 * g + 8 * c);
+        qhi[g] = *reinterpret_cast<const uint4*>(qrow + 64 * g + 32 + 8 * c);
+      } else {
+        qlo[g] = make_uint4(0, 0, 0, 0);
+        qhi[g] = make_uint4(0, 0, 0, 0);
+      }
+      const uint32_t ws[8] = {qlo[g].x, qlo[g].y, qlo[g].z, qlo[g].w,
+                              qhi[g].x, qhi[g].y, qhi[g].z, qhi[g].w};
+  #pragma unroll
+      for (int i = 0; i < 8; ++i)
+        qmax = fmaxf(qmax, fmaxf(fabsf(bf16lo_to_f32(ws[i])), fabsf(bf16hi_to_f32(ws[i]))));
+    }
+  #pragma unroll
+    for (int o = 16; o > 0; o >>= 1) qmax = fmaxf(qmax, __shfl_xor_sync(0xffffffffu, qmax, o));
+    // keep |q| * 2^-qe < 2^14 so the fp16 operand cannot overflow
+    const int qe = (qmax >= 16384.f) ? (ilogbf(qmax) - 13) : 0;
+    const float qs = ldexpf(1.f, -qe);
+    const float qs16 = qs * 0.0625f;
+
+    uint32_t qf[NG][4][2];
+    float Qg[NG];
+  #pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      float e[16];
+      const uint32_t ws[8] = {qlo[g].x, qlo[g].y, qlo[g].z, qlo[g].w,
+                              qhi[g].x, qhi[g].y, qhi[g].z, qhi[g].w};
+  #pragma unroll
+      for (int i = 0; i < 8; ++i) { e[2 * i] = bf16lo_to_f32(ws[i]); e[2 * i + 1] = bf16hi_to_f32(ws[i]); }
+      // word W covers d = base..base+7; nib0 -> (base, base+4), nib1 -> (base+1, base+5) x16,
+      // nib0 of W>>8 -> (base+2, base+6), nib1 of W>>8 -> (base+3, base+7) x16
+  #pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const float* x = e + 8 * h;
+        qf[g][2 * h + 0][0] = pack_f16x2(x[0] * qs, x[4] * qs);
+        qf[g][2 * h + 0][1] = pack_f16x2(x[1] * qs16, x[5] * qs16);
+        qf[g][2 * h + 1][0] = pack_f16x2(x[2] * qs, x[6] * qs);
+        qf[g][2 * h + 1][1] = pack_f16x2(x[3] * qs16, x[7] * qs16);
+      }
+      float sum = 0.f;
+  #pragma unroll
+      for (int i = 0; i < 16; ++i) sum += e[i];
+      sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+      sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+      Qg[g] = sum;
+    }
+    // QK bias B fragment for head r: k-slot k < NG is Q_k high, NG <= k < 2 NG
+    // is Q_{k-NG} low (the bf16 residual); thread c holds slots 2c, 2c+1.
+    uint32_t bq = 0;
+    {
+      float hi[NG], lo[NG];
+  #pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        hi[g] = __bfloat162float(__float2bfloat16_rn(Qg[g]));
+        lo[g] = Qg[g] - hi[g];
+      }
+      if constexpr (NG == 4) {
+        if (c == 0) bq = pack_bf16x2(hi[0], hi[1]);
+        else if (c == 1) bq = pack_bf16x2(hi[2], hi[3]);
+        else if (c == 2) bq = pack_bf16x2(lo[0], lo[1]);
+        else bq = pack_bf16x2(lo[2], lo[3]);
+      } else {
+        if (c == 0) bq = pack_bf16x2(hi[0], hi[1]);
+        else if (c == 1) bq = pack_bf16x2(lo[0], lo[1]);
+      }
+    }
+    const float cA = a.scale_log2 * 16777216.f * ldexpf(1.f, qe);
+    const float cB = a.scale_log2;
+
+    // ---- page ids: lane i holds the page of this warp's iteration 32k + i ------
+    // (two blocks of 32 in flight so the dependent load never stalls an issue)
+    auto load_pages = [&](int blk) -> int {
+      const int it = blk * 32 + lane;
+      int page = -1;
+      if (it < my_n) {
+        const int pidx = (chunk_of(it) * DTOK) >> a.log2P;
+        if (pidx < a.pt_stride) page = __ldg(a.page_table + (int64_t)b * a.pt_stride + pidx);
+      }
+      return page;
+    };
+    int pg_cur = load_pages(0);
+    int pg_next = load_pages(1);
+
+    // ---- TMA producer (lane 0 of each warp feeds its own ring) -------------
+    // decode reads each page once per call: evict it from L2 first; the
+    // verifier's n-tile CTAs read the same pages, so L2 keeps them normally
+    const uint64_t l2pol = VER ? l2_evict_normal_policy() : l2_evict_first_policy();
+    uint32_t valid = 0;
+    auto issue = [&](int it) {
+      const int s = it % DSTAGES;
+      if (it >= 32 && (it & 31) == 0) {
+        pg_cur = pg_next;
+        pg_next = load_pages((it >> 5) + 1);
+      }
+      const int page = __shfl_sync(0xffffffffu, pg_cur, it & 31);
+      const bool ok = page >= 0 && page < a.num_pages;
+      if (lane == 0) {
+        const int inp = (chunk_of(it) * DTOK) & (a.P - 1);
+        uint64_t* bar = &bars[warp * DSTAGES + s];
+        if (!ok) {
+          flag_error(a.status, JF_DEV_ERR_PAGE_ID);
+          mbar_arrive(bar);
+        } else {
+          uint8_t* kc = codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF;
+          uint8_t* ks = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
+          const uint8_t* gsb = a.pool + (int64_t)page * a.page_bytes + a.sb_base +
+                               ((int64_t)kvh * a.P + inp) * SBB;
+          mbar_arrive_expect_tx(bar, L::STAGE_TX);
+          tma_load_5d_hint(kc, &tmap, 0, inp, kvh, 0, page, bar, l2pol);
+          tma_load_5d_hint(kc + L::CODE_BUF, &tmap, 0, inp, kvh, 1, page, bar, l2pol);
+          bulk_g2s_hint(ks, gsb, L::SB_BUF, bar, l2pol);
+          bulk_g2s_hint(ks + L::SB_BUF, gsb + a.sb_region, L::SB_BUF, bar, l2pol);
+        }
+      }
+      valid = (valid & ~(1u << s)) | ((uint32_t)ok << s);
+    };
+
+    const int npro = my_n < DSTAGES ? my_n : DSTAGES;
+    for (int it = 0; it < npro; ++it) issue(it);
+
+    // ---- running state ---------------------------------------------------
+    DecodeState<NG> st;
+    st.init();
+
+    // ldmatrix row address pieces: matrix m = lane>>3 -> (position half, chunk)
+    const int ld_t = (lane & 7) + 8 * ((lane >> 3) & 1);
+    const int ld_ch = lane >> 4;
+    if (warp == 0) {
+  #pragma unroll
+      for (int g = 0; g < NG; ++g) {
+        qsm[(2 * g) * 32 + lane] = make_uint4(qf[g][0][0], qf[g][0][1], qf[g][1][0], qf[g][1][1]);
+        qsm[(2 * g + 1) * 32 + lane] = make_uint4(qf[g][2][0], qf[g][2][1], qf[g][3][0], qf[g][3][1]);
+      }
+    }
+    __syncthreads();
+    ChunkCtx<NG> cc{qsm + lane, bq, cA, cB, r, c, {}};
+  #pragma unroll
+    for (int g = 0; g < NG; ++g) cc.koff[g] = swz<L::CB>(ld_t, 2 * g + ld_ch);
+
+    // verifier causal limits: query token i of L sees positions < ctx - L + 1 + i;
+    // a chunk below ctx_all is visible to every row (decode: ctx_all = ctx)
+    int ctx_all = ctx, lim0 = ctx, lim1 = ctx;
+    if constexpr (VER) {
+      ctx_all = ctx - a.L + 1;
+      lim0 = min(ctx, ctx_all + (8 * nt + 2 * c) / a.G);
+      lim1 = min(ctx, ctx_all + (8 * nt + 2 * c + 1) / a.G);
+    }
+    int done = 0;
+    // unrolled by the ring depth, so every stage address is a constant offset
+  #pragma unroll DSTAGES
+    for (int it = 0; it < my_n; ++it) {
+      const int s = it % DSTAGES;
+      if (!mbar_wait_bounded(&bars[warp * DSTAGES + s], (ph >> s) & 1u)) {
+        if (lane == 0) flag_error(a.status, JF_DEV_ERR_TIMEOUT);
+        break;
+      }
+      ph ^= 1u << s;
+      done = it + 1;
+      const bool ok = (valid >> s) & 1u;
+      const int tokbase = chunk_of(it) * DTOK;
+      const uint32_t kc = smem_u32(codes + (warp * DSTAGES + s) * 2 * L::CODE_BUF);
+      const uint8_t* ksb = sbuf + (warp * DSTAGES + s) * 2 * L::SB_BUF;
+      if (ok && tokbase + DTOK <= (VER ? ctx_all : ctx)) {
+        process_chunk<D, true>(st, cc, kc, ksb, 0, 0, 0);
+      } else if constexpr (VER) {
+        process_chunk<D, false>(st, cc, kc, ksb, ok ? ctx - tokbase : 0,
+                                ok ? lim0 - tokbase : 0, ok ? lim1 - tokbase : 0);
+      } else {
+        const int nv = ok ? ctx - tokbase : 0;
+        process_chunk<D, false>(st, cc, kc, ksb, nv, nv, nv);
+      }
+
+      __syncwarp();
+      if (it + DSTAGES < my_n) {
+        fence_proxy_async_smem();
+        issue(it + DSTAGES);
+      }
+    }
+    const bool gave_up = done < my_n;
+    if (gave_up) {
+      // a wait gave up: give copies still in flight a bounded chance to land
+      for (int it = done; it < my_n && it < done + DSTAGES; ++it)
+        mbar_wait_bounded(&bars[warp * DSTAGES + it % DSTAGES], (ph >> (it % DSTAGES)) & 1u,
+                          1u << 16);
+    }
+    float& m0 = st.m0;
+    float& m1 = st.m1;
+    float& l0 = st.l0;
+    float& l1 = st.l1;
+    auto& O = st.O;
+
+    // the merge kernel may start launching; it waits for this grid to finish
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+
+    // ---- per-warp finalize ---------------------------------------------------
+  #pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+    }
+    // bias sums: lane (r = g, c) of the MMA accumulator holds group g, heads 2c, 2c+1
+    float Bs[NG][2];
+  #pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      Bs[g][0] = __shfl_sync(0xffffffffu, st.Bs[0], g * 4 + c);
+      Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
+    }
+    // This warp's ring is idle now (each of its copies has landed and been
+    // read), so its O rows (padded by 4 floats: the 128-bit stores of one
+    // quarter-warp hit 8 distinct bank groups) and (m, l) per head go into its
+    // own stage buffers at once, without waiting for the other warps.
+    constexpr int SROW = D + 4;
+    constexpr int WCODES = DSTAGES * 2 * L::CODE_BUF;   // one warp's code ring (bytes)
+    constexpr int WSB = DSTAGES * 2 * L::SB_BUF;        // one warp's scale/bias ring
+    static_assert(8 * SROW * 4 <= WCODES && 8 * 2 * 4 <= WSB, "combine rows fit a warp's ring");
+    {
+      float* so = reinterpret_cast<float*>(codes + warp * WCODES);   // [8][SROW]
+      float* sml = reinterpret_cast<float*>(sbuf + warp * WSB);      // [8][2]
+  #pragma unroll
+      for (int g = 0; g < NG; ++g) {
+  #pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {          // d block 64g + 32 hf + 4r + e
+  #pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {        // head 2c + hh
+            if (2 * c + hh < rows) {
+              float4 v;
+              // 2^24 undoes the fp16 subnormal codes (2^20 for the hi nibbles)
+              v.x = fmaf(O[g][0][2 * hf + hh], 16777216.f, Bs[g][hh]);
+              v.y = fmaf(O[g][1][2 * hf + hh], 1048576.f, Bs[g][hh]);
+              v.z = fmaf(O[g][2][2 * hf + hh], 16777216.f, Bs[g][hh]);
+              v.w = fmaf(O[g][3][2 * hf + hh], 1048576.f, Bs[g][hh]);
+              *reinterpret_cast<float4*>(so + (2 * c + hh) * SROW + 64 * g + 32 * hf + 4 * r) = v;
+            }
+          }
+        }
+      }
+      if (r == 0) {
+        sml[(2 * c) * 2 + 0] = m0;
+        sml[(2 * c) * 2 + 1] = l0;
+        sml[(2 * c + 1) * 2 + 0] = m1;
+        sml[(2 * c + 1) * 2 + 1] = l1;
+      }
+    }
+    __syncthreads();
+
+    // ---- combine the warps of this CTA --------------------------------------
+    // per head: M = max_w m_w, weights 2^(m_w - M) (divided by L when this CTA
+    // writes the final output), L = sum_w 2^(m_w - M) l_w; every thread works
+    // out the weights of its own head.
+    for (int idx = threadIdx.x; idx < rows * (D / 4); idx += blockDim.x) {
+      const int h = idx / (D / 4), d = 4 * (idx % (D / 4));
+      float mw[NW], lw[NW];
+      float M = NEG_INF;
+  #pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float2 v = *reinterpret_cast<const float2*>(sbuf + w * WSB + h * 8);
+        mw[w] = v.x;
+        lw[w] = v.y;
+        M = fmaxf(M, v.x);
+      }
+      float f[NW];
+      float Lsum = 0.f;
+  #pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        f[w] = (mw[w] != NEG_INF) ? fast_exp2(mw[w] - M) : 0.f;
+        Lsum = fmaf(f[w], lw[w], Lsum);
+      }
+      const float inv = direct ? (Lsum > 0.f ? 1.f / Lsum : 0.f) : 1.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  #pragma unroll
+      for (int w = 0; w < NW; ++w) {
+        const float fw = f[w] * inv;
+        const float4 v = *reinterpret_cast<const float4*>(
+            reinterpret_cast<const float*>(codes + w * WCODES) + h * SROW + d);
+        if (fw != 0.f) {
+          acc.x = fmaf(fw, v.x, acc.x);
+          acc.y = fmaf(fw, v.y, acc.y);
+          acc.z = fmaf(fw, v.z, acc.z);
+          acc.w = fmaf(fw, v.w, acc.w);
+        }
+      }
+      const int fr = row_of(h);
+      if (direct) {
+        uint2 o;
+        o.x = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.x)) |
+              ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.y)) << 16);
+        o.y = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.z)) |
+              ((uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(acc.w)) << 16);
+        *reinterpret_cast<uint2*>(a.out + ((int64_t)b * a.HqL + fr) * D + d) = o;
+      } else {
+        const int64_t row = prow0 + prow_step * fr;   // this split's partial row
+        *reinterpret_cast<float4*>(a.part_o + row * D + d) = acc;
+        if (d == 0) {
+          a.part_ml[row * 2 + 0] = M;
+          a.part_ml[row * 2 + 1] = Lsum;
+        }
+      }
+    }
+    // one CTA-wide answer (and the barrier after which a span plan's next
+    // split may reuse the rings and query fragments)
+    return __syncthreads_or(gave_up ? 1 : 0) == 0;
+  };
+
+  if (!aligned) {
+    if (threadIdx.x == 0) flag_error(a.status, JF_DEV_ERR_LAYOUT);
+    return;
+  }
+  // pieces of W chunks cut from the batch's chunks laid end to end; piece
+  // x meets requests in segments, each a split with partial row x + b
+  const long long T = span_total(a, lane);
+  const int W = span_width(T, a.budget);
+  long long pos = (long long)blockIdx.x * W;
+  const long long end = min(pos + W, T);
+  while (pos < end) {
+    const SpanHit h = span_find(a, pos, lane);
+    if (h.b < 0) break;
+    const int c0 = (int)(pos - h.start);
+    const int c1 = (int)(min(end, h.start + h.nch) - h.start);
+    const int ctx = checked_ctx(a, h.b, c0);
+    if (!run_split(h.b, ctx, c0, c1, ((int64_t)blockIdx.x + h.b) * a.HqL, 1, false,
+                   c1 == h.nch))
+      return;   // a bounded wait gave up (reported); the CTA stops
+    pos = h.start + c1;
+  }
+}
+
 
 // Merge for one or a few requests: one CTA per (32-wide slice of head_dim,
 // query row, request); its 8 warps take interleaved splits and reduce through
@@ -781,8 +1190,11 @@ constexpr int MERGE_NSG = MERGE_THREADS / MERGE_DSLICE;   // split groups
 constexpr int MERGE_SG_BATCH = 16;                        // splits per thread per batch
 constexpr int MERGE_MLB = MERGE_SG_BATCH * MERGE_NSG / 32;   // (m, l) rows per lane per batch
 
-template <int D>
+template <int D, bool SPAN>
 __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_sg_kernel(const DecodeArgs a) {
+  // SPAN: partial rows of the span plan.  A template parameter: the span
+  // branch in the single-request instance, though never taken, had slowed
+  // the 256K call by ~1.2 us.
   __shared__ float red[MERGE_NSG][MERGE_DSLICE];
   // the next kernel in the stream may be scheduled now; it waits for this
   // grid to complete before it reads anything
@@ -808,6 +1220,19 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_sg_kernel(const De
       if (lane == 0) {
         plan_sh[0] = p.g0;
         plan_sh[1] = p.nsplit;
+      }
+    }
+    __syncthreads();
+    row0 = (int64_t)plan_sh[0] * a.HqL + hq;
+    rs = a.HqL;
+    nsplit_bal = plan_sh[1];
+    S = nsplit_bal;
+  } else if constexpr (SPAN) {
+    if (t < 32) {
+      const SpanRows sr = span_rows(a, b, lane);
+      if (lane == 0) {
+        plan_sh[0] = sr.row;
+        plan_sh[1] = sr.n;
       }
     }
     __syncthreads();
@@ -841,7 +1266,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_sg_kernel(const De
   if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
   split_plan(ctx, a.plan_splits, nch, cps, nsplit);
-  if (a.balanced) nsplit = nsplit_bal;
+  if (a.balanced || SPAN) nsplit = nsplit_bal;
   uint16_t* orow = a.out + ((int64_t)b * a.HqL + hq) * D + d0;
   if (nsplit == 0) {
     if (t < MERGE_DSLICE) orow[t] = 0;
@@ -909,7 +1334,7 @@ __global__ void __launch_bounds__(MERGE_THREADS) decode_merge_sg_kernel(const De
 // the workspace holds there).
 constexpr int MERGE_BATCH = 64;   // splits per batch: two per lane for the weights
 
-template <int D>
+template <int D, bool SPAN>
 __global__ void __launch_bounds__(D / 2) decode_merge_kernel(const DecodeArgs a) {
   // the next kernel in the stream may be scheduled now; it waits for this
   // grid to complete before it reads anything
@@ -926,6 +1351,12 @@ __global__ void __launch_bounds__(D / 2) decode_merge_kernel(const DecodeArgs a)
     rs = a.HqL;
     nsplit_bal = p.nsplit;
     S = p.nsplit;
+  } else if constexpr (SPAN) {
+    const SpanRows sr = span_rows(a, b, lane);
+    row0 = (int64_t)sr.row * a.HqL + hq;
+    rs = a.HqL;
+    nsplit_bal = sr.n;
+    S = sr.n;
   } else {
     row0 = ((int64_t)b * a.HqL + hq) * a.num_splits;
     rs = 1;
@@ -951,7 +1382,7 @@ __global__ void __launch_bounds__(D / 2) decode_merge_kernel(const DecodeArgs a)
   if (ctx > cap) ctx = (int)cap;
   int nch, cps, nsplit;
   split_plan(ctx, a.plan_splits, nch, cps, nsplit);
-  if (a.balanced) nsplit = nsplit_bal;
+  if (a.balanced || SPAN) nsplit = nsplit_bal;
   uint32_t* orow = reinterpret_cast<uint32_t*>(a.out + ((int64_t)b * a.HqL + hq) * D) + t;
   if (nsplit == 0) {
     *orow = 0u;
@@ -1057,22 +1488,32 @@ int launch_decode_merge(const DecodeArgs& a, int D, int B, cudaStream_t stream) 
   mc.attrs = pdl;
   mc.numAttrs = 1;
   cudaError_t e;
-  if (sg)
-    e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<256>, a)
-                   : cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<128>, a);
-  else
-    e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256>, a)
-                   : cudaLaunchKernelEx(&mc, decode_merge_kernel<128>, a);
+  if (sg) {
+    if (a.span)
+      e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<256, true>, a)
+                     : cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<128, true>, a);
+    else
+      e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<256, false>, a)
+                     : cudaLaunchKernelEx(&mc, decode_merge_sg_kernel<128, false>, a);
+  } else {
+    if (a.span)
+      e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256, true>, a)
+                     : cudaLaunchKernelEx(&mc, decode_merge_kernel<128, true>, a);
+    else
+      e = (D == 256) ? cudaLaunchKernelEx(&mc, decode_merge_kernel<256, false>, a)
+                     : cudaLaunchKernelEx(&mc, decode_merge_kernel<128, false>, a);
+  }
   return e == cudaSuccess ? JF_OK : JF_ERR_CUDA;
 }
 
-template <int D, int NW>
+template <int D, bool VER, int NW, bool SPAN>
 static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
                            cudaStream_t stream) {
   using L = DecodeSmem<D, NW>;
-  if (smem_optin((const void*)decode_split_kernel<D, false, NW>, L::TOTAL) != JF_OK ||
-      smem_optin((const void*)decode_split_kernel<D, true, NW>, L::TOTAL) != JF_OK)
-    return JF_ERR_CUDA;
+  static_assert(!SPAN || (NW == 12 && !VER), "the span kernel is the 12-warp decode");
+  const void* kernel = SPAN ? (const void*)decode_span_kernel<D>
+                            : (const void*)decode_split_kernel<D, VER, NW>;
+  if (smem_optin(kernel, L::TOTAL) != JF_OK) return JF_ERR_CUDA;
   // Both kernels use programmatic dependent launch: each may be scheduled
   // while the previous kernel in the stream drains, and waits (griddepcontrol)
   // before it reads anything that kernel wrote.
@@ -1080,40 +1521,39 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
   pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   pdl[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
-  // batch plan: a.budget + B CTAs per KV head cover every split (sum_b n_b <=
-  // T / cps + B <= budget + B); per-request plans: plan_splits per request
-  cfg.gridDim = a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)(a.Hkv * a.NT), 1u)
+  // span plan: budget pieces per KV head; batch plan: a.budget + B CTAs per
+  // KV head cover every split (sum_b n_b <= T / cps + B <= budget + B);
+  // per-request plans: plan_splits per request
+  cfg.gridDim = SPAN ? dim3((unsigned)a.budget, (unsigned)a.Hkv, 1u)
+              : a.balanced ? dim3((unsigned)(a.budget + B), (unsigned)(a.Hkv * a.NT), 1u)
                            : dim3((unsigned)a.plan_splits, (unsigned)(a.Hkv * a.NT), (unsigned)B);
   cfg.blockDim = dim3(NW * 32);
   cfg.dynamicSmemBytes = L::TOTAL;
   cfg.stream = stream;
   cfg.attrs = pdl;
   cfg.numAttrs = 1;
-  const cudaError_t e =
-      (a.L > 1) ? cudaLaunchKernelEx(&cfg, decode_split_kernel<D, true, NW>, tmap, a)
-                : cudaLaunchKernelEx(&cfg, decode_split_kernel<D, false, NW>, tmap, a);
+  cudaError_t e;
+  if constexpr (SPAN)
+    e = cudaLaunchKernelEx(&cfg, decode_span_kernel<D>, tmap, a);
+  else
+    e = cudaLaunchKernelEx(&cfg, decode_split_kernel<D, VER, NW>, tmap, a);
   if (e != cudaSuccess) return JF_ERR_CUDA;
-  if (a.balanced || a.plan_splits > 1) return launch_decode_merge(a, D, B, stream);
+  if (a.span || a.balanced || a.plan_splits > 1) return launch_decode_merge(a, D, B, stream);
   return JF_OK;
 }
 
-// Warps per split CTA for a call (the NW template parameter).  Two 6-warp
+// Warps per split CTA (the NW template parameter) and the plan.  Two 6-warp
 // CTAs on one SM do not share it evenly: the CTA placed first keeps issue
-// priority and ends its share ~4 us (of ~50) before the other, so one request
-// (and a batch whose workspace has fewer partial rows than the 6-warp grid
-// has CTA slots) runs one 12-warp CTA per SM.  A batch with rows to spare
-// keeps the 6-warp CTAs: their pieces are half as long, so cutting unequal
-// requests into pieces leaves less unevenness.
+// priority and ends its share ~4 us (of ~50) before the other, so decode runs
+// one 12-warp CTA per SM: a single request with per-request splits, a batch
+// with the span plan (equal pieces, so the longer pieces of 12-warp CTAs
+// leave no unevenness).  The packed verifier keeps 6-warp CTAs (measured
+// faster) and the batch plan of whole-request pieces; many requests that do
+// not fit one wave of 12-warp CTAs use 6-warp CTAs.
 static int decode_warps(int batch, int num_splits, int Hkv, int NT) {
-  if (NT > 1) return 6;   // packed verifier: measured slower with 12-warp CTAs
-  const int64_t sms = sm_count();
-  if (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) {   // batch split plan
-    const int64_t slots6 = (2 * sms + Hkv * NT - 1) / (Hkv * NT);
-    const int64_t fit = (int64_t)batch * num_splits - batch;
-    return fit < slots6 ? 12 : 6;
-  }
-  // per-request plans: one 12-warp CTA per SM while they fit in one wave
-  return (batch == 1 || (int64_t)batch * Hkv * NT * num_splits <= sms) ? 12 : 6;
+  if (NT > 1) return 6;
+  if (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) return 12;   // span plan
+  return (batch == 1 || (int64_t)batch * Hkv * NT * num_splits <= sm_count()) ? 12 : 6;
 }
 
 int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
@@ -1156,21 +1596,35 @@ int launch_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap
   const int slots = (per_sm * sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
   // per-request plans: one CTA wave (12-warp CTAs) or the caller's cap
   a.plan_splits = (nw == 12 && num_splits > slots) ? slots : num_splits;
-  // Batches of up to BAL_MAX_B requests size their splits for the whole batch
-  // (balanced_plan): one CTA per slot in all, fewer than B * num_splits
-  // (minus B/2 for rounding) so every split's partial row fits the workspace.
-  a.balanced = (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) ? 1 : 0;
+  // Batches of up to BAL_MAX_B requests size their splits for the whole
+  // batch: decode with the span plan (one piece per CTA slot, within the
+  // workspace's B * num_splits rows: budget <= B (num_splits - 1) + 1), the
+  // verifier with balanced_plan (whole-request pieces, fewer than
+  // B * num_splits minus B/2 for rounding).
+  const bool batch_plan = batch > 1 && batch <= BAL_MAX_B && num_splits > 1;
+  a.span = (batch_plan && q_len == 1) ? 1 : 0;
+  a.balanced = (batch_plan && q_len > 1) ? 1 : 0;
   a.budget = 1;
-  if (a.balanced) {
+  if (a.span) {
+    const int64_t fit = (int64_t)batch * (num_splits - 1) + 1;
+    a.budget = (int)(fit < slots ? fit : slots);
+  } else if (a.balanced) {
     const int64_t fit = (int64_t)batch * num_splits - batch;
     const int64_t cap = fit < slots ? fit : slots;
     a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);
   }
+  const bool d256 = g.D == 256;
+  if (q_len > 1)
+    return d256 ? launch_decode_t<256, true, 6, false>(tmap, a, batch, stream)
+                : launch_decode_t<128, true, 6, false>(tmap, a, batch, stream);
+  if (a.span)
+    return d256 ? launch_decode_t<256, false, 12, true>(tmap, a, batch, stream)
+                : launch_decode_t<128, false, 12, true>(tmap, a, batch, stream);
   if (nw == 12)
-    return g.D == 256 ? launch_decode_t<256, 12>(tmap, a, batch, stream)
-                      : launch_decode_t<128, 12>(tmap, a, batch, stream);
-  return g.D == 256 ? launch_decode_t<256, 6>(tmap, a, batch, stream)
-                    : launch_decode_t<128, 6>(tmap, a, batch, stream);
+    return d256 ? launch_decode_t<256, false, 12, false>(tmap, a, batch, stream)
+                : launch_decode_t<128, false, 12, false>(tmap, a, batch, stream);
+  return d256 ? launch_decode_t<256, false, 6, false>(tmap, a, batch, stream)
+              : launch_decode_t<128, false, 6, false>(tmap, a, batch, stream);
 }
 
 }  // namespace jfkv

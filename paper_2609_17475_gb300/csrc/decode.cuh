@@ -38,6 +38,7 @@ struct DecodeArgs {
   int32_t NT;          // CTAs per KV head, each for 8 of its G * L (token, head) rows
   int32_t HqL;         // L * Hq: rows of q, out and the partials per request
   int32_t balanced;    // 1: batch split plan (balanced_plan), partial rows by global split
+  int32_t span;        // 1: batch span plan (span_find), partial rows (piece + request)
   int32_t budget;      // balanced: target splits per KV head over the whole batch
 };
 
@@ -102,6 +103,84 @@ static __device__ BalPlan balanced_plan(const DecodeArgs& a, int x, int want_b, 
     base += __shfl_sync(0xffffffffu, incl, 31);
   }
   return p;
+}
+
+// Span plan (batches of the affine decode).  The chunks of all requests are
+// laid end to end (request 0 first) and cut into pieces of W chunks,
+// W = max(MIN_CPS, ceil(T / budget)), T the total: every piece carries the
+// same work however unequal the requests are.  Piece x meets requests in
+// segments; the segment of request b is one split whose partial rows are
+// (x + b) * HqL + hq (along the sequence every piece or request boundary
+// advances x + b, so the numbers never repeat, and a request's rows are
+// contiguous: x0_b + b .. x1_b + b).  The workspace holds B * num_splits
+// rows per query row, so budget <= B * (num_splits - 1) + 1.
+__device__ __forceinline__ int span_nch(const DecodeArgs& a, int b) {
+  const int64_t cap = (int64_t)a.pt_stride * a.P;
+  int64_t c = a.ctx[b];
+  c = c < 0 ? 0 : (c > cap ? cap : c);
+  return (int)((c + DTOK - 1) / DTOK);
+}
+
+// total chunks of the batch (every lane of the calling warp gets it)
+static __device__ long long span_total(const DecodeArgs& a, int lane) {
+  long long T = 0;
+  for (int bb = lane; bb < a.B; bb += 32) T += span_nch(a, bb);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) T += __shfl_xor_sync(0xffffffffu, T, o);
+  return T;
+}
+
+__host__ __device__ inline int span_width(long long T, int budget) {
+  long long w = (T + budget - 1) / (budget > 0 ? budget : 1);
+  return (int)(w < MIN_CPS ? MIN_CPS : w);
+}
+
+struct SpanHit {
+  int b;            // request (-1: none)
+  long long start;  // its first chunk in the batch sequence
+  int nch;          // its chunks
+};
+
+// The request holding batch chunk `pos` (pos >= 0), or, with pos < 0, request
+// want_b itself.  Called by a whole warp.
+static __device__ SpanHit span_find(const DecodeArgs& a, long long pos, int lane,
+                                    int want_b = -1) {
+  long long base = 0;
+  for (int b0 = 0; b0 < a.B; b0 += 32) {
+    const int bb = b0 + lane;
+    const int n = (bb < a.B) ? span_nch(a, bb) : 0;
+    long long incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const long long excl = base + incl - n;
+    const bool hit = (pos >= 0) ? (bb < a.B && n > 0 && pos >= excl && pos < excl + n)
+                                : (bb == want_b);
+    const unsigned m = __ballot_sync(0xffffffffu, hit);
+    if (m) {
+      const int src = __ffs(m) - 1;
+      return SpanHit{__shfl_sync(0xffffffffu, bb, src), __shfl_sync(0xffffffffu, excl, src),
+                     __shfl_sync(0xffffffffu, n, src)};
+    }
+    base += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  return SpanHit{-1, 0, 0};
+}
+
+// Partial rows of request b under the span plan: rows row .. row + n - 1
+// (n = 0 for an empty request).  Called by a whole warp.
+struct SpanRows {
+  int row, n;
+};
+static __device__ SpanRows span_rows(const DecodeArgs& a, int b, int lane) {
+  const long long T = span_total(a, lane);
+  const SpanHit h = span_find(a, -1, lane, b);
+  if (h.nch <= 0) return SpanRows{0, 0};
+  const int W = span_width(T, a.budget);
+  const int x0 = (int)(h.start / W), x1 = (int)((h.start + h.nch - 1) / W);
+  return SpanRows{x0 + b, x1 - x0 + 1};
 }
 
 // Context length of request b clamped to [0, pt_stride * P].  An out-of-range

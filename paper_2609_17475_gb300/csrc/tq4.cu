@@ -988,6 +988,7 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   a.part_o = reinterpret_cast<float*>(ws + 256 + (rows * 8 + 255) / 256 * 256);
   a.num_splits = num_splits;
   a.plan_splits = num_splits;
+  a.span = 0;
   a.scale_log2 = softmax_scale * 1.4426950408889634f;
   a.B = batch;
   a.balanced = (batch > 1 && batch <= 1024 && num_splits > 1) ? 1 : 0;

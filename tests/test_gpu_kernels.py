@@ -167,10 +167,31 @@ def test_decode_matches_oracle(Hq, Hkv, D, P, ctx, splits, outliers):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("Hq,Hkv,D,P,splits", [(8, 2, 128, 64, 2), (24, 4, 256, 128, 3)])
+def test_decode_batch_pieces_spanning_many_requests(Hq, Hkv, D, P, splits):
+    """Batches cut the requests' chunks, laid end to end, into equal pieces:
+    with few splits and many short requests a piece crosses many request
+    boundaries (empty requests, single positions, exact chunk and page
+    multiples), and every request still matches the oracle."""
+    ctx = [0, 1, 31, 32, 33, 64, 65, 500, 0, 2048, 7, 1000, 3, 4096, 129, 1, 0, 777, 256, 5000,
+           31, 33, 96, 97, 1500, 2, 640, 2049, 15, 300]
+    case = make_case(700 + D, Hq, Hkv, D, P, ctx, outliers=True)
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    out = gpu_decode(case, pool, splits)
+    ref = OT.paged_decode(ref_pool, case.layout, case.page_table.numpy(), ctx, bits(case.q),
+                          1 / math.sqrt(D))
+    assert_attention_close(out, ref)
+    for b, c in enumerate(ctx):
+        if c == 0:
+            assert (out[b].float() == 0).all()
+
+
 @pytest.mark.parametrize("Hq,Hkv,D,P,ctx,splits", [
     (24, 4, 256, 256, [5000, 257, 1], 76),   # new rows mid-page, at slot 0 of a page, alone
     (8, 2, 128, 64, [64, 65, 999], 4),
     (16, 2, 256, 128, [3000], 1),            # one split writes and reads directly
+    (8, 2, 128, 64, [1, 40, 2, 33, 700, 65, 3], 2),   # pieces spanning requests
 ])
 def test_fused_append_decode_equals_append_then_decode(Hq, Hkv, D, P, ctx, splits):
     """jf_paged_decode_append_attn leaves the same pool bytes and output as
