@@ -262,3 +262,61 @@ def test_nvtx_ranges_wrap_every_enqueueing_call_when_enabled():
                          env=dict(os.environ, JFKV_NVTX="0"))
     assert on.stdout.split() == ["True", "True"], on.stderr
     assert off.stdout.split() == ["False", "False"], off.stderr
+
+
+def _span_segments(ctx, budget, dtok=32, min_cps=16):
+    """The span plan's segments as the decode kernels work them out
+    (decode.cuh: span_width, span_find, span_rows): requests' chunks laid end
+    to end, pieces of W chunks, segment (piece x, request b) -> row x + b."""
+    nch = [(max(0, c) + dtok - 1) // dtok for c in ctx]
+    T = sum(nch)
+    W = max(min_cps, -(-T // max(budget, 1)))
+    starts = [sum(nch[:b]) for b in range(len(nch))]
+    segs = []
+    for x in range(budget):
+        pos, end = x * W, min((x + 1) * W, T)
+        while pos < end:
+            b = next(b for b in range(len(nch)) if nch[b] and starts[b] <= pos < starts[b] + nch[b])
+            c1 = min(end, starts[b] + nch[b]) - starts[b]
+            segs.append((x, b, pos - starts[b], c1))
+            pos = starts[b] + c1
+    merge = {}
+    for b in range(len(nch)):
+        if nch[b]:
+            x0, x1 = starts[b] // W, (starts[b] + nch[b] - 1) // W
+            merge[b] = (x0 + b, x1 - x0 + 1)
+    return nch, W, segs, merge
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_span_plan_rows_are_unique_contiguous_and_inside_the_workspace(seed):
+    """Every request's chunks are covered exactly once by segments; each
+    segment's partial row x + b is distinct, a request's rows are the
+    contiguous run the merge reads, and every row fits the workspace's
+    B * num_splits rows when budget <= B (num_splits - 1) + 1."""
+    rng = np.random.default_rng(seed)
+    B = int(rng.integers(2, 40))
+    num_splits = int(rng.integers(2, 8))
+    ctx = [int(c) for c in rng.choice([0, 1, 31, 32, 33, 500, 4096, 70000], size=B)]
+    ctx = [c if rng.random() < 0.5 else int(rng.integers(0, 90000)) for c in ctx]
+    slots = 38
+    budget = min(slots, B * (num_splits - 1) + 1)
+    nch, W, segs, merge = _span_segments(ctx, budget)
+    rows = [x + b for (x, b, c0, c1) in segs]
+    assert len(rows) == len(set(rows))
+    assert max(rows, default=0) < B * num_splits
+    for b in range(B):
+        mine = sorted((c0, c1, x + b) for (x, bb, c0, c1) in segs if bb == b)
+        covered = [c for c0, c1, _ in mine for c in range(c0, c1)]
+        assert covered == list(range(nch[b]))
+        if nch[b]:
+            first, n = merge[b]
+            assert [r for _, _, r in mine] == list(range(first, first + n))
+        else:
+            assert b not in merge
+    # the pieces carry equal work: every piece but the last holds exactly W chunks
+    per_piece = {}
+    for (x, b, c0, c1) in segs:
+        per_piece[x] = per_piece.get(x, 0) + (c1 - c0)
+    full = [per_piece[x] for x in sorted(per_piece)][:-1]
+    assert all(w == W for w in full)
