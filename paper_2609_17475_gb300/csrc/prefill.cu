@@ -117,6 +117,26 @@ struct PfSmem {
   static_assert(TOTAL <= 227 * 1024, "shared memory per CTA");
 };
 
+// packed fp32 pairs (Blackwell f32x2 arithmetic)
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};\n" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack_f32x2(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;\n" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t sub_f32x2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;\n" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t add_f32x2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;\n" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
 __device__ __forceinline__ uint32_t hmul2(uint32_t a, uint32_t b) {
   uint32_t r;
   asm("mul.rn.f16x2 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
@@ -571,15 +591,27 @@ prefill_kernel(const __grid_constant__ PrefillArgs a) {
         m_ref = nref;
       }
       uint32_t p[32];
-      float l4[4] = {0.f, 0.f, 0.f, 0.f};
+      if (m_ref == -INFINITY) {   // nothing visible yet on this row
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        const float p0 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c] - m_ref);
-        const float p1 = (m_ref == -INFINITY) ? 0.f : fast_exp2(x[2 * c + 1] - m_ref);
-        l4[c & 3] += p0 + p1;
-        p[c] = pack_f16x2(p0, p1);
+        for (int c = 0; c < 32; ++c) p[c] = 0u;
+      } else {
+        // x - m and the running sums on packed fp32 pairs (one instruction
+        // per two elements); the exponentials stay on the special-function unit
+        const uint64_t mm = f32x2(m_ref, m_ref);
+        uint64_t l2[2] = {f32x2(0.f, 0.f), f32x2(0.f, 0.f)};
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          float d0, d1;
+          unpack_f32x2(sub_f32x2(f32x2(x[2 * c], x[2 * c + 1]), mm), d0, d1);
+          const float p0 = fast_exp2(d0), p1 = fast_exp2(d1);
+          l2[c & 1] = add_f32x2(l2[c & 1], f32x2(p0, p1));
+          p[c] = pack_f16x2(p0, p1);
+        }
+        float a0, a1, b0, b1;
+        unpack_f32x2(l2[0], a0, a1);
+        unpack_f32x2(l2[1], b0, b1);
+        l += (a0 + a1) + (b0 + b1);
       }
-      l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
       tc::st32(tb + (j & 1) * 32 + lane_off, p);
       tc::wait_st();
       tc::fence_before();
