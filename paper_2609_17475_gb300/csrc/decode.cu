@@ -54,6 +54,40 @@ __device__ __forceinline__ uint32_t shr8(uint32_t w) { return __umulhi(w, 0x0100
 __device__ __forceinline__ uint32_t nib0(uint32_t w) { return w & 0x000F000Fu; }
 __device__ __forceinline__ uint32_t nib1(uint32_t w) { return w & 0x00F000F0u; }
 
+// packed fp32 pairs (f32x2 arithmetic: one instruction for two lanes of
+// work, each rounded as the scalar operation would be)
+struct f2 {
+  uint64_t v;
+};
+__device__ __forceinline__ f2 mk2(float lo, float hi) {
+  f2 r;
+  asm("mov.b64 %0, {%1, %2};\n" : "=l"(r.v) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void un2(f2 a, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;\n" : "=f"(lo), "=f"(hi) : "l"(a.v));
+}
+__device__ __forceinline__ f2 fma2(f2 a, f2 b, f2 c) {
+  f2 r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;\n" : "=l"(r.v) : "l"(a.v), "l"(b.v), "l"(c.v));
+  return r;
+}
+__device__ __forceinline__ f2 mul2(f2 a, f2 b) {
+  f2 r;
+  asm("mul.rn.f32x2 %0, %1, %2;\n" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+__device__ __forceinline__ f2 add2(f2 a, f2 b) {
+  f2 r;
+  asm("add.rn.f32x2 %0, %1, %2;\n" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+__device__ __forceinline__ f2 sub2(f2 a, f2 b) {
+  f2 r;
+  asm("sub.rn.f32x2 %0, %1, %2;\n" : "=l"(r.v) : "l"(a.v), "l"(b.v));
+  return r;
+}
+
 // bf16 MMA (m16n8k16, fp32 accumulate) for the bias terms
 __device__ __forceinline__ void mma_bf16(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
@@ -206,17 +240,17 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
       }
       mma_bf16_zc(t2, aa, ab, 0u, 0u, cc.bq, 0u);
     }
-    float t1[4] = {0.f, 0.f, 0.f, 0.f};
+    // t1 = sum_g scale_g acc_g on (head 2c, 2c+1) pairs
+    f2 t1a = mk2(0.f, 0.f), t1b = mk2(0.f, 0.f);
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
       const float sa = bf16lo_to_f32(wa[g]), sbv = bf16lo_to_f32(wb[g]);
-      t1[0] = fmaf(sa, acc[g][0], t1[0]);
-      t1[1] = fmaf(sa, acc[g][1], t1[1]);
-      t1[2] = fmaf(sbv, acc[g][2], t1[2]);
-      t1[3] = fmaf(sbv, acc[g][3], t1[3]);
+      t1a = fma2(mk2(sa, sa), mk2(acc[g][0], acc[g][1]), t1a);
+      t1b = fma2(mk2(sbv, sbv), mk2(acc[g][2], acc[g][3]), t1b);
     }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) sc[j][i] = fmaf(t1[i], cc.cA, t2[i] * cc.cB);
+    const f2 cA2 = mk2(cc.cA, cc.cA), cB2 = mk2(cc.cB, cc.cB);
+    un2(fma2(t1a, cA2, mul2(mk2(t2[0], t2[1]), cB2)), sc[j][0], sc[j][1]);
+    un2(fma2(t1b, cA2, mul2(mk2(t2[2], t2[3]), cB2)), sc[j][2], sc[j][3]);
     if constexpr (!FULL) {
       if (ta >= nv0) sc[j][0] = NEG_INF;
       if (ta >= nv1) sc[j][1] = NEG_INF;
@@ -261,18 +295,24 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
 #pragma unroll
   for (int j = 0; j < NJ; ++j) {
     if constexpr (FULL) {
-      p[j][0] = fast_exp2(sc[j][0] - st.m0);
-      p[j][1] = fast_exp2(sc[j][1] - st.m1);
-      p[j][2] = fast_exp2(sc[j][2] - st.m0);
-      p[j][3] = fast_exp2(sc[j][3] - st.m1);
+      const f2 m2 = mk2(st.m0, st.m1);
+      float d0, d1, d2, d3;
+      un2(sub2(mk2(sc[j][0], sc[j][1]), m2), d0, d1);
+      un2(sub2(mk2(sc[j][2], sc[j][3]), m2), d2, d3);
+      p[j][0] = fast_exp2(d0);
+      p[j][1] = fast_exp2(d1);
+      p[j][2] = fast_exp2(d2);
+      p[j][3] = fast_exp2(d3);
     } else {
       p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
       p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
       p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
       p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
     }
-    st.l0 += p[j][0] + p[j][2];
-    st.l1 += p[j][1] + p[j][3];
+    float l0n, l1n;
+    un2(add2(mk2(st.l0, st.l1), add2(mk2(p[j][0], p[j][1]), mk2(p[j][2], p[j][3]))), l0n, l1n);
+    st.l0 = l0n;
+    st.l1 = l1n;
   }
 
   // ---- PV ---------------------------------------------------------------
@@ -318,8 +358,11 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
         if (!va) sva = 0.f;
         if (!vb) svb = 0.f;
       }
-      const uint32_t b0 = movm_t(pack_f16x2(sva * p[j][0], sva * p[j][1]));
-      const uint32_t b1 = movm_t(pack_f16x2(svb * p[j][2], svb * p[j][3]));
+      float b00, b01, b10, b11;
+      un2(mul2(mk2(sva, sva), mk2(p[j][0], p[j][1])), b00, b01);
+      un2(mul2(mk2(svb, svb), mk2(p[j][2], p[j][3])), b10, b11);
+      const uint32_t b0 = movm_t(pack_f16x2(b00, b01));
+      const uint32_t b1 = movm_t(pack_f16x2(b10, b11));
       uint32_t v0, v1, v2, v3;
       ldsm_x4_t(v0, v1, v2, v3, vc + cc.koff[g] + 16 * j * CB);
       const uint32_t h0 = shr8(v0), h1 = shr8(v1), h2 = shr8(v2), h3 = shr8(v3);
