@@ -35,7 +35,7 @@ struct DecodeArgs {
   float scale_log2;    // softmax_scale * log2(e)
   int32_t B;           // requests
   int32_t L;           // query tokens per request (1: decode; 2-4: packed verifier)
-  int32_t NT;          // CTAs per KV head, each for 8 of its G * L (token, head) rows
+  int32_t NT;          // n-tiles per KV head: ceil(G * L / 8) groups of 8 (token, head) rows
   int32_t HqL;         // L * Hq: rows of q, out and the partials per request
   int32_t balanced;    // 1: batch split plan (balanced_plan), partial rows by global split
   int32_t span;        // 1: batch span plan (span_find), partial rows (piece + request)
@@ -209,5 +209,10 @@ __device__ __forceinline__ uint32_t swz(int t, int ch) {
 int sm_count();
 // Merge phase for D = 128 or 256 (launched after a split kernel on `stream`).
 int launch_decode_merge(const DecodeArgs& a, int D, int B, cudaStream_t stream);
+// Packed verifier for NT >= 2 n-tiles per KV head (verify.cu): CTAs per KV
+// head and split, and the split launch (+ merge).
+int verify_pair_ctas(int NT);
+int launch_verify_pairs(const CUtensorMap& tmap, const DecodeArgs& a, int D, int B,
+                        cudaStream_t stream);
 
 }  // namespace jfkv

@@ -230,8 +230,13 @@ def test_split_planners_on_a_152_sm_gpu():
     assert B.default_num_splits(1, 4, num_sms=152) == 76
     assert B.default_num_splits(1, 4, num_sms=152, format=B.JF_FMT_TQ4) == 38
     assert B.default_num_splits(2, 4, num_sms=152) == 38 + 2      # batch: even share + 2
-    # verifier: ceil(G q_len / 8) CTAs per split (24 / 4 heads: 2, 3, 3)
-    assert [B.default_verify_splits(1, L, 24, 4, num_sms=152) for L in (2, 3, 4)] == [38, 25, 25]
+    # verifier (affine): 24 / 4 heads give 2, 3, 3 row groups, all in one
+    # 8-warp CTA per split and KV head, one CTA per SM; 8 / 4 heads at q_len 2
+    # fit one group (6-warp CTAs, two per SM); 32 / 2 heads at q_len 4 give
+    # 8 groups, 3 CTAs per split
+    assert [B.default_verify_splits(1, L, 24, 4, num_sms=152) for L in (2, 3, 4)] == [38, 38, 38]
+    assert B.default_verify_splits(1, 2, 8, 4, num_sms=152) == 76
+    assert B.default_verify_splits(1, 4, 32, 2, num_sms=152) == 25
     assert [B.default_verify_splits(1, L, 24, 4, num_sms=152, format=B.JF_FMT_TQ4)
             for L in (2, 3, 4)] == [19, 12, 12]
     # prefill history splits (24 / 4 heads, 42 queries per CTA pair)

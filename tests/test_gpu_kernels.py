@@ -253,11 +253,14 @@ def test_fused_append_decode_reports_bad_page_id():
 
 
 @pytest.mark.parametrize("Hq,Hkv,D,P,ctx,L,splits", [
-    (24, 4, 256, 256, [5000], 2, None),          # 12 (token, head) rows: 2 CTAs per split
+    (24, 4, 256, 256, [5000], 2, None),          # 12 (token, head) rows: 2 row groups, one CTA
     (24, 4, 256, 128, [3000, 777], 4, None),     # 24 rows, batch plan
     (24, 4, 256, 256, [4096], 3, 1),             # one split: rows written directly
     (8, 2, 128, 64, [3, 65, 300, 2001], 3, 5),   # a context equal to q_len, partial pages
-    (16, 2, 256, 64, [1000], 4, 7),              # G = 8: 32 rows
+    (16, 2, 256, 64, [1000], 4, 7),              # G = 8: 32 rows, two CTAs (3 + 1 groups)
+    (14, 2, 256, 64, [2500], 4, 6),              # G = 7: 28 rows, two CTAs (3 + 1 groups)
+    (12, 2, 128, 128, [9000], 4, 1),             # D = 128, 3 groups, 70 chunks per warp pair
+    (8, 4, 128, 64, [700, 31], 4, 3),            # 8 rows: one group (the 6-warp kernel)
 ])
 def test_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
     """Token i of each request attends positions up to ctx - L + i; the oracle
@@ -463,6 +466,45 @@ def test_decode_full_window_256k_sampled_heads():
                 o1 = L1.codes_offset(kind, 0, 0)
                 n = geo.page_size * L4.code_bytes
                 assert np.array_equal(gp[page, o4:o4 + n], opool[page, o1:o1 + n])
+
+
+@pytest.mark.parametrize("L", [2, 4])
+def test_verifier_full_window_256k_sampled_heads(L):
+    """The packed verifier on the 256K full-window workload (24/4/256, 1,024
+    pages in a random physical order) in the launch shape the benchmark uses
+    (default split cap, warp pairs sharing the unpacking); KV heads 0 and 3
+    against the oracle's causal chunk attention of the L tokens."""
+    from paper_2609_17475_gb300 import synth
+    w = synth.WORKLOADS["full_window_256k"]
+    geo = w["geometry"]
+    ctx = w["context_lens"][0]
+    gen = synth.generator(w["seed"] + 17)
+    channels = synth.outlier_channels(gen, geo.num_kv_heads, geo.head_dim)
+    k, v = synth.kv_rows(gen, ctx, geo.num_kv_heads, geo.head_dim, channels)
+    pt, npages = synth.page_tables(gen, [ctx], geo.page_size)
+    q = synth.normal_bf16(gen, (1, L, geo.num_q_heads, geo.head_dim))
+    req, pos = synth.append_rows_for([ctx])
+    pool = jf.KVPool.allocate(npages, geo.page_size, geo.num_kv_heads, geo.head_dim, device=DEV)
+    err = torch.zeros(1, dtype=torch.int32, device=DEV)
+    jf.jf_kv_quantize_append(pool, pt.to(DEV), req.to(DEV), pos.to(DEV), k.to(DEV), v.to(DEV), err)
+    Hq, Hkv, D = geo.num_q_heads, geo.num_kv_heads, geo.head_dim
+    splits = jf.default_verify_splits(1, L, Hq, Hkv)
+    ws = jf.verify_workspace(1, L, Hq, Hkv, D, splits, device=DEV)
+    out = torch.empty(1, L, Hq, D, dtype=torch.bfloat16, device=DEV)
+    scale = 1 / math.sqrt(D)
+    jf.jf_paged_verify_attn(pool, pt.to(DEV), torch.tensor([ctx], dtype=torch.int32, device=DEV),
+                            q.to(DEV), scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0 and jf.workspace_status(ws) == 0
+    G = geo.group
+    for kvh in (0, 3):
+        L1 = OA.PoolLayout(1, geo.page_size, D)
+        opool = OA.new_pool(L1, npages)
+        OA.append(opool, L1, pt.numpy(), req.numpy(), pos.numpy(),
+                  bits(k[:, kvh:kvh + 1]), bits(v[:, kvh:kvh + 1]))
+        ref = OT.prefill_chunk(opool, L1, pt[0].numpy(), bits(q[0, :, kvh * G:(kvh + 1) * G]),
+                               ctx - L, scale)
+        assert_attention_close(out[0, :, kvh * G:(kvh + 1) * G], ref)
 
 
 # --------------------------------------------------------------------------
