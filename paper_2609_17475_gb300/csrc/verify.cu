@@ -154,25 +154,17 @@ __device__ __forceinline__ void pair_qk(float (&sc)[NTC][2][4], const PairCtx<D,
       const uint32_t a20 = nib0(w2), a21 = nib0(w3), a22 = nib1(w2), a23 = nib1(w3);
       const uint32_t a30 = nib0(h2), a31 = nib0(h3), a32 = nib1(h2), a33 = nib1(h3);
       const float sa = bf16lo_to_f32(wa[gg]), sbv = bf16lo_to_f32(wb[gg]);
-      // the n-tiles' MMA chains interleaved (the MMAs issue in source order)
-      float acc[NTC][4];
-      uint4 q[NTC];
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) q[t] = cc.qf[((t * NG + gg) * 2) * 32];
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) mma_f16_zc(acc[t], a00, a01, a02, a03, q[t].x, q[t].y);
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) mma_f16(acc[t], a10, a11, a12, a13, q[t].z, q[t].w);
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) q[t] = cc.qf[((t * NG + gg) * 2 + 1) * 32];
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) mma_f16(acc[t], a20, a21, a22, a23, q[t].x, q[t].y);
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) mma_f16(acc[t], a30, a31, a32, a33, q[t].z, q[t].w);
 #pragma unroll
       for (int t = 0; t < NTC; ++t) {
-        t1a[t] = fma2(mk2(sa, sa), mk2(acc[t][0], acc[t][1]), t1a[t]);
-        t1b[t] = fma2(mk2(sbv, sbv), mk2(acc[t][2], acc[t][3]), t1b[t]);
+        const uint4 qa = cc.qf[((t * NG + gg) * 2) * 32];
+        const uint4 qb = cc.qf[((t * NG + gg) * 2 + 1) * 32];
+        float acc[4];
+        mma_f16_zc(acc, a00, a01, a02, a03, qa.x, qa.y);
+        mma_f16(acc, a10, a11, a12, a13, qa.z, qa.w);
+        mma_f16(acc, a20, a21, a22, a23, qb.x, qb.y);
+        mma_f16(acc, a30, a31, a32, a33, qb.z, qb.w);
+        t1a[t] = fma2(mk2(sa, sa), mk2(acc[0], acc[1]), t1a[t]);
+        t1b[t] = fma2(mk2(sbv, sbv), mk2(acc[2], acc[3]), t1b[t]);
       }
     }
     // bias term over this warp's groups: A rows = positions, k-slots as in
@@ -188,14 +180,13 @@ __device__ __forceinline__ void pair_qk(float (&sc)[NTC][2][4], const PairCtx<D,
       ab = (cc.c < 2) ? (cc.h ? hi_halves(0u, wb[0]) : hi_halves(wb[0], 0u)) : 0u;
     }
     const f2 cB2 = mk2(cc.cB, cc.cB);
-    float t2[NTC][4];
-#pragma unroll
-    for (int t = 0; t < NTC; ++t) mma_bf16_zc(t2[t], aa, ab, 0u, 0u, cc.bq[t * 64], 0u);
 #pragma unroll
     for (int t = 0; t < NTC; ++t) {
+      float t2[4];
+      mma_bf16_zc(t2, aa, ab, 0u, 0u, cc.bq[t * 64], 0u);
       const f2 cA2 = mk2(cc.cA[t], cc.cA[t]);
-      un2(fma2(t1a[t], cA2, mul2(mk2(t2[t][0], t2[t][1]), cB2)), sc[t][j][0], sc[t][j][1]);
-      un2(fma2(t1b[t], cA2, mul2(mk2(t2[t][2], t2[t][3]), cB2)), sc[t][j][2], sc[t][j][3]);
+      un2(fma2(t1a[t], cA2, mul2(mk2(t2[0], t2[1]), cB2)), sc[t][j][0], sc[t][j][1]);
+      un2(fma2(t1b[t], cA2, mul2(mk2(t2[2], t2[3]), cB2)), sc[t][j][2], sc[t][j][3]);
     }
   }
 }
@@ -306,14 +297,12 @@ __device__ __forceinline__ void pair_softmax_pv(PairState<D / 128> (&st)[NTC],
         a0 = hi_halves(x0, x1);
         a2 = hi_halves(x2, x3);
       }
-      uint32_t pb[NTC][2];
 #pragma unroll
       for (int t = 0; t < NTC; ++t) {
-        pb[t][0] = movm_t(pack_bf16x2(p[t][j][0], p[t][j][1]));
-        pb[t][1] = movm_t(pack_bf16x2(p[t][j][2], p[t][j][3]));
+        const uint32_t pb0 = movm_t(pack_bf16x2(p[t][j][0], p[t][j][1]));
+        const uint32_t pb1 = movm_t(pack_bf16x2(p[t][j][2], p[t][j][3]));
+        mma_bf16(st[t].Bs, a0, 0u, a2, 0u, pb0, pb1);
       }
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) mma_bf16(st[t].Bs, a0, 0u, a2, 0u, pb[t][0], pb[t][1]);
     }
 #pragma unroll
     for (int gg = 0; gg < NGH; ++gg) {
@@ -331,21 +320,17 @@ __device__ __forceinline__ void pair_softmax_pv(PairState<D / 128> (&st)[NTC],
       const uint32_t e20 = nib0(h0), e21 = nib0(h2), e22 = nib0(h1), e23 = nib0(h3);
       const uint32_t e30 = nib1(h0), e31 = nib1(h2), e32 = nib1(h1), e33 = nib1(h3);
       const f2 sa2 = mk2(sva, sva), sb2 = mk2(svb, svb);
-      uint32_t bo[NTC][2];
 #pragma unroll
       for (int t = 0; t < NTC; ++t) {
         float b00, b01, b10, b11;
         un2(mul2(sa2, mk2(p[t][j][0], p[t][j][1])), b00, b01);
         un2(mul2(sb2, mk2(p[t][j][2], p[t][j][3])), b10, b11);
-        bo[t][0] = movm_t(pack_f16x2(b00, b01));
-        bo[t][1] = movm_t(pack_f16x2(b10, b11));
-      }
-#pragma unroll
-      for (int t = 0; t < NTC; ++t) {
-        mma_f16(st[t].O[gg][0], e00, e01, e02, e03, bo[t][0], bo[t][1]);
-        mma_f16(st[t].O[gg][1], e10, e11, e12, e13, bo[t][0], bo[t][1]);
-        mma_f16(st[t].O[gg][2], e20, e21, e22, e23, bo[t][0], bo[t][1]);
-        mma_f16(st[t].O[gg][3], e30, e31, e32, e33, bo[t][0], bo[t][1]);
+        const uint32_t b0 = movm_t(pack_f16x2(b00, b01));
+        const uint32_t b1 = movm_t(pack_f16x2(b10, b11));
+        mma_f16(st[t].O[gg][0], e00, e01, e02, e03, b0, b1);
+        mma_f16(st[t].O[gg][1], e10, e11, e12, e13, b0, b1);
+        mma_f16(st[t].O[gg][2], e20, e21, e22, e23, b0, b1);
+        mma_f16(st[t].O[gg][3], e30, e31, e32, e33, b0, b1);
       }
     }
   }
