@@ -380,15 +380,15 @@ def default_verify_splits(batch: int, q_len: int, num_q_heads: int, num_kv_heads
                           num_sms: Optional[int] = None) -> int:
     """Split cap for the verifier, one full wave of split CTAs.  The G * q_len
     (token, head) rows of a KV head form nt = ceil(G * q_len / 8) groups of 8.
-    Affine pools: with nt >= 2 each split of a KV head runs ceil(nt / 3) CTAs
-    of 8 warps, one per SM (warp pairs sharing the unpacking); with nt = 1 one
-    6-warp CTA, two per SM.  TQ4 pools run nt CTAs per split, one per SM."""
+    With nt >= 2 each split of a KV head runs ceil(nt / 3) CTAs, one per SM
+    (warp pairs sharing the unpacking or the centroid lookups, either
+    format); with nt = 1 one CTA, two per SM (affine) or one (TQ4)."""
     nt = -(-(num_q_heads // num_kv_heads) * q_len // 8)
     sms = _num_sms(device, num_sms)
-    if format == JF_FMT_TQ4:
-        slots, per_head = sms, nt
-    elif nt >= 2:
+    if nt >= 2:
         slots, per_head = sms, -(-nt // min(nt, 3))
+    elif format == JF_FMT_TQ4:
+        slots, per_head = sms, 1
     else:
         slots, per_head = 2 * sms, 1
     per = slots // (batch * num_kv_heads * per_head)   # one full wave

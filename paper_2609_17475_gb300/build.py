@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libjfkv.so")
 SOURCES = ["api.cu", "append.cu", "checkpoint.cu", "decode.cu", "prefill.cu", "selftest.cu",
-           "tq4.cu", "verify.cu"]
+           "tq4.cu", "tq4_verify.cu", "verify.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

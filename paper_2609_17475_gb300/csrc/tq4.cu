@@ -954,6 +954,10 @@ static int launch_tq4_split_any(const cudaLaunchConfig_t& cfg, const CUtensorMap
   return launch_tq4_split<D, false, false>(cfg, tmap, a, prm);
 }
 
+// packed verifier with more than 8 rows per KV head (tq4_verify.cu)
+int launch_tq4_verify_pairs(const CUtensorMap& tmap, const DecodeArgs& a, const Tq4Params& prm,
+                            int D, int B, cudaStream_t stream);
+
 int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& tmap,
                       const Tq4Params& prm, const int32_t* page_table, int32_t pt_stride,
                       const int32_t* context_lens, int32_t batch, const void* q, int32_t Hq,
@@ -993,6 +997,20 @@ int launch_tq4_decode(const Geom& g, const jf_kv_pool& pool, const CUtensorMap& 
   a.B = batch;
   a.balanced = (batch > 1 && batch <= 1024 && num_splits > 1) ? 1 : 0;
   a.budget = 1;
+  if (q_len > 1 && a.NT >= 2) {
+    // warp pairs sharing the centroid lookups: ceil(NT / 3) CTAs per KV head
+    // and split, one CTA per SM
+    const int ntc = a.NT < 3 ? a.NT : 3;
+    const int per_head = g.Hkv * ((a.NT + ntc - 1) / ntc);
+    const int vslots = sm_count() / per_head > 1 ? sm_count() / per_head : 1;
+    a.plan_splits = num_splits < vslots ? num_splits : vslots;
+    if (a.balanced) {
+      const int64_t fit = (int64_t)batch * num_splits - batch;
+      const int64_t cap = fit < vslots ? fit : vslots;
+      a.budget = (int)(cap - batch / 2 > 1 ? cap - batch / 2 : 1);
+    }
+    return launch_tq4_verify_pairs(tmap, a, prm, g.D, batch, stream);
+  }
   if (a.balanced) {   // one CTA per SM in all
     const int slots = (sm_count() + g.Hkv * a.NT - 1) / (g.Hkv * a.NT);
     const int64_t fit = (int64_t)batch * num_splits - batch;

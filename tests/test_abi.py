@@ -237,8 +237,10 @@ def test_split_planners_on_a_152_sm_gpu():
     assert [B.default_verify_splits(1, L, 24, 4, num_sms=152) for L in (2, 3, 4)] == [38, 38, 38]
     assert B.default_verify_splits(1, 2, 8, 4, num_sms=152) == 76
     assert B.default_verify_splits(1, 4, 32, 2, num_sms=152) == 25
+    # TQ4 verifier: the same warp-pair CTAs (one per SM) for two or more groups
     assert [B.default_verify_splits(1, L, 24, 4, num_sms=152, format=B.JF_FMT_TQ4)
-            for L in (2, 3, 4)] == [19, 12, 12]
+            for L in (2, 3, 4)] == [38, 38, 38]
+    assert B.default_verify_splits(1, 2, 8, 4, num_sms=152, format=B.JF_FMT_TQ4) == 38
     # prefill history splits (24 / 4 heads, 42 queries per CTA pair)
     ps = lambda qs, cl: B.default_prefill_splits(qs, cl, 24, 4, num_sms=152)
     assert ps([32704], [64]) == 9          # 4 pairs walking 512 tiles each

@@ -282,6 +282,9 @@ def test_tq4_no_workspace_decode_is_rejected():
     (24, 4, 256, 128, [3000, 40], 4, None),       # G * L = 24: 3 n-tiles, batch plan
     (8, 2, 128, 64, [700], 3, 5),
     (16, 2, 256, 256, [2100, 4], 4, 3),           # G * L = 32; a context of exactly q_len
+    (24, 4, 256, 64, [9000], 3, 1),               # one split written directly, 70 chunks per pair
+    (14, 2, 128, 128, [6000], 4, 1),              # G = 7, D = 128: 28 rows, two CTAs (3 + 1 groups)
+    (8, 4, 128, 64, [500, 33], 4, 2),             # 8 rows: one group (one CTA per n-tile kernel)
 ])
 def test_tq4_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
     case = make_case(900 + sum(ctx) + L, Hq, Hkv, D, P, ctx)
