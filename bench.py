@@ -274,33 +274,72 @@ def run_ours(args, world, rank, local):
     app_ms = None
 
     # ---- end-to-end through the public API with host buffers ----
-    qh = q.cpu().pin_memory()
-    kh = knew.cpu().pin_memory()
-    vh = vnew.cpu().pin_memory()
-    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    qd, kd, vd = torch.empty_like(q), torch.empty_like(knew), torch.empty_like(vnew)
+    # Every step copies its inputs (q, new K/V rows of all layers) from pinned
+    # host memory and reads its outputs back, as a serving loop would: two
+    # sets of device buffers, the copies of step i + 1 and the read-back of
+    # step i - 1 on a copy stream overlapping step i's eager API calls on the
+    # compute stream.  The timed region runs from before the first step's
+    # copies to the end of the last step's read-back.
+    nb = 2
+    qh = [q.cpu().pin_memory() for _ in range(nb)]
+    kh = [knew.cpu().pin_memory() for _ in range(nb)]
+    vh = [vnew.cpu().pin_memory() for _ in range(nb)]
+    oh = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(nb)]
+    qd = [torch.empty_like(q) for _ in range(nb)]
+    kd = [torch.empty_like(knew) for _ in range(nb)]
+    vd = [torch.empty_like(vnew) for _ in range(nb)]
+    od = [torch.empty_like(out) for _ in range(nb)]
+    cstream = torch.cuda.Stream(device=dev)
     e2e_steps = max(3, min(args.steps, 50))
 
-    def e2e_step():
-        qd.copy_(qh, non_blocking=True)
-        kd.copy_(kh, non_blocking=True)
-        vd.copy_(vh, non_blocking=True)
-        step(qd, kd, vd, out)
-        oh.copy_(out, non_blocking=True)
+    def e2e_run(n):
+        loaded = [torch.cuda.Event() for _ in range(n)]
+        computed = [torch.cuda.Event() for _ in range(n)]
+        read = [torch.cuda.Event() for _ in range(n)]
 
-    with torch.cuda.stream(stream):
-        for _ in range(2):
-            e2e_step()
-        stream.synchronize()
-        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        f0.record(stream)
-        for _ in range(e2e_steps):
-            e2e_step()
-        f1.record(stream)
-    stream.synchronize()
+        def load(i):
+            j = i % nb
+            with torch.cuda.stream(cstream):
+                if i >= nb:   # step i - nb has consumed these inputs
+                    cstream.wait_event(computed[i - nb])
+                qd[j].copy_(qh[j], non_blocking=True)
+                kd[j].copy_(kh[j], non_blocking=True)
+                vd[j].copy_(vh[j], non_blocking=True)
+                loaded[i].record(cstream)
+
+        def readback(i):
+            j = i % nb
+            with torch.cuda.stream(cstream):
+                cstream.wait_event(computed[i])
+                oh[j].copy_(od[j], non_blocking=True)
+                read[i].record(cstream)
+
+        load(0)
+        for i in range(n):
+            if i + 1 < n:
+                load(i + 1)
+            j = i % nb
+            with torch.cuda.stream(stream):
+                stream.wait_event(loaded[i])
+                if i >= nb:   # the read-back of step i - nb has left od[j]
+                    stream.wait_event(read[i - nb])
+                step(qd[j], kd[j], vd[j], od[j])
+                computed[i].record(stream)
+            if i >= 1:
+                readback(i - 1)
+        readback(n - 1)
+
+    e2e_run(2)
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(cstream)
+    stream.wait_event(f0)
+    e2e_run(e2e_steps)
+    f1.record(cstream)   # after the last read-back, which follows every step
+    torch.cuda.synchronize()
     e2e_ms = max_over_ranks(f0.elapsed_time(f1) / e2e_steps, world, dev)
-    h2d = qh.numel() * 2 + kh.numel() * 2 + vh.numel() * 2
-    d2h = oh.numel() * 2
+    h2d = qh[0].numel() * 2 + kh[0].numel() * 2 + vh[0].numel() * 2
+    d2h = oh[0].numel() * 2
     torch.cuda.synchronize()
     assert int(err.item()) == 0 and jf.workspace_status(ws) == 0, "device error flag set"
 
