@@ -465,7 +465,9 @@ tq4_verify_pair_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArg
   const int bar_id = 1 + pr;
   int done = 0;
   bool gave_up = false;
-#pragma unroll 1
+  // two n-tiles: unrolled by 2 (the exchange buffer's parity a constant)
+  constexpr int UNR = NTC <= 2 ? 2 : 1;
+#pragma unroll UNR
   for (int it = 0; it < my_n; ++it) {
     const int s = it % VST;
     const uint32_t par = (it / VST) & 1;
