@@ -369,7 +369,8 @@ def test_tq4_fused_append_decode_equals_append_then_decode(Hq, Hkv, D, P, ctx, s
 def test_tq4_decode_full_window_256k_one_head():
     """The 256K full-window workload (24/4/256, 1,024 pages in a random physical
     order, K outlier channels) in TQ4 at full size and in the benchmark's launch
-    shape; KV head 2 checked against the oracle, bytes of sampled pages too."""
+    shape; KV head 2 checked against the oracle, bytes of sampled pages too,
+    then the packed verifier (4 tokens, warp pairs) on the same pages."""
     w = synth.WORKLOADS["full_window_256k"]
     geo = w["geometry"]
     ctx = w["context_lens"][0]
@@ -409,6 +410,21 @@ def test_tq4_decode_full_window_256k_one_head():
             o4, o1 = L4.norm_offset(kind, kvh, 0), L1.norm_offset(kind, 0, 0)
             assert np.array_equal(gp[page, o4:o4 + 2 * geo.page_size],
                                   opool[page, o1:o1 + 2 * geo.page_size])
+    # packed verifier: tokens ctx - 4 .. ctx - 1 against the oracle's causal chunk
+    Lq = 4
+    qv = synth.normal_bf16(gen, (1, Lq, geo.num_q_heads, geo.head_dim))
+    sv = jf.default_verify_splits(1, Lq, geo.num_q_heads, geo.num_kv_heads,
+                                  format=jf.JF_FMT_TQ4)
+    wv = jf.verify_workspace(1, Lq, geo.num_q_heads, geo.num_kv_heads, geo.head_dim, sv,
+                             device=DEV)
+    ov = torch.empty(1, Lq, geo.num_q_heads, geo.head_dim, dtype=torch.bfloat16, device=DEV)
+    jf.jf_paged_verify_attn(pool, pt.to(DEV), torch.tensor([ctx], dtype=torch.int32, device=DEV),
+                            qv.to(DEV), scale, ov, wv, sv)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(wv) == 0
+    ref_v = OT.prefill_chunk(opool, L1, pt[0].numpy(), bits(qv[0, :, kvh * G:(kvh + 1) * G]),
+                             ctx - Lq, scale)
+    assert_attention_close(ov[0, :, kvh * G:(kvh + 1) * G], ref_v)
 
 
 def test_tq4_prefill_wave_balanced_chunk():
