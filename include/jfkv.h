@@ -224,8 +224,14 @@ int jf_paged_decode_attn(const jf_kv_pool* pool, const int32_t* page_table, int3
  * context_lens[b] - q_len + i (i < q_len), already appended to the pool;
  * token i attends positions [0, context_lens[b] - q_len + i] causally:
  *   out[b, i, h, :] = sum_t softmax_t(scale * <q[b, i, h], K_t>) V_t.
- * The page reads are shared by the tokens: the split CTAs of a KV head each
- * take 8 of its G * q_len (token, head) rows over the same chunk range.
+ * The page reads are shared by the tokens.  With more than 8 (token, head)
+ * rows per KV head (G * q_len > 8) a split CTA holds up to 24 of them and its
+ * warps work in pairs on each 32-position chunk, each warp for half of D, so
+ * every 4-bit code (or TQ4 index) is unpacked once per chunk; more than 24
+ * rows take ceil(G * q_len / 24) CTAs per split over the same chunk range.
+ * A single request then uses at most one split per SM and CTA of a KV head
+ * (min(num_splits, SMs / (Hkv * CTAs)) splits; the workspace row stride
+ * stays num_splits).  With 8 rows or fewer, one CTA per split holds them.
  *   q, out        bf16 [batch, q_len, Hq, D]
  *   q_len         1..4 (1 is plain decode)
  *   context_lens  int32 [batch], >= q_len for every request that has tokens
