@@ -336,7 +336,8 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
   uint64_t* bars = reinterpret_cast<uint64_t*>(sbuf + L::SB_BYTES + L::QF_BYTES);
 
   // decode: one CTA per KV head holds its G query heads; verifier: NT CTAs
-  // each hold 8 of its G * L (token, head) rows
+  // each hold 8 of its G * L (token, head) rows (launched for NT = 1; more
+  // rows go to the warp-pair kernel of verify.cu)
   const int kvh = VER ? (int)blockIdx.y / a.NT : (int)blockIdx.y;
   const int nt = VER ? (int)blockIdx.y % a.NT : 0;
   const int rows = VER ? min(8, a.G * a.L - 8 * nt) : a.G;
@@ -1508,9 +1509,10 @@ static int launch_decode_t(const CUtensorMap& tmap, const DecodeArgs& a, int B,
 // priority and ends its share ~4 us (of ~50) before the other, so decode runs
 // one 12-warp CTA per SM: a single request with per-request splits, a batch
 // with the span plan (equal pieces, so the longer pieces of 12-warp CTAs
-// leave no unevenness).  The packed verifier keeps 6-warp CTAs (measured
-// faster) and the batch plan of whole-request pieces; many requests that do
-// not fit one wave of 12-warp CTAs use 6-warp CTAs.
+// leave no unevenness).  The packed verifier with at most 8 rows per KV head
+// (one n-tile) keeps 6-warp CTAs (measured faster) and the batch plan of
+// whole-request pieces (more rows go to the warp-pair kernel, verify.cu);
+// many requests that do not fit one wave of 12-warp CTAs use 6-warp CTAs.
 static int decode_warps(int batch, int num_splits, int Hkv, int NT) {
   if (NT > 1) return 6;
   if (batch > 1 && batch <= BAL_MAX_B && num_splits > 1) return 12;   // span plan

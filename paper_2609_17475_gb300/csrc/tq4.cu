@@ -578,8 +578,9 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
 }
 
 // VER: packed verifier (a.L > 1 query tokens, per-row causal limits; each CTA
-// holds 8 of the KV head's G * L (token, head) rows); otherwise decode.  APP:
-// the step's new K/V row is appended first (a.knew, a.vnew).
+// holds 8 of the KV head's G * L (token, head) rows; launched for at most 8
+// rows, more go to the warp-pair kernel of tq4_verify.cu); otherwise decode.
+// APP: the step's new K/V row is appended first (a.knew, a.vnew).
 template <int D, bool VER, bool APP>
 __global__ void __launch_bounds__(TQ_WARPS * 32, 1)
 tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
