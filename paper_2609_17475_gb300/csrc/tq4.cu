@@ -446,13 +446,14 @@ __device__ __forceinline__ float h2f(const uint8_t* p) {
   return __half2float(__ushort_as_half(*reinterpret_cast<const uint16_t*>(p)));
 }
 
-// One 32-position chunk; positions >= nvalid get -inf logits and zero weights
-// (their bytes are never trusted), and the rows of this thread's columns 2c
-// and 2c+1 see only positions < nv0 and < nv1 (the verifier's causal limits;
-// both are nvalid for a single query).  The masks are plain selects, so full and
-// partial chunks share one body (the body is large: one copy keeps it in the
-// instruction cache).
-template <int D, bool VER>
+// One 32-position chunk.  FULL: every position valid and visible to every
+// row, no masks.  Otherwise positions >= nvalid get -inf logits and zero
+// weights (their bytes are never trusted), and the rows of this thread's
+// columns 2c and 2c+1 see only positions < nv0 and < nv1 (the verifier's
+// causal limits; both are nvalid for a single query), as plain selects.  The
+// chunk loop stays rolled, so the kernel holds two copies of the body (four,
+// unrolled by the ring depth, had missed the instruction cache).
+template <int D, bool VER, bool FULL>
 __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[D / 32][2][2],
                                           uint32_t kc, const uint8_t* kn, uint32_t lut_lane,
                                           const uint32_t (&koff)[D / 64], float cS, int r,
@@ -488,7 +489,12 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
     }
     const int ta = 16 * j + r, tb = ta + 8;
     const float na = h2f(kn + 2 * ta) * cS, nb = h2f(kn + 2 * tb) * cS;
-    if constexpr (VER) {
+    if constexpr (FULL) {
+      sc[j][0] = acc[0] * na;
+      sc[j][1] = acc[1] * na;
+      sc[j][2] = acc[2] * nb;
+      sc[j][3] = acc[3] * nb;
+    } else if constexpr (VER) {
       sc[j][0] = (ta < nv0) ? acc[0] * na : NEG_INF;
       sc[j][1] = (ta < nv1) ? acc[1] * na : NEG_INF;
       sc[j][2] = (tb < nv0) ? acc[2] * nb : NEG_INF;
@@ -533,10 +539,17 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
   float p[NJ][4];
 #pragma unroll
   for (int j = 0; j < NJ; ++j) {
-    p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
-    p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
-    p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
-    p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
+    if constexpr (FULL) {
+      p[j][0] = fast_exp2(sc[j][0] - st.m0);
+      p[j][1] = fast_exp2(sc[j][1] - st.m1);
+      p[j][2] = fast_exp2(sc[j][2] - st.m0);
+      p[j][3] = fast_exp2(sc[j][3] - st.m1);
+    } else {
+      p[j][0] = (sc[j][0] == NEG_INF) ? 0.f : fast_exp2(sc[j][0] - st.m0);
+      p[j][1] = (sc[j][1] == NEG_INF) ? 0.f : fast_exp2(sc[j][1] - st.m1);
+      p[j][2] = (sc[j][2] == NEG_INF) ? 0.f : fast_exp2(sc[j][2] - st.m0);
+      p[j][3] = (sc[j][3] == NEG_INF) ? 0.f : fast_exp2(sc[j][3] - st.m1);
+    }
     st.l0 += p[j][0] + p[j][2];
     st.l1 += p[j][1] + p[j][3];
   }
@@ -545,8 +558,8 @@ __device__ __forceinline__ void tq4_chunk(Tq4State<D>& st, const uint32_t (&bq)[
 #pragma unroll
   for (int j = 0; j < NJ; ++j) {
     const int ta = 16 * j + r, tb = ta + 8;
-    const float wa = (ta < nvalid) ? h2f(vn + 2 * ta) * 0.00390625f : 0.f;
-    const float wb = (tb < nvalid) ? h2f(vn + 2 * tb) * 0.00390625f : 0.f;
+    const float wa = (FULL || ta < nvalid) ? h2f(vn + 2 * ta) * 0.00390625f : 0.f;
+    const float wb = (FULL || tb < nvalid) ? h2f(vn + 2 * tb) * 0.00390625f : 0.f;
     const uint32_t b0 = movm_t(pack_f16x2(wa * p[j][0], wa * p[j][1]));
     const uint32_t b1 = movm_t(pack_f16x2(wb * p[j][2], wb * p[j][3]));
 #pragma unroll
@@ -802,7 +815,9 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     lim0 = min(ctx, ctx_all + (8 * nt + 2 * c) / a.G);
     lim1 = min(ctx, ctx_all + (8 * nt + 2 * c + 1) / a.G);
   }
+  const int ctx_full = VER ? ctx - a.L + 1 : ctx;   // chunks below it: no masks
   int done = 0;
+#pragma unroll 1
   for (int it = 0; it < my_n; ++it) {
     const int s = it % TQ_STAGES;
     const uint32_t par = (it / TQ_STAGES) & 1;
@@ -815,9 +830,13 @@ tq4_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a,
     const int tokbase = chunk_of(it) * DTOK;
     const uint32_t kc = smem_u32(codes + (warp * TQ_STAGES + s) * 2 * L::CODE_BUF);
     const uint8_t* kn = norms + (warp * TQ_STAGES + s) * 2 * L::NORM_BUF;
-    const int nv = ok ? min(ctx - tokbase, DTOK) : 0;
-    tq4_chunk<D, VER>(st, bq, kc, kn, lut_lane, koff, cS, r, nv,
-                      ok ? min(lim0 - tokbase, nv) : 0, ok ? min(lim1 - tokbase, nv) : 0);
+    if (ok && tokbase + DTOK <= ctx_full) {
+      tq4_chunk<D, VER, true>(st, bq, kc, kn, lut_lane, koff, cS, r, DTOK, DTOK, DTOK);
+    } else {
+      const int nv = ok ? min(ctx - tokbase, DTOK) : 0;
+      tq4_chunk<D, VER, false>(st, bq, kc, kn, lut_lane, koff, cS, r, nv,
+                               ok ? min(lim0 - tokbase, nv) : 0, ok ? min(lim1 - tokbase, nv) : 0);
+    }
     __syncwarp();
     if (it + TQ_STAGES < my_n) {
       fence_proxy_async_smem();
