@@ -77,11 +77,12 @@ template <int NGH>
 struct PairState {
   float m0, m1, l0, l1;
   float O[NGH][4][4];
-  float Bs[4];   // bias term sum_t bias_{t,g} p_t (MMA layout: row = group, col = column)
+  float Bs[NGH][2];   // this thread's positions' share of sum_t bias_{t,g} p_t, columns 2c, 2c+1
   __device__ __forceinline__ void init() {
     m0 = m1 = -INFINITY;
     l0 = l1 = 0.f;
-    Bs[0] = Bs[1] = Bs[2] = Bs[3] = 0.f;
+#pragma unroll
+    for (int g = 0; g < NGH; ++g) Bs[g][0] = Bs[g][1] = 0.f;
 #pragma unroll
     for (int g = 0; g < NGH; ++g)
 #pragma unroll
@@ -222,8 +223,8 @@ __device__ __forceinline__ void pair_softmax_pv(PairState<D / 128> (&st)[NTC],
           un2(mul2(mk2(s.O[g][e][0], s.O[g][e][1]), ff), s.O[g][e][0], s.O[g][e][1]);
           un2(mul2(mk2(s.O[g][e][2], s.O[g][e][3]), ff), s.O[g][e][2], s.O[g][e][3]);
         }
-      un2(mul2(mk2(s.Bs[0], s.Bs[1]), ff), s.Bs[0], s.Bs[1]);
-      un2(mul2(mk2(s.Bs[2], s.Bs[3]), ff), s.Bs[2], s.Bs[3]);
+#pragma unroll
+      for (int g = 0; g < NGH; ++g) un2(mul2(mk2(s.Bs[g][0], s.Bs[g][1]), ff), s.Bs[g][0], s.Bs[g][1]);
       un2(mul2(mk2(s.l0, s.l1), ff), s.l0, s.l1);
       s.m0 = nm0;
       s.m1 = nm1;
@@ -262,32 +263,21 @@ __device__ __forceinline__ void pair_softmax_pv(PairState<D / 128> (&st)[NTC],
       va = ta < nvalid;
       vb = tb < nvalid;
     }
-    // bias term: A rows = groups (only this warp's), k-slots = positions
-    // 2c, 2c+1, 2c+8, 2c+9
-    {
-      uint32_t a0 = 0, a2 = 0;
-      if (r >= cc.h * NGH && r < cc.h * NGH + NGH) {
-        const uint8_t* base = vsb + (16 * j + 2 * cc.c) * SBB + r * 4;
-        uint32_t x0 = *reinterpret_cast<const uint32_t*>(base);
-        uint32_t x1 = *reinterpret_cast<const uint32_t*>(base + SBB);
-        uint32_t x2 = *reinterpret_cast<const uint32_t*>(base + 8 * SBB);
-        uint32_t x3 = *reinterpret_cast<const uint32_t*>(base + 9 * SBB);
-        if constexpr (!FULL) {
-          const int t0 = 16 * j + 2 * cc.c;
-          if (t0 >= nvalid) x0 = 0;
-          if (t0 + 1 >= nvalid) x1 = 0;
-          if (t0 + 8 >= nvalid) x2 = 0;
-          if (t0 + 9 >= nvalid) x3 = 0;
-        }
-        a0 = hi_halves(x0, x1);
-        a2 = hi_halves(x2, x3);
-      }
+    // bias term sum_t bias_{t,g} p_t in fp32: this thread's positions ta, tb
+    // (summed over the lanes of a column at the end)
 #pragma unroll
-      for (int t = 0; t < NTC; ++t) {
-        const uint32_t pb0 = movm_t(pack_bf16x2(p[t][j][0], p[t][j][1]));
-        const uint32_t pb1 = movm_t(pack_bf16x2(p[t][j][2], p[t][j][3]));
-        mma_bf16(st[t].Bs, a0, 0u, a2, 0u, pb0, pb1);
+    for (int gg = 0; gg < NGH; ++gg) {
+      float ba = bf16hi_to_f32(wa[gg]), bb = bf16hi_to_f32(wb[gg]);
+      if constexpr (!FULL) {
+        if (!va) ba = 0.f;
+        if (!vb) bb = 0.f;
       }
+      const f2 ba2 = mk2(ba, ba), bb2 = mk2(bb, bb);
+#pragma unroll
+      for (int t = 0; t < NTC; ++t)
+        un2(fma2(bb2, mk2(p[t][j][2], p[t][j][3]),
+                 fma2(ba2, mk2(p[t][j][0], p[t][j][1]), mk2(st[t].Bs[gg][0], st[t].Bs[gg][1]))),
+            st[t].Bs[gg][0], st[t].Bs[gg][1]);
     }
 #pragma unroll
     for (int gg = 0; gg < NGH; ++gg) {
@@ -670,12 +660,17 @@ verify_pair_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a)
       l0 += __shfl_xor_sync(0xffffffffu, l0, o);
       l1 += __shfl_xor_sync(0xffffffffu, l1, o);
     }
-    // bias sums: lane (r = g, c) of the MMA accumulator holds group g
+    // bias sums over the 8 lanes of each column pair
     float Bs[NGH][2];
 #pragma unroll
     for (int gg = 0; gg < NGH; ++gg) {
-      Bs[gg][0] = __shfl_sync(0xffffffffu, st[t].Bs[0], (h * NGH + gg) * 4 + c);
-      Bs[gg][1] = __shfl_sync(0xffffffffu, st[t].Bs[1], (h * NGH + gg) * 4 + c);
+      Bs[gg][0] = st[t].Bs[gg][0];
+      Bs[gg][1] = st[t].Bs[gg][1];
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        Bs[gg][0] += __shfl_xor_sync(0xffffffffu, Bs[gg][0], o);
+        Bs[gg][1] += __shfl_xor_sync(0xffffffffu, Bs[gg][1], o);
+      }
     }
 #pragma unroll
     for (int gg = 0; gg < NGH; ++gg) {
