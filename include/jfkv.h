@@ -201,7 +201,8 @@ int jf_kv_quantize_append(const jf_kv_pool* pool, const int32_t* page_table, int
  * accumulation (q is rescaled by a power of two per KV head when max|q| >= 2^14,
  * so any finite bf16 q is accepted); the softmax runs in fp32 with the
  * maximum subtracted; probabilities scaled by the V group scale enter fp16
- * products, so V group scales must stay below 65504.  Output rounded RNE.
+ * products, so V group scales must stay below 65504; the V bias term
+ * sum_t bias_t p_t is accumulated in fp32.  Output rounded RNE.
  * TQ4 pools (pool->tq4 required): the query is rotated once, q' = H S_K q /
  * sqrt(D), and scaled by a power of two into the fp16 range; indices meet
  * fp16 centroids in fp16 tensor-core products with fp32 accumulation, scores

@@ -23,7 +23,8 @@
 //  * PV: A = V codes transposed [16 d x 16 positions] (ldmatrix.trans gives the
 //    position pairs), B = p_t * scale_{t,g} as f16 [16 positions x 8 heads]
 //    (the QK accumulator transposed with movmatrix); the bias term
-//    sum_t bias_{t,g} p_t is one more bf16 MMA.
+//    sum_t bias_{t,g} p_t is accumulated in fp32 by each thread over its own
+//    positions and summed over the lanes of a head pair at the end.
 //  * Online softmax in the log2 domain.  The reference maximum moves only when
 //    a logit exceeds it by more than 2^DTAU, so the common chunk needs no
 //    cross-lane reduction; the accumulators are rescaled only then.
@@ -78,11 +79,12 @@ template <int NG>
 struct DecodeState {
   float m0, m1, l0, l1;
   float O[NG][4][4];
-  float Bs[4];   // bias term sum_t bias_{t,g} p_t (MMA layout: row = group, col = head)
+  float Bs[NG][2];   // this thread's positions' share of sum_t bias_{t,g} p_t, heads 2c, 2c+1
   __device__ __forceinline__ void init() {
     m0 = m1 = -INFINITY;
     l0 = l1 = 0.f;
-    Bs[0] = Bs[1] = Bs[2] = Bs[3] = 0.f;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) Bs[g][0] = Bs[g][1] = 0.f;
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
 #pragma unroll
@@ -202,8 +204,11 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
         st.O[g][e][1] *= f1; st.O[g][e][3] *= f1;
       }
     }
-    st.Bs[0] *= f0; st.Bs[2] *= f0;
-    st.Bs[1] *= f1; st.Bs[3] *= f1;
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      st.Bs[g][0] *= f0;
+      st.Bs[g][1] *= f1;
+    }
     st.l0 *= f0;
     st.l1 *= f1;
     st.m0 = nm0;
@@ -245,28 +250,18 @@ __device__ __forceinline__ void process_chunk(DecodeState<D / 64>& st, const Chu
       va = ta < nvalid;
       vb = tb < nvalid;
     }
-    // bias term: A rows = groups (r < NG), k-slots = positions 2c, 2c+1, 2c+8, 2c+9
-    {
-      uint32_t a0 = 0, a2 = 0;
-      if (r < NG) {
-        const uint8_t* base = vsb + (16 * j + 2 * cc.c) * SBB + r * 4;
-        uint32_t x0 = *reinterpret_cast<const uint32_t*>(base);
-        uint32_t x1 = *reinterpret_cast<const uint32_t*>(base + SBB);
-        uint32_t x2 = *reinterpret_cast<const uint32_t*>(base + 8 * SBB);
-        uint32_t x3 = *reinterpret_cast<const uint32_t*>(base + 9 * SBB);
-        if constexpr (!FULL) {
-          const int t0 = 16 * j + 2 * cc.c;
-          if (t0 >= nvalid) x0 = 0;
-          if (t0 + 1 >= nvalid) x1 = 0;
-          if (t0 + 8 >= nvalid) x2 = 0;
-          if (t0 + 9 >= nvalid) x3 = 0;
-        }
-        a0 = hi_halves(x0, x1);
-        a2 = hi_halves(x2, x3);
+    // bias term sum_t bias_{t,g} p_t in fp32: this thread's positions ta, tb
+    // (summed over the lanes of a head pair at the end)
+#pragma unroll
+    for (int g = 0; g < NG; ++g) {
+      float ba = bf16hi_to_f32(wa[g]), bb = bf16hi_to_f32(wb[g]);
+      if constexpr (!FULL) {
+        if (!va) ba = 0.f;
+        if (!vb) bb = 0.f;
       }
-      const uint32_t pb0 = movm_t(pack_bf16x2(p[j][0], p[j][1]));
-      const uint32_t pb1 = movm_t(pack_bf16x2(p[j][2], p[j][3]));
-      mma_bf16(st.Bs, a0, 0u, a2, 0u, pb0, pb1);
+      un2(fma2(mk2(bb, bb), mk2(p[j][2], p[j][3]),
+               fma2(mk2(ba, ba), mk2(p[j][0], p[j][1]), mk2(st.Bs[g][0], st.Bs[g][1]))),
+          st.Bs[g][0], st.Bs[g][1]);
     }
 #pragma unroll
     for (int g = 0; g < NG; ++g) {
@@ -624,12 +619,17 @@ decode_split_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a
     l0 += __shfl_xor_sync(0xffffffffu, l0, o);
     l1 += __shfl_xor_sync(0xffffffffu, l1, o);
   }
-  // bias sums: lane (r = g, c) of the MMA accumulator holds group g, heads 2c, 2c+1
+  // bias sums over the 8 lanes of each head pair
   float Bs[NG][2];
 #pragma unroll
   for (int g = 0; g < NG; ++g) {
-    Bs[g][0] = __shfl_sync(0xffffffffu, st.Bs[0], g * 4 + c);
-    Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
+    Bs[g][0] = st.Bs[g][0];
+    Bs[g][1] = st.Bs[g][1];
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+      Bs[g][0] += __shfl_xor_sync(0xffffffffu, Bs[g][0], o);
+      Bs[g][1] += __shfl_xor_sync(0xffffffffu, Bs[g][1], o);
+    }
   }
   // This warp's ring is idle now (each of its copies has landed and been
   // read), so its O rows (padded by 4 floats: the 128-bit stores of one
@@ -1011,12 +1011,17 @@ decode_span_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a)
       l0 += __shfl_xor_sync(0xffffffffu, l0, o);
       l1 += __shfl_xor_sync(0xffffffffu, l1, o);
     }
-    // bias sums: lane (r = g, c) of the MMA accumulator holds group g, heads 2c, 2c+1
+    // bias sums over the 8 lanes of each head pair
     float Bs[NG][2];
   #pragma unroll
     for (int g = 0; g < NG; ++g) {
-      Bs[g][0] = __shfl_sync(0xffffffffu, st.Bs[0], g * 4 + c);
-      Bs[g][1] = __shfl_sync(0xffffffffu, st.Bs[1], g * 4 + c);
+      Bs[g][0] = st.Bs[g][0];
+      Bs[g][1] = st.Bs[g][1];
+  #pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        Bs[g][0] += __shfl_xor_sync(0xffffffffu, Bs[g][0], o);
+        Bs[g][1] += __shfl_xor_sync(0xffffffffu, Bs[g][1], o);
+      }
     }
     // This warp's ring is idle now (each of its copies has landed and been
     // read), so its O rows (padded by 4 floats: the 128-bit stores of one
