@@ -286,6 +286,29 @@ def test_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("Hq,Hkv,D,L,splits", [(24, 4, 256, 4, 5), (24, 4, 256, 2, 3),
+                                                (12, 2, 128, 3, 1)])
+def test_verifier_warp_pairs_are_deterministic(Hq, Hkv, D, L, splits):
+    """The two warps of a pair swap partial logits through double-buffered
+    shared memory once per chunk: repeated calls on the same inputs give the
+    same bits (a buffer reused too early would show up as run-to-run noise)."""
+    from paper_2609_17475_gb300 import synth
+    case = make_case(4242 + L, Hq, Hkv, D, 64, [7000, 3001])
+    pool = pool_from_numpy(case, case.oracle_pool())
+    q = synth.normal_bf16(synth.generator(4343 + L), (2, L, Hq, D)).to(DEV)
+    ws = jf.verify_workspace(2, L, Hq, Hkv, D, splits, device=DEV)
+    ctx = torch.tensor(case.ctx, dtype=torch.int32, device=DEV)
+    outs = []
+    for _ in range(3):
+        out = torch.empty(2, L, Hq, D, dtype=torch.bfloat16, device=DEV)
+        jf.jf_paged_verify_attn(pool, case.page_table.to(DEV), ctx, q, 1 / math.sqrt(D), out, ws,
+                                splits)
+        outs.append(out)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
 def test_verifier_with_one_token_is_decode():
     case = make_case(77, 24, 4, 256, 256, [3333, 1234])
     pool = pool_from_numpy(case, case.oracle_pool())

@@ -308,6 +308,25 @@ def test_tq4_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
     assert_attention_close(out, ref)
 
 
+def test_tq4_verifier_warp_pairs_are_deterministic():
+    """Repeated TQ4 verifier calls on the same inputs give the same bits (the
+    warp pairs' per-chunk exchange of partial dot products)."""
+    case = make_case(4444, 24, 4, 256, 64, [6000, 2500])
+    _, ref_pool = oracle_pool(case)
+    pool = pool_from_numpy(case, ref_pool)
+    q = synth.normal_bf16(synth.generator(4545), (2, 3, 24, 256)).to(DEV)
+    ws = jf.verify_workspace(2, 3, 24, 4, 256, 4, device=DEV)
+    ctx = torch.tensor(case.ctx, dtype=torch.int32, device=DEV)
+    outs = []
+    for _ in range(3):
+        out = torch.empty(2, 3, 24, 256, dtype=torch.bfloat16, device=DEV)
+        jf.jf_paged_verify_attn(pool, case.page_table.to(DEV), ctx, q, 1 / 16, out, ws, 4)
+        outs.append(out)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+
+
 def test_tq4_verifier_with_one_token_is_decode():
     case = make_case(78, 24, 4, 256, 256, [3333, 1234])
     _, ref_pool = oracle_pool(case)
