@@ -286,6 +286,37 @@ def test_verifier_matches_oracle(Hq, Hkv, D, P, ctx, L, splits):
     assert_attention_close(out, ref)
 
 
+@pytest.mark.parametrize("splits", [1, 3])
+def test_verifier_context_shorter_than_q_len(splits):
+    """A request whose context is shorter than q_len: token i sees positions
+    < ctx - q_len + 1 + i, so the first tokens see nothing and their rows are
+    zero (the oracle's softmax over an empty set is undefined, NaN); the
+    others match the oracle.  Warp-pair kernel (24 rows per KV head)."""
+    from paper_2609_17475_gb300 import synth
+    Hq, Hkv, D, P, L = 24, 4, 256, 64, 4
+    case = make_case(5151 + splits, Hq, Hkv, D, P, [2, 900])
+    ref_pool = case.oracle_pool()
+    pool = pool_from_numpy(case, ref_pool)
+    q = synth.normal_bf16(synth.generator(5252), (2, L, Hq, D))
+    ws = jf.verify_workspace(2, L, Hq, Hkv, D, splits, device=DEV)
+    out = torch.full((2, L, Hq, D), float("nan"), dtype=torch.bfloat16, device=DEV)
+    scale = 1 / math.sqrt(D)
+    jf.jf_paged_verify_attn(pool, case.page_table.to(DEV),
+                            torch.tensor(case.ctx, dtype=torch.int32, device=DEV), q.to(DEV),
+                            scale, out, ws, splits)
+    torch.cuda.synchronize()
+    assert jf.workspace_status(ws) == 0
+    got = out.float().cpu()
+    assert (got[0, :2] == 0).all()                       # tokens 0, 1 of the 2-position request
+    with np.errstate(invalid="ignore"):   # the rows of tokens 0, 1 are NaN in the oracle
+        ref0 = OT.prefill_chunk(ref_pool, case.layout, case.page_table[0].numpy(), bits(q[0]),
+                                2 - L, scale)
+    assert_attention_close(out[0, 2:], ref0[2:])
+    ref1 = OT.prefill_chunk(ref_pool, case.layout, case.page_table[1].numpy(), bits(q[1]),
+                            900 - L, scale)
+    assert_attention_close(out[1], ref1)
+
+
 @pytest.mark.parametrize("Hq,Hkv,D,L,splits", [(24, 4, 256, 4, 5), (24, 4, 256, 2, 3),
                                                 (12, 2, 128, 3, 1)])
 def test_verifier_warp_pairs_are_deterministic(Hq, Hkv, D, L, splits):
