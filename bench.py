@@ -238,7 +238,7 @@ def run_ours(args, world, rank, local):
     clocks = clk.summary()
 
     # ---- the same step over a region of at least one second (more graph
-    # replays), so that run-to-run spread can be judged on a longer window
+    # replays), so that run-to-run spread can be assessed on a longer window
     n_long = max(args.steps, int(math.ceil(1000.0 / max(ms / args.steps, 1e-3))))
     with ClockSampler(local) as clk_long:
         with torch.cuda.stream(stream):
