@@ -1132,13 +1132,16 @@ decode_span_kernel(const __grid_constant__ CUtensorMap tmap, const DecodeArgs a)
   while (pos < end) {
     const SpanHit h = span_find(a, pos, lane);
     if (h.b < 0) break;
-    const int c0 = (int)(pos - h.start);
-    const int c1 = (int)(min(end, h.start + h.nch) - h.start);
-    const int ctx = checked_ctx(a, h.b, c0);
+    // offsets in the request's sequence range: its first SPAN_HDR places stand
+    // for the segment setup, then come its chunks
+    const int v0 = (int)(pos - h.start);
+    const int v1 = (int)(min(end, h.start + h.nch) - h.start);
+    const int c0 = max(v0 - SPAN_HDR, 0), c1 = max(v1 - SPAN_HDR, 0);
+    const int ctx = checked_ctx(a, h.b, v0);
     if (!run_split(h.b, ctx, c0, c1, ((int64_t)blockIdx.x + h.b) * a.HqL, 1, false,
-                   c1 == h.nch))
+                   v1 == h.nch))
       return;   // a bounded wait gave up (reported); the CTA stops
-    pos = h.start + c1;
+    pos = h.start + v1;
   }
 }
 

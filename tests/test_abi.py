@@ -271,26 +271,33 @@ def test_nvtx_ranges_wrap_every_enqueueing_call_when_enabled():
     assert off.stdout.split() == ["False", "False"], off.stderr
 
 
-def _span_segments(ctx, budget, dtok=32, min_cps=16):
+SPAN_HDR = 32   # decode.cuh: places standing for a segment's start
+
+
+def _span_segments(ctx, budget, dtok=32, min_cps=16, hdr=SPAN_HDR):
     """The span plan's segments as the decode kernels work them out
-    (decode.cuh: span_width, span_find, span_rows): requests' chunks laid end
-    to end, pieces of W chunks, segment (piece x, request b) -> row x + b."""
+    (decode.cuh: span_nch, span_width, span_find, span_rows): each request a
+    run of hdr places then its chunks, the runs laid end to end, pieces of W
+    places, segment (piece x, request b) -> row x + b and real chunks
+    [max(v0 - hdr, 0), max(v1 - hdr, 0))."""
     nch = [(max(0, c) + dtok - 1) // dtok for c in ctx]
-    T = sum(nch)
+    run = [n + hdr if n else 0 for n in nch]
+    T = sum(run)
     W = max(min_cps, -(-T // max(budget, 1)))
-    starts = [sum(nch[:b]) for b in range(len(nch))]
+    starts = [sum(run[:b]) for b in range(len(run))]
     segs = []
     for x in range(budget):
         pos, end = x * W, min((x + 1) * W, T)
         while pos < end:
-            b = next(b for b in range(len(nch)) if nch[b] and starts[b] <= pos < starts[b] + nch[b])
-            c1 = min(end, starts[b] + nch[b]) - starts[b]
-            segs.append((x, b, pos - starts[b], c1))
-            pos = starts[b] + c1
+            b = next(b for b in range(len(run)) if run[b] and starts[b] <= pos < starts[b] + run[b])
+            v1 = min(end, starts[b] + run[b]) - starts[b]
+            v0 = pos - starts[b]
+            segs.append((x, b, max(v0 - hdr, 0), max(v1 - hdr, 0), v1 - v0))
+            pos = starts[b] + v1
     merge = {}
-    for b in range(len(nch)):
-        if nch[b]:
-            x0, x1 = starts[b] // W, (starts[b] + nch[b] - 1) // W
+    for b in range(len(run)):
+        if run[b]:
+            x0, x1 = starts[b] // W, (starts[b] + run[b] - 1) // W
             merge[b] = (x0 + b, x1 - x0 + 1)
     return nch, W, segs, merge
 
@@ -309,21 +316,22 @@ def test_span_plan_rows_are_unique_contiguous_and_inside_the_workspace(seed):
     slots = 38
     budget = min(slots, B * (num_splits - 1) + 1)
     nch, W, segs, merge = _span_segments(ctx, budget)
-    rows = [x + b for (x, b, c0, c1) in segs]
+    rows = [x + b for (x, b, c0, c1, _) in segs]
     assert len(rows) == len(set(rows))
     assert max(rows, default=0) < B * num_splits
     for b in range(B):
-        mine = sorted((c0, c1, x + b) for (x, bb, c0, c1) in segs if bb == b)
+        mine = sorted((c0, c1, x + b) for (x, bb, c0, c1, _) in segs if bb == b)
         covered = [c for c0, c1, _ in mine for c in range(c0, c1)]
         assert covered == list(range(nch[b]))
         if nch[b]:
             first, n = merge[b]
-            assert [r for _, _, r in mine] == list(range(first, first + n))
+            assert sorted(r for _, _, r in mine) == list(range(first, first + n))
         else:
             assert b not in merge
-    # the pieces carry equal work: every piece but the last holds exactly W chunks
+    # the pieces carry equal work: every piece but the last holds exactly W
+    # places (a request's start counts SPAN_HDR places before its chunks)
     per_piece = {}
-    for (x, b, c0, c1) in segs:
-        per_piece[x] = per_piece.get(x, 0) + (c1 - c0)
+    for (x, b, c0, c1, places) in segs:
+        per_piece[x] = per_piece.get(x, 0) + places
     full = [per_piece[x] for x in sorted(per_piece)][:-1]
     assert all(w == W for w in full)
